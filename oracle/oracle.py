@@ -1,0 +1,187 @@
+"""ctypes front end of the C oracle (oracle/vsd_oracle.c).
+
+TEST INFRASTRUCTURE ONLY: the tests, the smoke check and the benchmark's
+CPU-baseline leg call this module; the library under test never does.  It
+takes numpy arrays, widens logits to float32 (bf16 values are exact in f32)
+and returns float64/int results.  Each function cites the passage of the paper
+(arxiv 2602.05774) it restates; see vsd_oracle.c for the readings R1..R10.
+"""
+import ctypes as C
+import numpy as np
+
+from .build import build_oracle
+
+_lib = None
+
+
+class _LinearIn(C.Structure):
+    _fields_ = [
+        ("draft", C.c_void_p), ("target", C.c_void_p),
+        ("B", C.c_int32), ("K", C.c_int32), ("D", C.c_int32),
+        ("V", C.c_int64), ("T", C.c_double),
+        ("u_draft", C.c_void_p), ("u_accept", C.c_void_p), ("u_correct", C.c_void_p),
+        ("ref_logkappa", C.c_void_p),
+        ("w_base", C.c_double), ("tau_car", C.c_double), ("zeta_mode", C.c_int32),
+    ]
+
+
+class _LinearOut(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in (
+        "tokens", "logq_tok", "alpha", "accept", "accept_len", "corr_tokens",
+        "logq_corr", "alpha_corr", "logkappa", "logkappa_corr", "logkappa_ref",
+        "ref_tokens", "expected_len", "row_lse", "weights", "loss", "grad", "margins")]
+
+
+class _TreeIn(C.Structure):
+    _fields_ = [
+        ("draft", C.c_void_p), ("target", C.c_void_p),
+        ("B", C.c_int32), ("N", C.c_int32), ("V", C.c_int64), ("T", C.c_double),
+        ("parent", C.c_void_p), ("tokens", C.c_void_p),
+        ("u_accept", C.c_void_p), ("u_correct", C.c_void_p),
+    ]
+
+
+class _TreeOut(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in (
+        "alpha", "accept", "path_accept", "logkappa", "corr_tokens", "deepest",
+        "accept_len", "bonus", "margins")]
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _lib = C.CDLL(build_oracle())
+        _lib.vso_linear.argtypes = [C.POINTER(_LinearIn), C.POINTER(_LinearOut)]
+        _lib.vso_linear.restype = C.c_int
+        _lib.vso_tree.argtypes = [C.POINTER(_TreeIn), C.POINTER(_TreeOut)]
+        _lib.vso_tree.restype = C.c_int
+        _lib.vso_log_softmax.argtypes = [C.c_void_p, C.c_int64, C.c_double, C.c_void_p]
+        _lib.vso_log_softmax.restype = C.c_double
+        _lib.vso_sample.argtypes = [C.c_void_p, C.c_int64, C.c_double, C.c_void_p]
+        _lib.vso_sample.restype = C.c_int64
+        _lib.vso_prefix_weights.argtypes = [
+            C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+            C.c_double, C.c_double, C.c_int, C.c_void_p]
+        _lib.vso_prefix_weights.restype = C.c_double
+        _lib.vso_prefix_objective.argtypes = [
+            C.c_void_p, C.c_int, C.c_int, C.c_int64, C.c_double, C.c_void_p, C.c_void_p,
+            C.c_void_p, C.c_double, C.c_int, C.c_void_p]
+        _lib.vso_prefix_objective.restype = C.c_double
+    return _lib
+
+
+def _f32(a):
+    return np.ascontiguousarray(np.asarray(a, dtype=np.float32))
+
+
+def _i32(a):
+    return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data
+
+
+def log_softmax(x, T=1.0):
+    """Eq. 1's distributions: log softmax(x / T) of one row, float64."""
+    x = _f32(x).reshape(-1)
+    out = np.empty(x.size, dtype=np.float64)
+    lib().vso_log_softmax(_ptr(x), x.size, float(T), _ptr(out))
+    return out
+
+
+def sample(prob, u):
+    """Inverse-CDF draw (smallest v with u < F(v)); returns (v, margin)."""
+    prob = np.ascontiguousarray(np.asarray(prob, dtype=np.float64)).reshape(-1)
+    m = np.zeros(1, dtype=np.float64)
+    v = lib().vso_sample(_ptr(prob), prob.size, float(u), _ptr(m))
+    return int(v), float(m[0])
+
+
+def linear(draft, target, T, u_draft, u_accept, u_correct, K, D, ref_logkappa=None,
+           w_base=1.05, tau_car=0.2, zeta_mode=0, want_grad=True):
+    """E-step + M-step over linear paths (Algorithm 1, Algorithm 2, Eqs. 1, 2, 11,
+    beta, zeta, advance).
+
+    draft, target: [B*K*D, V] (any float dtype; widened to f32 exactly).
+    Returns a dict of numpy arrays named as the C-ABI outputs.
+    """
+    draft = _f32(draft)
+    target = _f32(target)
+    V = draft.shape[-1]
+    R = draft.size // V
+    B = R // (K * D)
+    assert B * K * D == R and target.shape == draft.shape
+    ud, ua, uc = _f32(u_draft).reshape(-1), _f32(u_accept).reshape(-1), _f32(u_correct).reshape(-1)
+    assert ud.size == R and ua.size == R and uc.size == R
+    ref = None if ref_logkappa is None else _f32(ref_logkappa).reshape(-1)
+    if ref is not None:
+        assert ref.size == B * D
+    o = dict(
+        tokens=np.zeros(R, np.int32), logq_tok=np.zeros(R), alpha=np.zeros(R),
+        accept=np.zeros(R, np.uint8), accept_len=np.zeros(B * K, np.int32),
+        corr_tokens=np.zeros(R, np.int32), logq_corr=np.zeros(R), alpha_corr=np.zeros(R),
+        logkappa=np.zeros(R), logkappa_corr=np.zeros(R), logkappa_ref=np.zeros(R),
+        ref_tokens=np.zeros(R, np.int32), expected_len=np.zeros(B * K),
+        row_lse=np.zeros((R, 2)), weights=np.zeros((B, D, K, 4)), loss=np.zeros(B + 1),
+        grad=np.zeros((R, V)) if want_grad else None, margins=np.zeros((R, 6)))
+    li = _LinearIn(_ptr(draft), _ptr(target), B, K, D, V, float(T), _ptr(ud), _ptr(ua),
+                   _ptr(uc), _ptr(ref), float(w_base), float(tau_car), int(zeta_mode))
+    lo = _LinearOut(*[_ptr(o[n]) for n, _ in _LinearOut._fields_])
+    rc = lib().vso_linear(C.byref(li), C.byref(lo))
+    if rc != 0:
+        raise ValueError("oracle rejected the arguments (code %d)" % rc)
+    return o
+
+
+def tree(draft, target, T, parent, tokens, u_accept, u_correct):
+    """Verification of a draft tree with parent pointers (App. E tree, Eq. 1 per
+    node, Sec. 3 residual).  draft/target [B*N, V]; parent, tokens, uniforms [B, N]."""
+    draft = _f32(draft)
+    target = _f32(target)
+    parent = _i32(parent)
+    B, N = parent.shape
+    V = draft.shape[-1]
+    assert draft.size == B * N * V and target.shape == draft.shape
+    tokens = _i32(tokens).reshape(B, N)
+    ua, uc = _f32(u_accept).reshape(B, N), _f32(u_correct).reshape(B, N)
+    o = dict(alpha=np.zeros((B, N)), accept=np.zeros((B, N), np.uint8),
+             path_accept=np.zeros((B, N), np.uint8), logkappa=np.zeros((B, N)),
+             corr_tokens=np.zeros((B, N), np.int32), deepest=np.zeros(B, np.int32),
+             accept_len=np.zeros(B, np.int32), bonus=np.zeros(B, np.int32),
+             margins=np.zeros((B, N, 2)))
+    ti = _TreeIn(_ptr(draft), _ptr(target), B, N, V, float(T), _ptr(parent), _ptr(tokens),
+                 _ptr(ua), _ptr(uc))
+    to = _TreeOut(*[_ptr(o[n]) for n, _ in _TreeOut._fields_])
+    rc = lib().vso_tree(C.byref(ti), C.byref(to))
+    if rc != 0:
+        raise ValueError("oracle rejected the tree (code %d)" % rc)
+    return o
+
+
+def prefix_weights(logkappa, logkappa_corr, logkappa_ref, logq_path, w_base=1.05,
+                   tau_car=0.2, zeta_mode=0):
+    """o~, o', beta, zeta of one prefix (Algorithm 1 M-step lines, Eqs. beta and
+    zeta).  Inputs are [K, D] tables; returns ([D, K, 4] weights, N_b)."""
+    lk = np.ascontiguousarray(logkappa, dtype=np.float64)
+    K, D = lk.shape
+    args = [np.ascontiguousarray(a, dtype=np.float64).reshape(K, D)
+            for a in (logkappa_corr, logkappa_ref, logq_path)]
+    w = np.zeros((D, K, 4))
+    N = lib().vso_prefix_weights(K, D, _ptr(lk), _ptr(args[0]), _ptr(args[1]), _ptr(args[2]),
+                                 float(w_base), float(tau_car), int(zeta_mode), _ptr(w))
+    return w, N
+
+
+def prefix_objective(draft, T, tokens, corr_tokens, weights, N, B_total, want_grad=True):
+    """J_b of Eq. advance for one prefix with fixed weights, and the gradient of
+    -(1/B) J_b / N_b with respect to the draft logits.  draft [K, D, V]."""
+    draft = _f32(draft)
+    K, D, V = draft.shape
+    tok = _i32(tokens).reshape(K, D)
+    ctok = _i32(corr_tokens).reshape(K, D)
+    w = np.ascontiguousarray(weights, dtype=np.float64).reshape(D, K, 4)
+    g = np.zeros((K, D, V)) if want_grad else None
+    J = lib().vso_prefix_objective(_ptr(draft), K, D, V, float(T), _ptr(tok), _ptr(ctok),
+                                   _ptr(w), float(N), int(B_total), _ptr(g))
+    return J, g

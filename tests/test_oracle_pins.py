@@ -1,0 +1,440 @@
+"""Pins of the CPU oracle to facts fixed by the paper and by mathematics.
+
+Every test here checks the oracle against something other than itself:
+exact lattice enumerations over the uniforms with dyadic distributions (so the
+expected probabilities are exact), closed forms from Sec. 4.4, special cases
+that reduce to library routines (cross-entropy and its autograd), hand-derived
+worked examples stored under tests/golden/, theorems of Sec. 4.4 checked by
+brute force, and finite differences of the oracle's own objective.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+GOLDEN = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "worked_examples.json")))
+
+Q4 = np.array([1 / 2, 1 / 4, 1 / 8, 1 / 8])
+P_UNI = np.array([1 / 4, 1 / 4, 1 / 4, 1 / 4])
+P_B = np.array([1 / 8, 3 / 8, 1 / 4, 1 / 4])
+
+
+def logits(prob, scale=1.0):
+    return (scale * np.log(np.asarray(prob, dtype=np.float64))).astype(np.float32)
+
+
+def lattice(M):
+    return ((np.arange(M) + 0.5) / M).astype(np.float32)
+
+
+def midpoint(prob, t):
+    """A uniform that the inverse CDF maps to token t (middle of its interval)."""
+    F = np.concatenate([[0.0], np.cumsum(prob)])
+    return np.float32((F[t] + F[t + 1]) / 2)
+
+
+# --------------------------------------------------------------------------
+# Eq. 1 distributions and the inverse-CDF draw
+
+
+def test_log_softmax_closed_forms(oracle):
+    # equal logits -> uniform
+    lp = oracle.log_softmax(np.full(7, 3.25, np.float32), 1.0)
+    assert np.allclose(np.exp(lp), 1 / 7, rtol=0, atol=1e-15)
+    # two tokens: softmax is the logistic function of the gap over T
+    for T in (0.5, 1.0, 2.0):
+        lp = oracle.log_softmax(np.array([0.0, 1.5], np.float32), T)
+        assert abs(np.exp(lp[1]) - 1 / (1 + math.exp(-1.5 / T))) < 1e-15
+    # temperature: logits c*x at T=c equal x at T=1
+    x = np.random.default_rng(0).normal(size=33).astype(np.float32)
+    a = oracle.log_softmax(x * 4, 4.0)
+    b = oracle.log_softmax(x, 1.0)
+    assert np.allclose(a, b, atol=1e-13)
+
+
+def test_inverse_cdf_lattice_is_exact(oracle):
+    M = 64
+    counts = np.zeros(4)
+    for u in lattice(M):
+        v, m = oracle.sample(Q4, u)
+        counts[v] += 1
+        assert m > 0
+    assert np.array_equal(counts / M, Q4)
+
+
+def test_inverse_cdf_boundaries(oracle):
+    # strict u < F(v): a uniform on a boundary goes to the next token
+    assert oracle.sample([0.5, 0.5], 0.5)[0] == 1
+    assert oracle.sample([0.5, 0.5], 0.0)[0] == 0
+    # zero-probability tokens are never drawn
+    assert oracle.sample([0.0, 0.5, 0.0, 0.5], 0.0)[0] == 1
+    assert oracle.sample([0.0, 0.5, 0.0, 0.5], 0.5)[0] == 3
+    # rounding that leaves no crossing picks the last token with mass
+    assert oracle.sample([0.25, 0.25, 0.0], 0.75)[0] == 1
+
+
+# --------------------------------------------------------------------------
+# Sec. 3: the accept/resample mixture reproduces the target distribution
+
+
+@pytest.mark.parametrize("T", [1.0, 2.0])
+def test_mixture_reproduces_target_exactly(oracle, T):
+    M = 16
+    ud, ua, uc = np.meshgrid(lattice(M), lattice(M), lattice(M), indexing="ij")
+    B = M ** 3
+    draft = np.tile(logits(Q4, T), (B, 1))
+    target = np.tile(logits(P_UNI, T), (B, 1))
+    o = oracle.linear(draft, target, T, ud.ravel(), ua.ravel(), uc.ravel(), K=1, D=1,
+                      want_grad=False)
+    out = o["corr_tokens"]
+    hist = np.bincount(out, minlength=4) / B
+    assert np.array_equal(hist, P_UNI)
+    # acceptance rate sum_v min(p, q)
+    assert o["accept"].mean() == np.minimum(P_UNI, Q4).sum()
+    # a residual token always has p > q, so its alpha is 1
+    rej = o["accept"] == 0
+    assert np.all(o["alpha_corr"][rej] == 1.0)
+    assert set(np.unique(out[rej])) <= {2, 3}
+
+
+def test_mixture_random_distributions(oracle):
+    """Non-dyadic p, q: lattice histogram within the lattice's resolution of p."""
+    rng = np.random.default_rng(5)
+    V = 6
+    xq = rng.normal(0, 1.5, V).astype(np.float32)
+    xp = rng.normal(0, 1.5, V).astype(np.float32)
+    M = 40
+    ud, ua, uc = np.meshgrid(lattice(M), lattice(M), lattice(M), indexing="ij")
+    B = M ** 3
+    o = oracle.linear(np.tile(xq, (B, 1)), np.tile(xp, (B, 1)), 1.0, ud.ravel(), ua.ravel(),
+                      uc.ravel(), K=1, D=1, want_grad=False)
+    hist = np.bincount(o["corr_tokens"], minlength=V) / B
+    p = np.exp(xp - xp.max()) / np.exp(xp - xp.max()).sum()
+    assert np.abs(hist - p).max() < 4.0 / M
+
+
+# --------------------------------------------------------------------------
+# Sec. 4.4: survival S_k and the expected accepted length
+
+
+def _three_step_rows():
+    rows_q = [Q4, Q4, P_UNI]
+    rows_p = [P_UNI, P_B, P_B]
+    toks = [0, 0, 1]  # alphas 1/2, 1/4, 1
+    return rows_q, rows_p, toks
+
+
+def test_survival_and_expected_length(oracle):
+    g = GOLDEN["expected_length_three_steps"]
+    rows_q, rows_p, toks = _three_step_rows()
+    M = 16
+    a0, a1, a2 = np.meshgrid(lattice(M), lattice(M), lattice(M), indexing="ij")
+    B = M ** 3
+    draft = np.tile(np.stack([logits(r) for r in rows_q]), (B, 1))
+    target = np.tile(np.stack([logits(r) for r in rows_p]), (B, 1))
+    ud = np.tile([midpoint(rows_q[d], toks[d]) for d in range(3)], B)
+    ua = np.stack([a0.ravel(), a1.ravel(), a2.ravel()], 1).ravel()
+    uc = np.full(B * 3, 0.5, np.float32)
+    o = oracle.linear(draft, target, 1.0, ud, ua, uc, K=1, D=3, want_grad=False)
+    assert np.array_equal(o["tokens"].reshape(B, 3)[0], toks)
+    A = o["accept_len"]
+    for k in range(1, 4):
+        assert np.mean(A >= k) == g["survival"][k - 1]
+    assert np.mean(A) == g["expected_length"]
+    assert np.allclose(o["expected_len"], g["expected_length"], atol=1e-14)
+    assert np.allclose(np.exp(o["logkappa"].reshape(B, 3)), g["survival"], atol=1e-14)
+
+
+def test_correction_after_first_rejection_samples_p(oracle):
+    """Reading R3: residual at the first rejection, then p-samples."""
+    M = 16
+    c0, c1 = np.meshgrid(lattice(M), lattice(M), indexing="ij")
+    B = M * M
+    draft = np.tile(np.stack([logits(Q4), logits(Q4)]), (B, 1))
+    target = np.tile(np.stack([logits(P_UNI), logits(P_B)]), (B, 1))
+    ud = np.tile([midpoint(Q4, 0), midpoint(Q4, 0)], B)
+    ua = np.full(2 * B, 0.99, np.float32)  # alpha_0 = 1/2 -> rejected, A = 0
+    uc = np.stack([c0.ravel(), c1.ravel()], 1).ravel()
+    o = oracle.linear(draft, target, 1.0, ud, ua, uc, K=1, D=2, want_grad=False)
+    assert np.all(o["accept_len"] == 0)
+    z = o["corr_tokens"].reshape(B, 2)
+    assert np.array_equal(np.bincount(z[:, 0], minlength=4) / B, [0, 0, 0.5, 0.5])
+    assert np.array_equal(np.bincount(z[:, 1], minlength=4) / B, P_B)
+
+
+def test_accept_tie_and_full_acceptance(oracle):
+    """u = alpha accepts (Eq. 1 text 'r <= alpha'); A = D keeps z' = z~."""
+    rng = np.random.default_rng(1)
+    K, D, V = 2, 3, 9
+    x = rng.normal(0, 2, (K * D, V)).astype(np.float32)
+    o = oracle.linear(x, x, 1.0, rng.random(K * D), np.ones(K * D), rng.random(K * D),
+                      K=K, D=D, want_grad=False)
+    assert np.all(o["alpha"] == 1.0) and np.all(o["accept"] == 1)
+    assert np.all(o["accept_len"] == D)
+    assert np.array_equal(o["corr_tokens"], o["tokens"])
+    assert np.allclose(o["expected_len"], D)
+
+
+def test_greedy_reference_tokens(oracle):
+    """Algorithm 2 reference: argmax of the target row, lowest index on ties."""
+    V = 8
+    target = np.array([[0, 3, 1, 3, -2, 3, 0, 1]], np.float32)
+    draft = np.zeros((1, V), np.float32)
+    o = oracle.linear(draft, target, 1.0, [0.3], [0.3], [0.3], K=1, D=1, want_grad=False)
+    assert o["ref_tokens"][0] == 1
+    p = np.exp(target[0] - target[0].max()); p /= p.sum()
+    assert abs(o["logkappa_ref"][0] - math.log(min(1.0, p[1] / (1 / V)))) < 1e-14
+
+
+# --------------------------------------------------------------------------
+# M-step special cases
+
+
+def _ce_weighted(draft, T, tokens, weights):
+    """Library cross-entropy with per-row weights, and its autograd."""
+    torch = pytest.importorskip("torch")
+    import torch.nn.functional as F
+    x = torch.tensor(draft, dtype=torch.float64, requires_grad=True)
+    ce = F.cross_entropy(x / T, torch.tensor(tokens, dtype=torch.int64), reduction="none")
+    loss = (torch.tensor(weights, dtype=torch.float64) * ce).sum()
+    loss.backward()
+    return loss.item(), x.grad.numpy()
+
+
+@pytest.mark.parametrize("D,T", [(1, 1.0), (4, 0.7)])
+def test_single_proposal_is_weighted_cross_entropy(oracle, D, T):
+    """K = 1: beta = 0 (empty leave-one-out sum), so Eq. advance reduces to the
+    basic gradient (Eq. basic), a w(l)-weighted cross-entropy of the kept path."""
+    rng = np.random.default_rng(2)
+    B, V = 3, 11
+    R = B * D
+    draft = rng.normal(0, 2, (R, V)).astype(np.float32)
+    target = (draft + rng.normal(0, 0.5, (R, V))).astype(np.float32)
+    ref = np.full(B * D, -1e30, np.float32)  # every proposal passes the oracle
+    o = oracle.linear(draft, target, T, rng.random(R), rng.random(R), rng.random(R), K=1, D=D,
+                      ref_logkappa=ref)
+    w = o["weights"]
+    assert np.all(w[..., 0] == 1.0) and np.all(w[..., 2] == 0.0)
+    wl = 1.05 ** np.arange(1, D + 1)
+    assert np.allclose(w[:, :, 0, 1], wl)
+    # row d of path is counted by every l >= d
+    row_w = np.array([wl[d:].sum() for d in range(D)]) / wl.sum()
+    loss, grad = _ce_weighted(draft, T, o["tokens"], np.tile(row_w, B) / B)
+    assert abs(o["loss"][B] - loss) < 1e-12
+    assert np.allclose(o["grad"], grad, atol=1e-14)
+
+
+def test_draft_equals_target_closed_form(oracle):
+    """draft == target: alpha = 1, o~ = 1, o' = w(l), beta = 1 (Sec. 4.3 'automatic
+    early stopping'); with tau -> infinity zeta = 1/K, and the loss is the
+    cross-entropy of z~ weighted by w(l)(1 - 1/K) / N_b."""
+    rng = np.random.default_rng(3)
+    B, K, D, V = 2, 3, 4, 13
+    R = B * K * D
+    x = rng.normal(0, 2, (R, V)).astype(np.float32)
+    o = oracle.linear(x, x, 1.0, rng.random(R), rng.random(R), rng.random(R), K=K, D=D,
+                      tau_car=1e30)
+    w = o["weights"]
+    wl = 1.05 ** np.arange(1, D + 1)
+    assert np.all(w[..., 0] == 1.0)
+    assert np.allclose(w[..., 1], wl[None, :, None])
+    assert np.all(w[..., 2] == 1.0)
+    assert np.allclose(w[..., 3], 1.0 / K)
+    N = K * wl.sum()
+    row_w = np.array([wl[d:].sum() for d in range(D)]) * (1 - 1 / K) / N
+    loss, grad = _ce_weighted(x, 1.0, o["tokens"], np.tile(row_w, B * K) / B)
+    assert abs(o["loss"][B] - loss) < 1e-12
+    assert np.allclose(o["grad"], grad, atol=1e-14)
+
+
+def _forced_rows(cases):
+    """Rows for K proposals of depth 1: (q, p, token, u_accept) per proposal."""
+    draft = np.stack([logits(c[0]) for c in cases])
+    target = np.stack([logits(c[1]) for c in cases])
+    ud = np.array([midpoint(c[0], c[2]) for c in cases], np.float32)
+    ua = np.array([c[3] for c in cases], np.float32)
+    return draft, target, ud, ua
+
+
+@pytest.mark.parametrize("name,u1", [("beta_one_rejected", 0.99), ("beta_one_invalid", 0.01)])
+def test_beta_worked_examples(oracle, name, u1):
+    g = GOLDEN[name]
+    cases = [(Q4, Q4, 1, 0.5), (Q4, P_UNI, 0, u1), (P_B, P_B, 2, 0.5)]
+    draft, target, ud, ua = _forced_rows(cases)
+    o = oracle.linear(draft, target, 1.0, ud, ua, np.full(3, 0.5, np.float32), K=3, D=1,
+                      ref_logkappa=np.zeros(1, np.float32))
+    w = o["weights"][0, 0]
+    assert np.array_equal(w[:, 0], g["o_tilde"])
+    assert np.allclose(w[:, 1], g["o_prime"], rtol=0, atol=1e-15)
+    assert np.allclose(w[:, 2], g["beta"], rtol=0, atol=1e-15)
+
+
+@pytest.mark.parametrize("mode,key", [(0, "zeta_prob"), (1, "zeta_logprob")])
+def test_zeta_worked_example(oracle, mode, key):
+    g = GOLDEN["zeta_two_paths"]
+    cases = [(Q4, P_UNI, 0, 0.5), (Q4, P_UNI, 1, 0.5)]  # q(z~) = 1/2, 1/4
+    draft, target, ud, ua = _forced_rows(cases)
+    o = oracle.linear(draft, target, 1.0, ud, ua, np.full(2, 0.5, np.float32), K=2, D=1,
+                      tau_car=0.2, zeta_mode=mode)
+    assert np.allclose(o["weights"][0, 0, :, 3], g[key], rtol=0, atol=1e-7)
+
+
+def test_zeta_uniform_limit(oracle):
+    rng = np.random.default_rng(4)
+    K, D, V = 5, 3, 10
+    R = K * D
+    x = rng.normal(0, 2, (R, V)).astype(np.float32)
+    y = (x + rng.normal(0, 1, (R, V))).astype(np.float32)
+    for mode in (0, 1):
+        o = oracle.linear(x, y, 1.0, rng.random(R), rng.random(R), rng.random(R), K=K, D=D,
+                          tau_car=1e300, zeta_mode=mode, want_grad=False)
+        assert np.allclose(o["weights"][..., 3], 1.0 / K, atol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# Gradient: finite differences of the objective with weights held fixed
+
+
+def test_gradient_finite_differences(oracle):
+    rng = np.random.default_rng(6)
+    B, K, D, V, T = 2, 3, 3, 7, 0.8
+    R = B * K * D
+    # logits on a 2^-8 grid so that x +- h is exact in float32
+    draft = (np.round(rng.normal(0, 1.5, (R, V)) * 256) / 256).astype(np.float32)
+    target = (draft + np.round(rng.normal(0, 1.0, (R, V)) * 256) / 256).astype(np.float32)
+    o = oracle.linear(draft, target, T, rng.random(R), rng.random(R), rng.random(R), K=K, D=D)
+    assert np.allclose(o["grad"].sum(axis=1), 0.0, atol=1e-15)
+    h = 2.0 ** -8
+    for b in range(B):
+        rows = slice(b * K * D, (b + 1) * K * D)
+        wts = o["weights"][b]
+        N = wts[..., 1].sum()
+        tok = o["tokens"][rows]
+        ctok = o["corr_tokens"][rows]
+        x0 = draft[rows].reshape(K, D, V)
+        J, g = oracle.prefix_objective(x0, T, tok, ctok, wts, N, B)
+        assert abs(-J / N / B - o["loss"][b] / B) < 1e-13
+        assert np.allclose(g.reshape(-1, V), o["grad"][rows], atol=1e-15)
+        for (s, d, v) in [(0, 0, 0), (1, 2, 3), (2, 1, 6), (0, 2, tok[2])]:
+            xp, xm = x0.copy(), x0.copy()
+            xp[s, d, v] += h
+            xm[s, d, v] -= h
+            Jp, _ = oracle.prefix_objective(xp, T, tok, ctok, wts, N, B, want_grad=False)
+            Jm, _ = oracle.prefix_objective(xm, T, tok, ctok, wts, N, B, want_grad=False)
+            fd = -(Jp - Jm) / (2 * h) / N / B
+            assert abs(fd - g[s, d, v]) < 1e-5 * max(1.0, abs(g[s, d, v]))
+
+
+def test_reference_input_is_used(oracle):
+    rng = np.random.default_rng(7)
+    B, K, D, V = 2, 2, 3, 6
+    R = B * K * D
+    x = rng.normal(0, 2, (R, V)).astype(np.float32)
+    y = (x + rng.normal(0, 1, (R, V))).astype(np.float32)
+    ref = rng.normal(-1, 0.3, B * D).astype(np.float32)
+    o = oracle.linear(x, y, 1.0, rng.random(R), rng.random(R), rng.random(R), K=K, D=D,
+                      ref_logkappa=ref, want_grad=False)
+    lkr = o["logkappa_ref"].reshape(B, K, D)
+    assert np.allclose(lkr, ref.reshape(B, 1, D))
+    ot = o["weights"][..., 0]  # [B, D, K]
+    lk = o["logkappa"].reshape(B, K, D).transpose(0, 2, 1)
+    assert np.array_equal(ot, (lk >= ref.reshape(B, D, 1)).astype(float))
+
+
+# --------------------------------------------------------------------------
+# Tree verification
+
+
+def test_chain_tree_equals_linear_path(oracle):
+    rng = np.random.default_rng(8)
+    D, V = 6, 12
+    x = rng.normal(0, 2, (D, V)).astype(np.float32)
+    y = (x + rng.normal(0, 1, (D, V))).astype(np.float32)
+    ud, ua, uc = rng.random(D), rng.random(D), rng.random(D)
+    lin = oracle.linear(x, y, 1.0, ud, ua, uc, K=1, D=D, want_grad=False)
+    N = D + 1
+    xt = np.concatenate([x, np.zeros((1, V), np.float32)])
+    yt = np.concatenate([y, np.zeros((1, V), np.float32)])
+    parent = np.arange(-1, N - 1, dtype=np.int32)[None]
+    tokens = np.concatenate([[0], lin["tokens"]])[None]
+    tr = oracle.tree(xt, yt, 1.0, parent, tokens, np.concatenate([[0], ua])[None],
+                     np.concatenate([[0], uc])[None])
+    assert np.allclose(tr["alpha"][0, 1:], lin["alpha"])
+    assert np.allclose(tr["logkappa"][0, 1:], lin["logkappa"])
+    A = lin["accept_len"][0]
+    assert tr["accept_len"][0] == A and tr["deepest"][0] == A
+    if A < D:
+        assert tr["corr_tokens"][0, A + 1] == lin["corr_tokens"][A]
+        assert tr["bonus"][0] == lin["corr_tokens"][A]
+
+
+def test_tree_acceptance_lattice(oracle):
+    """P(node n on an accepted path) = product of alpha along its ancestors."""
+    # root -> {1, 2}; 1 -> {3}; 3 -> {4}
+    parent = np.array([-1, 0, 0, 1, 3], np.int32)
+    N, V = 5, 4
+    rq = [Q4, Q4, P_UNI, Q4, P_UNI]
+    rp = [P_UNI, P_B, P_B, P_UNI, P_UNI]
+    # node tokens drawn at the parent's row: node1 tok0 (alpha 1/2), node2 tok1
+    # (alpha 1), node3 tok0 at row1 (alpha 1/4), node4 tok0 at row3 (alpha 1/2)
+    tok = np.array([0, 0, 1, 0, 0], np.int32)
+    M = 8
+    grids = np.meshgrid(*([lattice(M)] * 4), indexing="ij")
+    B = M ** 4
+    ua = np.zeros((B, N), np.float32)
+    for i in range(4):
+        ua[:, i + 1] = grids[i].ravel()
+    draft = np.tile(np.stack([logits(r) for r in rq]), (B, 1))
+    target = np.tile(np.stack([logits(r) for r in rp]), (B, 1))
+    tr = oracle.tree(draft, target, 1.0, np.tile(parent, (B, 1)), np.tile(tok, (B, 1)), ua,
+                     np.full((B, N), 0.3, np.float32))
+    pa = tr["path_accept"].mean(axis=0)
+    assert np.array_equal(pa, [1, 1 / 2, 1, 1 / 8, 1 / 16])
+    # deepest: node 4 (depth 3) when accepted, else 3, else 1 or 2 (lowest index)
+    d = tr["accept_len"]
+    assert np.mean(d == 3) == 1 / 16 and np.mean(d == 2) == 1 / 8 - 1 / 16
+    assert np.all(tr["deepest"][d == 1] == np.where(tr["path_accept"][d == 1, 1] == 1, 1, 2))
+
+
+# --------------------------------------------------------------------------
+# Sec. 4.4 theorems by brute force on a tabulated autoregressive toy model
+
+
+def test_theorems_by_enumeration(oracle):
+    rng = np.random.default_rng(9)
+    V, D = 3, 3
+    import itertools
+    paths = list(itertools.product(range(V), repeat=D))
+    # tabulated conditionals: one (q, p) row per prefix of length 0..D-1
+    tab = {}
+    for d in range(D):
+        for pre in itertools.product(range(V), repeat=d):
+            tab[pre] = (rng.normal(0, 1.5, V).astype(np.float32),
+                        rng.normal(0, 1.5, V).astype(np.float32))
+    sm = lambda x: np.exp(x - x.max()) / np.exp(x - x.max()).sum()
+    draft = np.stack([tab[z[:d]][0] for z in paths for d in range(D)])
+    target = np.stack([tab[z[:d]][1] for z in paths for d in range(D)])
+    ud = np.array([midpoint(sm(tab[z[:d]][0].astype(np.float64)), z[d]) for z in paths
+                   for d in range(D)], np.float32)
+    B = len(paths)
+    o = oracle.linear(draft, target, 1.0, ud, np.full(B * D, 0.5), np.full(B * D, 0.5), K=1,
+                      D=D, want_grad=False)
+    assert np.array_equal(o["tokens"].reshape(B, D), np.array(paths))
+    logk = o["logkappa"].reshape(B, D)[:, -1]
+    lq = o["logq_tok"].reshape(B, D).sum(1)
+    lp_path = np.array([sum(np.log(sm(tab[z[:d]][1].astype(np.float64))[z[d]])
+                            for d in range(D)) for z in paths])
+    q = np.exp(lq)
+    assert abs(q.sum() - 1) < 1e-12
+    elbo = np.sum(q * (logk + lp_path - lq))
+    A = np.sum(q * o["expected_len"])
+    assert A >= D * math.exp(elbo)  # Theorem 1
+    Z = np.sum(np.exp(lp_path) * np.exp(logk))
+    qs = np.exp(lp_path) * np.exp(logk) / Z  # the valid-path posterior, Eq. 4
+    elbo_star = np.sum(qs * (logk + lp_path - np.log(qs)))
+    elbo_kl = np.sum(np.exp(lp_path) * logk)  # q = p
+    assert abs(elbo_star - math.log(Z)) < 1e-12  # Theorem 2, equality
+    assert elbo_star > elbo_kl  # Theorem 2, strict when kappa varies
+    assert elbo <= elbo_star + 1e-12  # the posterior maximises the ELBO
