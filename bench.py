@@ -1,0 +1,351 @@
+"""Benchmark of the fused VSD E-step + M-step (one persistent kernel per step).
+
+Workload (default): vocab128k -- B=32 prefixes x K=16 proposals x D=8 depth,
+V=128256, bf16 draft/target logits (Zipf-shaped target, draft = target +
+N(0, 1.5^2)), temperatures alternating 0.7 / 1.0 between steps, synthetic and
+seeded.  Inputs (2.1 GB) are larger than L2, so no flush is needed between
+steps.  One step = one call of vsd_estep_mstep over the whole batch.
+
+Prints ONE JSON line (rank 0).  `--impl reference` times the CPU oracle (the
+reference implementation of this tier) on a bounded sample of the same
+workload instead.
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = ("draft-logit rows/s and achieved HBM GB/s (fraction of GB300 roofline) for fused "
+          "E/M step")
+WORKLOADS = ("vocab128k", "vocab32k", "tiny")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=("ours", "reference"))
+    ap.add_argument("--config", default="vocab128k", choices=WORKLOADS)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(path))
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2602_05774_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        h.update(open(os.path.join(csrc, f), "rb").read())
+    h.update(open(os.path.join(ROOT, "include", "vsd.h"), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(workload):
+    """DRAM bytes per launch of the fused kernel from the committed ncu summary,
+    if it was taken on the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "k_fused_%s_traffic.json" % workload)
+    try:
+        d = json.load(open(path))
+        if d.get("kernel_source_hash") == kernel_source_hash():
+            return float(d["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled while the timed loop runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.rows = []
+        self.proc = None
+        self.thread = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.25)
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append([c.strip() for c in line.split(",")])
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.thread.join(timeout=2)
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in self.rows:
+            try:
+                sm.append(float(r[0]))
+                mx.append(float(r[1]))
+                for n, v in zip(names, r[4:8]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+            except Exception:
+                continue
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def algorithmic_bytes(R, V, elem, gelem):
+    """Bytes the method itself must move per step: draft and target logits read
+    once, the gradient written once, three uniforms per row read once."""
+    return R * V * (2 * elem + gelem) + R * 12
+
+
+def oracle_sample(prob, rows, T):
+    from oracle import oracle
+    K, D, V = prob["K"], prob["D"], prob["V"]
+    sub = {k: prob[k][:rows].float().cpu().numpy() for k in
+           ("draft", "target", "u_draft", "u_accept", "u_correct")}
+    k_paths = rows // D
+    t0 = time.perf_counter()
+    oracle.linear(sub["draft"], sub["target"], T, sub["u_draft"], sub["u_accept"],
+                  sub["u_correct"], min(K, k_paths), D)
+    return time.perf_counter() - t0
+
+
+def run_reference(args):
+    """The oracle, as it stands, on the host cores: each step a bounded sample
+    (the first paths of one prefix) of the same workload."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    import torch
+    from paper_2602_05774_gb300 import inputs
+    from oracle.build import build_oracle
+    build_oracle()
+    c = inputs.CONFIGS[args.config]
+    K, D, V = c["K"], c["D"], c["V"]
+    # bounded sample: one path (D rows) of prefix 0 per step, on the CPU generator
+    small = inputs.linear_problem(1, K, D, V, c["dtype"], {"vocab128k": "zipf",
+                                  "vocab32k": "spiked", "tiny": "gauss"}[args.config],
+                                  device="cpu", seed=inputs.BASE_SEED + 99)
+    temps = c["T"]
+    paths = 1
+    rows = paths * D
+    for i in range(args.warmup):
+        oracle_sample(small, rows, temps[i % len(temps)])
+    t = 0.0
+    for i in range(args.steps):
+        t += oracle_sample(small, rows, temps[i % len(temps)])
+    ms = t / args.steps * 1e3
+    val = rows / (ms / 1e3)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": val, "unit": "rows/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; same recipe)",
+        "config": {"workload": args.config, "B": c["B"], "K": K, "D": D, "V": V,
+                   "logits": c["dtype"], "temperatures": list(temps),
+                   "sample_per_step": "%d path(s) x %d rows of one prefix" % (paths, D)},
+        "cpu_baseline": {"value": val, "unit": "rows/s", "cores": 1, "kind": "oracle",
+                         "sample": "%d rows per step (one path of one prefix)" % rows},
+        "e2e": {"value": val, "unit": "rows/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2602_05774_gb300 import build, inputs, vsd
+    build.build_library()
+    vsd.load()
+    c = inputs.CONFIGS[args.config]
+    seed = inputs.BASE_SEED + list(inputs.CONFIGS).index(args.config) + 1000 * rank
+    prob = inputs.config(args.config, device=dev, seed=seed)
+    B, K, D, V = prob["B"], prob["K"], prob["D"], prob["V"]
+    R = B * K * D
+    temps = c["T"]
+    elem = prob["draft"].element_size()
+    prm = vsd.params(like=prob["draft"])
+    gelem = 2 if prm.grad_dtype == vsd.VSD_BF16 else 4
+    lay = vsd.layout(B, K, D, V)
+    ws = vsd.new_workspace(lay, dev)
+    gdt = torch.bfloat16 if gelem == 2 else torch.float32
+    out = vsd.linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=True)
+
+    def step(i):
+        vsd.estep_mstep(prob["draft"], prob["target"], prob["u_draft"], prob["u_accept"],
+                        prob["u_correct"], K, D, temps[i % len(temps)], prm=prm, workspace=ws,
+                        out=out)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize(dev)
+    code, bits = vsd.device_status(ws)
+    if code != 0:
+        raise RuntimeError("device status %d (bits %d) after warm-up" % (code, bits))
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    stream = torch.cuda.current_stream(dev)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    barrier()
+    with ClockSampler(local) as clk:
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for i in range(args.steps):
+            ev[i][0].record(stream)
+            step(i)
+            ev[i][1].record(stream)
+        t1.record(stream)
+        barrier()
+    total_ms = t0.elapsed_time(t1)
+    launch_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = tt.item()
+    ms = total_ms / args.steps
+    code, bits = vsd.device_status(ws)
+    if code != 0:
+        raise RuntimeError("device status %d (bits %d) after timing" % (code, bits))
+
+    # end-to-end through the public API from pinned host buffers
+    e2e = None
+    if not args.no_e2e:
+        hs = vsd.HostStep(B, K, D, V, prob["draft"].dtype, dev, prm=prm)
+        h_draft = prob["draft"].cpu().pin_memory()
+        h_target = prob["target"].cpu().pin_memory()
+        h_u = torch.stack([prob["u_draft"], prob["u_accept"], prob["u_correct"]]).cpu().pin_memory()
+        e_steps = max(3, min(args.steps, 30))
+        for i in range(2):
+            hs(h_draft, h_target, h_u, temps[i % len(temps)])
+        barrier()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(e_steps):
+            loss = hs(h_draft, h_target, h_u, temps[i % len(temps)])
+        b.record(stream)
+        barrier()
+        e_ms = a.elapsed_time(b) / e_steps
+        if world > 1:
+            import torch.distributed as dist
+            tt = torch.tensor([e_ms], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e_ms = tt.item()
+        e2e = {"value": R * world / (e_ms / 1e3), "unit": "rows/s",
+               "h2d_bytes_per_step": hs.h2d_bytes(), "d2h_bytes_per_step": hs.d2h_bytes(),
+               "ms_per_step": e_ms, "steps": e_steps}
+        assert torch.isfinite(loss).all()
+        del hs, h_draft, h_target, h_u
+
+    if rank != 0:
+        return
+    peak, peak_kind = peaks()
+    alg = algorithmic_bytes(R, V, elem, gelem)
+    achieved = alg / (launch_ms / 1e3) / 1e9
+    traffic = ncu_traffic(args.config)
+    value = R * world / (ms / 1e3)
+    line = {
+        "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if elem == 2 else "f32",
+        "data": "synthetic (seeded; Zipf target, noisy draft)",
+        "config": {"workload": args.config, "B": B, "K": K, "D": D, "V": V,
+                   "logits": "bf16" if elem == 2 else "f32",
+                   "grad": "bf16" if gelem == 2 else "f32", "temperatures": list(temps),
+                   "l2": "inputs larger than L2 (no flush)" if alg > 200e6 else "L2-resident",
+                   "rows_per_gpu": R},
+        "achieved_gbs": achieved,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
+                     "kernel": "k_fused", "algorithmic_bytes_per_launch": alg,
+                     "launch_ms": launch_ms},
+        "gpu_launches": args.steps,
+        "clocks": clk.summary(),
+    }
+    if e2e is not None:
+        line["e2e"] = e2e
+    if world == 1 and not args.no_cpu_baseline:
+        cpu_rows = K * D  # one prefix
+        secs = oracle_sample(prob, cpu_rows, temps[-1])
+        if secs < 8.0:
+            n = max(2, int(12.0 / max(secs, 1e-3)))
+            n = min(n, B)
+            cpu_rows = n * K * D
+            secs = oracle_sample(prob, cpu_rows, temps[-1])
+        line["cpu_baseline"] = {"value": cpu_rows / secs, "unit": "rows/s", "cores": 1,
+                                "kind": "oracle",
+                                "sample": "%d prefixes (%d rows) of the same workload, T=%g" % (
+                                    cpu_rows // (K * D), cpu_rows, temps[-1]),
+                                "seconds": secs}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

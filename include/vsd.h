@@ -1,0 +1,195 @@
+/*
+ * vsd.h -- C ABI of the GB300 (sm_103a) library for the data-parallel hot path
+ * of Variational Speculative Decoding (VSD, arxiv 2602.05774): the per-token,
+ * vocabulary-wide work of its Monte-Carlo EM draft training.
+ *
+ * For each prefix x (index b), K draft paths of depth D are drawn from the
+ * draft distribution q (Algorithm 1, E-step), every token is verified against
+ * the target distribution p with the speculative-sampling rule of Eq. 1, the
+ * accepted length and the path-level validity kappa (Eq. 2) are formed, the
+ * oracle of Algorithm 2 scores each proposal, and the M-step's weighted
+ * log-likelihood (Eq. advance, with the ARW coefficient of Eq. beta and the
+ * CAR weight of Eq. zeta) is evaluated together with its gradient with respect
+ * to the draft logits.  Names follow the paper: K is the paper's S (number of
+ * latent proposals), D its L (sampling length), T the sampling temperature,
+ * tau_car the CAR temperature tau.
+ *
+ * Conventions shared by every entry point
+ *   - Every array argument is a DEVICE pointer owned by the caller, unless the
+ *     argument says "host".  The library allocates nothing and keeps no pointer
+ *     after a call returns.
+ *   - Logit rows are row-major with the vocabulary contiguous.  Linear paths:
+ *     rows [B][K][D][V], row r = (b*K + s)*D + d, R = B*K*D rows.  Trees: rows
+ *     [B][N][V], row (b, n) is the distribution node n's children were drafted
+ *     from.  q_r = softmax(draft_r / T), p_r = softmax(target_r / T) (Eq. 1).
+ *   - Uniform random numbers are inputs (float32 in [0,1), one per row per
+ *     use).  A uniform u >= 1 draws the last token with mass; u < 0 the first.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t, NULL = the
+ *     legacy default stream).  Argument checks are synchronous and return an
+ *     error before anything is enqueued.  Data errors found on the device (a
+ *     NaN or all -inf row, a token outside [0,V), a malformed tree, a wait that
+ *     timed out) set bits of a status word in the workspace, readable with
+ *     vsd_device_status(); the kernels never trap.
+ *   - `ws` is caller-owned device scratch of at least vsd_workspace_bytes()
+ *     bytes; calls sharing one workspace must be ordered on one stream.
+ *   - Rows whose address is 16-byte aligned with V*sizeof(elem) a multiple of
+ *     16 take the 128-bit vector path; any other shape takes a scalar path with
+ *     identical results.
+ *   - Limits: 1 <= V <= 1048576, 1 <= D <= 64, 1 <= K <= 256, 1 <= N <= 1024,
+ *     B*K*D (or B*N) <= 16777216, T finite and > 0.
+ */
+#ifndef VSD_H_
+#define VSD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    VSD_OK = 0,
+    VSD_ERR_INVALID_ARG = 1, /* a size, pointer, dtype or parameter is invalid */
+    VSD_ERR_UNSUPPORTED = 2, /* a valid request this build does not serve (T = 0) */
+    VSD_ERR_CUDA = 3,        /* a CUDA runtime call failed                        */
+    VSD_ERR_TIMEOUT = 4,     /* a device-side wait gave up (vsd_device_status)    */
+    VSD_ERR_WORKSPACE = 5,   /* workspace missing or smaller than required        */
+    VSD_ERR_DEVICE_DATA = 6  /* a device-side data check failed (status bits)     */
+} vsd_status;
+
+typedef enum { VSD_F32 = 0, VSD_BF16 = 1 } vsd_dtype;
+
+/* Device status bits (vsd_device_status). */
+#define VSD_STATUS_BAD_ROW 1     /* a logit row holds NaN/+inf or is all -inf   */
+#define VSD_STATUS_TIMEOUT 2     /* a bounded device wait ran out               */
+#define VSD_STATUS_BAD_TREE 4    /* parent[0] != -1 or parent[n] not in [0, n)  */
+#define VSD_STATUS_BAD_TOKEN 8   /* a given token is outside [0, V)             */
+
+/* Problem shape.  parent == NULL: linear paths, R = B*K*D rows, N unused.
+ * parent != NULL: draft trees, device array [B][N] of parent indices
+ * (parent[b][0] = -1, 0 <= parent[b][n] < n), R = B*N rows, K and D unused. */
+typedef struct {
+    int32_t B, K, D, V, N;
+    const int32_t* parent;
+} vsd_layout;
+
+/* M-step parameters (App. F: w(l) = 1.05^l, tau = 0.2). */
+typedef struct {
+    float w_base;      /* w(l) = w_base^l, l = 1..D                                */
+    float tau_car;     /* CAR temperature tau of Eq. zeta                          */
+    int32_t zeta_mode; /* 0: softmax of q(z~_{<=l})/tau (as printed); 1: log q      */
+    int32_t grad_dtype;/* vsd_dtype of the gradient output                         */
+    uint64_t wait_timeout_ns; /* bound of every device wait; 0 = 2 s              */
+    int32_t test_never_publish; /* test hook, normally 0: if nonzero the fused kernel
+                                 never publishes a prefix's M-step, so every gradient
+                                 wait runs out after wait_timeout_ns, no gradient row
+                                 is written and VSD_STATUS_TIMEOUT is set            */
+} vsd_params;
+
+/* Output arrays of the linear E-step / M-step (all device, caller-owned).
+ * Per-row arrays have R entries, per-path arrays B*K.  A NULL member is
+ * not written, except where an entry point lists it as required. */
+typedef struct {
+    int32_t* tokens;        /* [R] z~_d, the draft sample (Algorithm 1)              */
+    float* logq_tok;        /* [R] log q_r(z~_d)                                      */
+    float* alpha;           /* [R] min(1, p_r(z~_d)/q_r(z~_d)) (Eq. 1)                */
+    uint8_t* accept;        /* [R] u_accept <= alpha                                  */
+    int32_t* accept_len;    /* [B*K] A: number of leading accepted tokens             */
+    int32_t* corr_tokens;   /* [R] z'_d: z~_d before the first rejection, a residual
+                               token norm(max(0,p-q)) at it, p-samples after it      */
+    float* logq_corr;       /* [R] log q_r(z'_d)                                      */
+    float* alpha_corr;      /* [R] min(1, p/q) at z'_d                                */
+    float* logkappa;        /* [R] log kappa(z~_{<=l}), l = d+1 (Eq. 2)               */
+    float* logkappa_corr;   /* [R] log kappa(z'_{<=l})                                */
+    float* logkappa_ref;    /* [R] log kappa of the greedy reference (Algorithm 2)    */
+    int32_t* ref_tokens;    /* [R] argmax of the target row (lowest index on ties)    */
+    float* expected_len;    /* [B*K] sum_{k<=D} S_k (Eq. 11)                          */
+    float* row_stats;       /* [R][4] m_q, logZ_q, m_p, logZ_p with
+                               log q(v) = (x_v - m_q)/T - logZ_q                     */
+    float* weights;         /* [B][D][K][4] o~, o', beta, zeta (Alg. 1, Eq. beta/zeta)*/
+    float* loss;            /* [B+1] loss_b = -J_b/N_b, then mean over b (Eq. advance)*/
+    void* grad;             /* [R][V] d loss / d draft logits, params.grad_dtype      */
+} vsd_linear_outputs;
+
+/* Output arrays of tree verification (device, caller-owned), [B][N] unless noted. */
+typedef struct {
+    float* alpha;           /* min(1, p/q) of node n's token at its parent's row; root 1 */
+    uint8_t* accept;        /* u_accept <= alpha; root 1                                 */
+    uint8_t* path_accept;   /* node and all its ancestors accepted                       */
+    float* logkappa;        /* sum of log alpha from the root to n                       */
+    int32_t* corr_tokens;   /* residual token at the parent's row for a rejected node
+                               whose parent is on an accepted path; -1 otherwise         */
+    int32_t* deepest;       /* [B] deepest node on an accepted path (lowest index)       */
+    int32_t* accept_len;    /* [B] depth of that node                                    */
+    int32_t* bonus;         /* [B] token after the accepted path: the residual of the
+                               deepest node's first child, or a p-sample at its row      */
+    float* row_stats;       /* optional [B*N][4] as in vsd_linear_outputs                */
+} vsd_tree_outputs;
+
+/* Bytes of device workspace the calls below need for `layout` (0 if invalid). */
+size_t vsd_workspace_bytes(vsd_layout layout);
+
+/* Draft sampling (Algorithm 1, z~ ~ q): for every linear row, the inverse-CDF
+ * draw z~_r = min{v : u_draft_r < sum_{j<=v} q_r(j)} and log q_r(z~_r).
+ * draft: [R][V] of `dtype`.  u_draft: [R].  Outputs: tokens [R], logq_tok [R],
+ * row_stats optional [R][4] (the p columns are written as 0).  Linear layout only. */
+vsd_status vsd_sample_paths(const void* draft, vsd_dtype dtype, vsd_layout layout, float T,
+                            const float* u_draft, int32_t* tokens, float* logq_tok,
+                            float* row_stats, void* ws, size_t ws_bytes, void* stream);
+
+/* Verification (Eq. 1 per token; Sec. 3 residual correction; Eqs. 2, 9-11;
+ * Algorithm 2's greedy reference).
+ * Linear layout: tokens are the drafted z~ [R] (for example from
+ * vsd_sample_paths); u_accept, u_correct [R]; ref_logkappa optional [B][D]
+ * (NULL: the greedy reference of each path, read from the same rows).  Writes
+ * every verification member of `out` that is non-NULL (required: accept_len,
+ * corr_tokens, logkappa); tokens/logq_tok are copied through.
+ * Tree layout: tokens [B][N] (node 0 ignored), u_accept, u_correct [B][N],
+ * ref_logkappa must be NULL, results in `tree_out` (all members but row_stats
+ * required); `out` is ignored. */
+vsd_status vsd_verify_paths(const void* draft, const void* target, vsd_dtype dtype,
+                            vsd_layout layout, float T, const int32_t* tokens,
+                            const float* u_accept, const float* u_correct,
+                            const float* ref_logkappa, vsd_linear_outputs* out,
+                            vsd_tree_outputs* tree_out, void* ws, size_t ws_bytes,
+                            void* stream);
+
+/* M-step (Algorithm 1 M-step, Algorithm 2 utility, Eqs. beta, zeta, advance):
+ * from the E-step results in `estep` (tokens, corr_tokens, logq_tok, logq_corr,
+ * logkappa, logkappa_corr, logkappa_ref, row_stats: all required) computes
+ * o~, o', beta, zeta, loss_b = -J_b/N_b, their mean, and the gradient of the
+ * mean loss with respect to the draft logits, with o~, o', beta, zeta, N_b held
+ * constant.  loss [B+1] and grad [R][V] (params->grad_dtype) are required,
+ * weights [B][D][K][4] optional.  Linear layout only. */
+vsd_status vsd_weighted_loss_fwd_bwd(const void* draft, vsd_dtype dtype, vsd_layout layout,
+                                     float T, const vsd_linear_outputs* estep,
+                                     const vsd_params* params, float* loss, void* grad,
+                                     float* weights, void* ws, size_t ws_bytes, void* stream);
+
+/* The fused E-step + M-step: one persistent kernel runs sampling, verification,
+ * utilities, weights, loss and gradient over all prefixes.  Required members
+ * of `out`: tokens, accept_len, corr_tokens, logkappa, loss, grad; the rest are
+ * optional.  Linear layout only. */
+vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtype,
+                           vsd_layout layout, float T, const float* u_draft,
+                           const float* u_accept, const float* u_correct,
+                           const float* ref_logkappa, const vsd_params* params,
+                           vsd_linear_outputs* out, void* ws, size_t ws_bytes, void* stream);
+
+/* Waits for `stream`, then reads and clears the device status word of `ws`
+ * into *status_bits (host).  Returns VSD_ERR_TIMEOUT if the timeout bit is set,
+ * VSD_ERR_DEVICE_DATA for any other bit, VSD_OK if none. */
+vsd_status vsd_device_status(void* ws, void* stream, int32_t* status_bits);
+
+/* A static English description of a status code. */
+const char* vsd_status_string(vsd_status status);
+
+/* Library version, "major.minor.patch". */
+const char* vsd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VSD_H_ */

@@ -1,0 +1,420 @@
+// vsd_api.cu -- the C ABI of include/vsd.h: argument checks, workspace layout
+// and launch sequencing on the caller's stream.  Every compute step runs in
+// the kernels of vsd_kernels_{f32,bf16}.cu; this file only marshals.
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <cuda_runtime.h>
+
+#include "vsd.h"
+#include "vsd_launch.h"
+
+namespace vsd {
+namespace {
+
+constexpr int kMaxV = 1 << 20;
+constexpr int kMaxD = 64;
+constexpr int kMaxK = 256;
+constexpr int kMaxN = 1024;
+constexpr int64_t kMaxRows = 1 << 24;
+constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+struct WsLayout {
+    size_t status, ticket, prefix_done, path_cnt, prefix_cnt, ready, zero_end;
+    size_t rows, rstats, es_tok, es_corr, es_lq_tok, es_lq_corr, es_lk, es_lkc, es_lkr;
+    size_t coef, wscr, total;
+};
+
+bool layout_ok(const vsd_layout& L) {
+    if (L.B < 1 || L.V < 1 || L.V > kMaxV) return false;
+    if (L.parent) {
+        if (L.N < 1 || L.N > kMaxN) return false;
+        return (int64_t)L.B * L.N <= kMaxRows;
+    }
+    if (L.K < 1 || L.K > kMaxK || L.D < 1 || L.D > kMaxD) return false;
+    return (int64_t)L.B * L.K * L.D <= kMaxRows;
+}
+
+int64_t rows_of(const vsd_layout& L) {
+    return L.parent ? (int64_t)L.B * L.N : (int64_t)L.B * L.K * L.D;
+}
+
+WsLayout ws_layout(const vsd_layout& L) {
+    WsLayout w;
+    const size_t R = (size_t)rows_of(L);
+    const size_t npath = L.parent ? (size_t)L.B : (size_t)L.B * L.K;
+    size_t o = 0;
+    w.status = 0;
+    w.ticket = 4;
+    w.prefix_done = 8;
+    o = 256;
+    w.path_cnt = o; o = align256(o + 4 * npath);
+    w.prefix_cnt = o; o = align256(o + 4 * (size_t)L.B);
+    w.ready = o; o = align256(o + 4 * (size_t)L.B);
+    w.zero_end = o;
+    w.rows = o; o = align256(o + sizeof(RowRec) * R);
+    w.rstats = o; o = align256(o + sizeof(float4) * R);
+    w.es_tok = o; o = align256(o + 4 * R);
+    w.es_corr = o; o = align256(o + 4 * R);
+    w.es_lq_tok = o; o = align256(o + 4 * R);
+    w.es_lq_corr = o; o = align256(o + 4 * R);
+    w.es_lk = o; o = align256(o + 4 * R);
+    w.es_lkc = o; o = align256(o + 4 * R);
+    w.es_lkr = o; o = align256(o + 4 * R);
+    w.coef = o; o = align256(o + sizeof(Coef) * R);
+    w.wscr = o; o = align256(o + sizeof(double2) * R);
+    w.total = o;
+    return w;
+}
+
+template <typename U> U* at(void* ws, size_t off) {
+    return reinterpret_cast<U*>(static_cast<char*>(ws) + off);
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+int num_sms() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 1;
+    return n > 0 ? n : 1;
+}
+
+size_t l2_bytes() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrL2CacheSize, dev) != cudaSuccess) return 0;
+    return (size_t)n;
+}
+
+vsd_status check_temperature(float T) {
+    if (T == 0.f) return VSD_ERR_UNSUPPORTED;  // greedy decoding is not served here
+    if (!(T > 0.f) || !isfinite(T)) return VSD_ERR_INVALID_ARG;
+    return VSD_OK;
+}
+
+vsd_status check_ws(const vsd_layout& L, void* ws, size_t ws_bytes) {
+    if (!ws) return VSD_ERR_WORKSPACE;
+    if (!aligned16(ws)) return VSD_ERR_WORKSPACE;
+    if (ws_bytes < ws_layout(L).total) return VSD_ERR_WORKSPACE;
+    return VSD_OK;
+}
+
+vsd_status from_cuda(cudaError_t e) { return e == cudaSuccess ? VSD_OK : VSD_ERR_CUDA; }
+
+vsd_params default_params(vsd_dtype dtype) {
+    vsd_params p;
+    p.w_base = 1.05f;
+    p.tau_car = 0.2f;
+    p.zeta_mode = 0;
+    p.grad_dtype = dtype;
+    p.wait_timeout_ns = kDefaultTimeoutNs;
+    p.test_never_publish = 0;
+    return p;
+}
+
+vsd_status check_params(const vsd_params& p) {
+    if (!(p.w_base > 0.f) || !isfinite(p.w_base)) return VSD_ERR_INVALID_ARG;
+    if (!(p.tau_car > 0.f)) return VSD_ERR_INVALID_ARG;  // +inf allowed: zeta = 1/K
+    if (p.zeta_mode != 0 && p.zeta_mode != 1) return VSD_ERR_INVALID_ARG;
+    if (p.grad_dtype != VSD_F32 && p.grad_dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
+    return VSD_OK;
+}
+
+// Fill the shape, temperature, workspace views of a problem.
+template <typename T>
+Problem<T> make_problem(const void* draft, const void* target, const vsd_layout& L, float T_,
+                        void* ws) {
+    Problem<T> P;
+    memset(&P, 0, sizeof(P));
+    P.draft = static_cast<const T*>(draft);
+    P.target = static_cast<const T*>(target);
+    P.B = L.B;
+    P.K = L.parent ? 1 : L.K;
+    P.D = L.parent ? 1 : L.D;
+    P.N = L.parent ? L.N : 0;
+    P.V = L.V;
+    P.R = (int)rows_of(L);
+    P.nch = (int)((L.V + chunk_elems<T>() - 1) / chunk_elems<T>());
+    P.ts.c = (float)(kLog2e / (double)T_);
+    P.ts.T = T_;
+    P.ts.Td = (double)T_;
+    P.parent = L.parent;
+    P.w_base = 1.05f;
+    P.tau_car = 0.2f;
+    P.timeout_ns = kDefaultTimeoutNs;
+    const WsLayout w = ws_layout(L);
+    P.status = at<int>(ws, w.status);
+    P.ticket = at<int>(ws, w.ticket);
+    P.prefix_done = at<int>(ws, w.prefix_done);
+    P.path_cnt = at<int>(ws, w.path_cnt);
+    P.prefix_cnt = at<int>(ws, w.prefix_cnt);
+    P.ready = at<int>(ws, w.ready);
+    P.rows = at<RowRec>(ws, w.rows);
+    P.rstats = at<float4>(ws, w.rstats);
+    P.es.tok = at<int32_t>(ws, w.es_tok);
+    P.es.corr = at<int32_t>(ws, w.es_corr);
+    P.es.lq_tok = at<float>(ws, w.es_lq_tok);
+    P.es.lq_corr = at<float>(ws, w.es_lq_corr);
+    P.es.lk = at<float>(ws, w.es_lk);
+    P.es.lkc = at<float>(ws, w.es_lkc);
+    P.es.lkr = at<float>(ws, w.es_lkr);
+    P.coef = at<Coef>(ws, w.coef);
+    P.wscr = at<double2>(ws, w.wscr);
+    return P;
+}
+
+template <typename T>
+void set_params(Problem<T>& P, const vsd_params& p) {
+    P.w_base = p.w_base;
+    P.tau_car = p.tau_car;
+    P.zeta_mode = p.zeta_mode;
+    P.grad_bf16 = p.grad_dtype == VSD_BF16;
+    P.timeout_ns = p.wait_timeout_ns ? p.wait_timeout_ns : kDefaultTimeoutNs;
+    P.inject_wait_fault = p.test_never_publish;
+}
+
+cudaError_t clear_counters(void* ws, const vsd_layout& L, cudaStream_t s) {
+    return cudaMemsetAsync(ws, 0, ws_layout(L).zero_end, s);
+}
+
+bool vec_ok(const void* a, const void* b, const void* g, int V, size_t elem, size_t gelem) {
+    if (!aligned16(a) || (b && !aligned16(b)) || (g && !aligned16(g))) return false;
+    if (((size_t)V * elem) % 16 != 0) return false;
+    if (g && ((size_t)V * gelem) % 16 != 0) return false;
+    return true;
+}
+
+// ------------------------------------------------------------ entry bodies
+template <typename T>
+vsd_status sample_impl(const void* draft, vsd_layout L, float T_, const float* u_draft,
+                       int32_t* tokens, float* logq_tok, float* row_stats, void* ws,
+                       cudaStream_t s) {
+    Problem<T> P = make_problem<T>(draft, nullptr, L, T_, ws);
+    P.u_draft = u_draft;
+    P.out.tokens = tokens;
+    P.out.logq_tok = logq_tok;
+    P.out.row_stats = row_stats;
+    const bool vec = vec_ok(draft, nullptr, nullptr, L.V, sizeof(T), 0);
+    cudaError_t e = clear_counters(ws, L, s);
+    if (e == cudaSuccess) e = Launch<T>::sample(P, vec, s);
+    return from_cuda(e);
+}
+
+template <typename T>
+vsd_status verify_impl(const void* draft, const void* target, vsd_layout L, float T_,
+                       const int32_t* tokens, const float* u_accept, const float* u_correct,
+                       const float* ref_logkappa, vsd_linear_outputs* out,
+                       vsd_tree_outputs* tout, void* ws, cudaStream_t s) {
+    Problem<T> P = make_problem<T>(draft, target, L, T_, ws);
+    P.given_tokens = tokens;
+    P.u_accept = u_accept;
+    P.u_correct = u_correct;
+    P.ref_logkappa = ref_logkappa;
+    const bool vec = vec_ok(draft, target, nullptr, L.V, sizeof(T), 0);
+    cudaError_t e = clear_counters(ws, L, s);
+    if (L.parent) {
+        P.tout = *tout;
+        if (e == cudaSuccess) e = Launch<T>::rows_verify(P, vec, true, s);
+        if (e == cudaSuccess) e = Launch<T>::tree(P, vec, s);
+    } else {
+        P.out = *out;
+        if (e == cudaSuccess) e = Launch<T>::rows_verify(P, vec, false, s);
+        if (e == cudaSuccess) e = Launch<T>::paths(P, vec, s);
+    }
+    return from_cuda(e);
+}
+
+template <typename T>
+vsd_status loss_impl(const void* draft, vsd_layout L, float T_, const vsd_linear_outputs* es,
+                     const vsd_params& p, float* loss, void* grad, float* weights, void* ws,
+                     cudaStream_t s) {
+    Problem<T> P = make_problem<T>(draft, nullptr, L, T_, ws);
+    set_params(P, p);
+    const EStepView E{es->tokens, es->corr_tokens, es->logq_tok, es->logq_corr,
+                      es->logkappa, es->logkappa_corr, es->logkappa_ref};
+    const size_t gelem = P.grad_bf16 ? 2 : 4;
+    const bool vec = vec_ok(draft, nullptr, grad, L.V, sizeof(T), gelem);
+    cudaError_t e = clear_counters(ws, L, s);
+    if (e == cudaSuccess) e = Launch<T>::weights(P, E, weights, loss, s);
+    if (e == cudaSuccess)
+        e = Launch<T>::grad(P, vec, reinterpret_cast<const float4*>(es->row_stats), grad,
+                            P.grad_bf16, s);
+    return from_cuda(e);
+}
+
+template <typename T>
+vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float T_,
+                      const float* u_draft, const float* u_accept, const float* u_correct,
+                      const float* ref_logkappa, const vsd_params& p,
+                      const vsd_linear_outputs* out, void* ws, cudaStream_t s) {
+    Problem<T> P = make_problem<T>(draft, target, L, T_, ws);
+    set_params(P, p);
+    P.u_draft = u_draft;
+    P.u_accept = u_accept;
+    P.u_correct = u_correct;
+    P.ref_logkappa = ref_logkappa;
+    P.out = *out;
+    const size_t gelem = P.grad_bf16 ? 2 : 4;
+    const bool vec = vec_ok(draft, target, out->grad, L.V, sizeof(T), gelem);
+    const int per_sm = Launch<T>::fused_blocks_per_sm(P, vec, P.grad_bf16);
+    const int64_t tickets = 2 * (int64_t)P.R;
+    int ctas = per_sm * num_sms();
+    if ((int64_t)ctas > tickets) ctas = (int)tickets;
+    const char* env_ctas = getenv("VSD_FUSED_CTAS");
+    if (env_ctas && atoi(env_ctas) > 0 && atoi(env_ctas) < ctas) ctas = atoi(env_ctas);
+    // Rows of `lag` prefixes are scheduled ahead of a prefix's gradient rows:
+    // enough independent work to cover the blocks in flight, capped so that
+    // the draft rows still to be re-read fit comfortably in L2.
+    const int Pp = P.K * P.D;
+    int lag = (2 * ctas + Pp - 1) / Pp;
+    const size_t l2 = l2_bytes();
+    const size_t prefix_bytes = (size_t)Pp * (size_t)L.V * sizeof(T);
+    while (lag > 1 && l2 && (size_t)(lag + 1) * prefix_bytes > (l2 * 3) / 5) --lag;
+    if (lag < 1) lag = 1;
+    const char* env_lag = getenv("VSD_FUSED_LAG");
+    if (env_lag && atoi(env_lag) > 0) lag = atoi(env_lag);
+    if (lag > P.B - 1) lag = P.B - 1 > 0 ? P.B - 1 : 0;
+    P.lag = lag;
+    cudaError_t e = clear_counters(ws, L, s);
+    if (e == cudaSuccess) e = Launch<T>::fused(P, vec, out->grad, P.grad_bf16, ctas, s);
+    return from_cuda(e);
+}
+
+}  // namespace
+}  // namespace vsd
+
+using namespace vsd;
+
+extern "C" {
+
+size_t vsd_workspace_bytes(vsd_layout layout) {
+    if (!layout_ok(layout)) return 0;
+    return ws_layout(layout).total;
+}
+
+vsd_status vsd_sample_paths(const void* draft, vsd_dtype dtype, vsd_layout layout, float T,
+                            const float* u_draft, int32_t* tokens, float* logq_tok,
+                            float* row_stats, void* ws, size_t ws_bytes, void* stream) {
+    if (!layout_ok(layout) || layout.parent) return VSD_ERR_INVALID_ARG;
+    if (!draft || !u_draft || !tokens || !logq_tok) return VSD_ERR_INVALID_ARG;
+    if (dtype != VSD_F32 && dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
+    vsd_status st = check_temperature(T);
+    if (st) return st;
+    if ((st = check_ws(layout, ws, ws_bytes))) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (dtype == VSD_F32)
+        return sample_impl<float>(draft, layout, T, u_draft, tokens, logq_tok, row_stats, ws, s);
+    return sample_impl<__nv_bfloat16>(draft, layout, T, u_draft, tokens, logq_tok, row_stats, ws,
+                                      s);
+}
+
+vsd_status vsd_verify_paths(const void* draft, const void* target, vsd_dtype dtype,
+                            vsd_layout layout, float T, const int32_t* tokens,
+                            const float* u_accept, const float* u_correct,
+                            const float* ref_logkappa, vsd_linear_outputs* out,
+                            vsd_tree_outputs* tree_out, void* ws, size_t ws_bytes,
+                            void* stream) {
+    if (!layout_ok(layout)) return VSD_ERR_INVALID_ARG;
+    if (!draft || !target || !tokens || !u_accept || !u_correct) return VSD_ERR_INVALID_ARG;
+    if (dtype != VSD_F32 && dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
+    if (layout.parent) {
+        if (!tree_out || ref_logkappa) return VSD_ERR_INVALID_ARG;
+        const vsd_tree_outputs& o = *tree_out;
+        if (!o.alpha || !o.accept || !o.path_accept || !o.logkappa || !o.corr_tokens ||
+            !o.deepest || !o.accept_len || !o.bonus)
+            return VSD_ERR_INVALID_ARG;
+    } else {
+        if (!out || !out->accept_len || !out->corr_tokens || !out->logkappa)
+            return VSD_ERR_INVALID_ARG;
+    }
+    vsd_status st = check_temperature(T);
+    if (st) return st;
+    if ((st = check_ws(layout, ws, ws_bytes))) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (dtype == VSD_F32)
+        return verify_impl<float>(draft, target, layout, T, tokens, u_accept, u_correct,
+                                  ref_logkappa, out, tree_out, ws, s);
+    return verify_impl<__nv_bfloat16>(draft, target, layout, T, tokens, u_accept, u_correct,
+                                      ref_logkappa, out, tree_out, ws, s);
+}
+
+vsd_status vsd_weighted_loss_fwd_bwd(const void* draft, vsd_dtype dtype, vsd_layout layout,
+                                     float T, const vsd_linear_outputs* estep,
+                                     const vsd_params* params, float* loss, void* grad,
+                                     float* weights, void* ws, size_t ws_bytes, void* stream) {
+    if (!layout_ok(layout) || layout.parent) return VSD_ERR_INVALID_ARG;
+    if (!draft || !estep || !loss || !grad) return VSD_ERR_INVALID_ARG;
+    if (!estep->tokens || !estep->corr_tokens || !estep->logq_tok || !estep->logq_corr ||
+        !estep->logkappa || !estep->logkappa_corr || !estep->logkappa_ref || !estep->row_stats)
+        return VSD_ERR_INVALID_ARG;
+    if (dtype != VSD_F32 && dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
+    vsd_status st = check_temperature(T);
+    if (st) return st;
+    const vsd_params p = params ? *params : default_params(dtype);
+    if ((st = check_params(p))) return st;
+    if ((st = check_ws(layout, ws, ws_bytes))) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (dtype == VSD_F32)
+        return loss_impl<float>(draft, layout, T, estep, p, loss, grad, weights, ws, s);
+    return loss_impl<__nv_bfloat16>(draft, layout, T, estep, p, loss, grad, weights, ws, s);
+}
+
+vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtype,
+                           vsd_layout layout, float T, const float* u_draft,
+                           const float* u_accept, const float* u_correct,
+                           const float* ref_logkappa, const vsd_params* params,
+                           vsd_linear_outputs* out, void* ws, size_t ws_bytes, void* stream) {
+    if (!layout_ok(layout) || layout.parent) return VSD_ERR_INVALID_ARG;
+    if (!draft || !target || !u_draft || !u_accept || !u_correct || !out)
+        return VSD_ERR_INVALID_ARG;
+    if (!out->tokens || !out->accept_len || !out->corr_tokens || !out->logkappa || !out->loss ||
+        !out->grad)
+        return VSD_ERR_INVALID_ARG;
+    if (dtype != VSD_F32 && dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
+    vsd_status st = check_temperature(T);
+    if (st) return st;
+    const vsd_params p = params ? *params : default_params(dtype);
+    if ((st = check_params(p))) return st;
+    if ((st = check_ws(layout, ws, ws_bytes))) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (dtype == VSD_F32)
+        return fused_impl<float>(draft, target, layout, T, u_draft, u_accept, u_correct,
+                                 ref_logkappa, p, out, ws, s);
+    return fused_impl<__nv_bfloat16>(draft, target, layout, T, u_draft, u_accept, u_correct,
+                                     ref_logkappa, p, out, ws, s);
+}
+
+vsd_status vsd_device_status(void* ws, void* stream, int32_t* status_bits) {
+    if (!ws || !status_bits) return VSD_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int32_t v = 0;
+    cudaError_t e = cudaMemcpyAsync(&v, ws, sizeof(v), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(ws, 0, sizeof(v), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return VSD_ERR_CUDA;
+    *status_bits = v;
+    if (v & VSD_STATUS_TIMEOUT) return VSD_ERR_TIMEOUT;
+    return v ? VSD_ERR_DEVICE_DATA : VSD_OK;
+}
+
+const char* vsd_status_string(vsd_status status) {
+    switch (status) {
+        case VSD_OK: return "ok";
+        case VSD_ERR_INVALID_ARG: return "invalid argument";
+        case VSD_ERR_UNSUPPORTED: return "unsupported request (temperature 0)";
+        case VSD_ERR_CUDA: return "CUDA runtime error";
+        case VSD_ERR_TIMEOUT: return "a device-side wait timed out";
+        case VSD_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+        case VSD_ERR_DEVICE_DATA: return "device-side data check failed";
+    }
+    return "unknown status";
+}
+
+const char* vsd_version(void) { return "0.1.0"; }
+
+}  // extern "C"

@@ -1,0 +1,213 @@
+// vsd_common.cuh -- low-level device helpers for the VSD E-step / M-step
+// kernels (sm_103a): cache-hinted 128-bit loads and stores, bf16/f32 unpacking,
+// warp reductions, the exponent scale of a temperature, bounded waits.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "vsd.h"
+
+namespace vsd {
+
+constexpr int kThreads = 256;            // threads of every block-level pass
+constexpr int kWarps = kThreads / 32;
+constexpr int kLoads = 4;                // 16-byte vectors per lane per chunk per tensor
+constexpr double kLog2e = 1.4426950408889634073599246810019;
+constexpr double kLn2 = 0.69314718055994530941723212145818;
+
+template <typename T> struct Traits;
+template <> struct Traits<float> {
+    static constexpr int kPerVec = 4;
+    static constexpr uint32_t kNegInf = 0xFF800000u;
+};
+template <> struct Traits<__nv_bfloat16> {
+    static constexpr int kPerVec = 8;
+    static constexpr uint32_t kNegInf = 0xFF80FF80u;  // two bf16 -inf
+};
+// A chunk is what one warp holds in registers at a time: 32 lanes x kLoads
+// vectors = 2 KB of one tensor (1024 bf16 or 512 f32 logits).
+template <typename T> __host__ __device__ constexpr int chunk_elems() {
+    return 32 * kLoads * Traits<T>::kPerVec;
+}
+
+// exp(x / T) = 2^(x * c) with c = log2(e) / T.
+struct TempScale {
+    float c;        // log2(e)/T rounded to float
+    float T;
+    double Td;
+};
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// ---------------------------------------------------------------- loads
+__device__ __forceinline__ uint64_t policy_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_last() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_normal() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+// Read-only 128-bit load that bypasses L1 and carries an L2 eviction policy.
+__device__ __forceinline__ uint4 ld_stream(const void* p, uint64_t pol) {
+    uint4 r;
+    asm("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+        : "l"(p), "l"(pol));
+    return r;
+}
+
+// 128-bit store with an L2 eviction policy.
+__device__ __forceinline__ void st_stream(void* p, uint4 v, uint64_t pol) {
+    asm volatile("st.global.L1::no_allocate.L2::cache_hint.v4.u32 [%0], {%1,%2,%3,%4}, %5;"
+                 :: "l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "l"(pol) : "memory");
+}
+
+// Coherent (L1-bypassing) loads of data written by other blocks of the same grid.
+template <typename U> __device__ __forceinline__ U ld_cg(const U* p) { return __ldcg(p); }
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release(int* p, int v) {
+    asm volatile("st.release.gpu.global.b32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Scalar element load (for rows that are not 16-byte aligned).
+__device__ __forceinline__ uint32_t raw_elem(const float* row, int64_t v) {
+    return __float_as_uint(__ldg(row + v));
+}
+__device__ __forceinline__ uint32_t raw_elem(const __nv_bfloat16* row, int64_t v) {
+    return (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(row) + v);
+}
+__device__ __forceinline__ float elem_value(const float* row, int64_t v) { return __ldg(row + v); }
+__device__ __forceinline__ float elem_value(const __nv_bfloat16* row, int64_t v) {
+    return __uint_as_float(raw_elem(row, v) << 16);
+}
+
+// Load chunk c of a row into registers: lane l, vector k holds elements
+// c*CE + k*32*PV + l*PV + [0, PV).  Elements at or beyond V read as -inf.
+template <typename T, bool VEC>
+__device__ __forceinline__ void load_chunk(const T* row, int64_t V, int c, int lane, uint64_t pol,
+                                           uint4 (&buf)[kLoads]) {
+    constexpr int PV = Traits<T>::kPerVec;
+    const int64_t base = (int64_t)c * chunk_elems<T>() + lane * PV;
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k) {
+        const int64_t v0 = base + (int64_t)k * 32 * PV;
+        if constexpr (VEC) {
+            if (v0 < V) {
+                buf[k] = ld_stream(row + v0, pol);
+            } else {
+                buf[k] = make_uint4(Traits<T>::kNegInf, Traits<T>::kNegInf, Traits<T>::kNegInf,
+                                    Traits<T>::kNegInf);
+            }
+        } else {
+            uint32_t w[4];
+            if constexpr (PV == 4) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    w[e] = (v0 + e < V) ? raw_elem(row, v0 + e) : Traits<T>::kNegInf;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    uint32_t lo = (v0 + 2 * e < V) ? raw_elem(row, v0 + 2 * e) : 0xFF80u;
+                    uint32_t hi = (v0 + 2 * e + 1 < V) ? raw_elem(row, v0 + 2 * e + 1) : 0xFF80u;
+                    w[e] = lo | (hi << 16);
+                }
+            }
+            buf[k] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+    }
+}
+
+template <typename T> __device__ __forceinline__ void unpack(const uint4& v, float* f);
+template <> __device__ __forceinline__ void unpack<float>(const uint4& v, float* f) {
+    f[0] = __uint_as_float(v.x); f[1] = __uint_as_float(v.y);
+    f[2] = __uint_as_float(v.z); f[3] = __uint_as_float(v.w);
+}
+template <> __device__ __forceinline__ void unpack<__nv_bfloat16>(const uint4& v, float* f) {
+    f[0] = __uint_as_float(v.x << 16); f[1] = __uint_as_float(v.x & 0xFFFF0000u);
+    f[2] = __uint_as_float(v.y << 16); f[3] = __uint_as_float(v.y & 0xFFFF0000u);
+    f[4] = __uint_as_float(v.z << 16); f[5] = __uint_as_float(v.z & 0xFFFF0000u);
+    f[6] = __uint_as_float(v.w << 16); f[7] = __uint_as_float(v.w & 0xFFFF0000u);
+}
+
+// Max over one 16-byte vector (NaN elements are ignored here; they surface
+// through the exponential sums).
+template <typename T> __device__ __forceinline__ float vec_max(const uint4& v);
+template <> __device__ __forceinline__ float vec_max<float>(const uint4& v) {
+    return fmaxf(fmaxf(__uint_as_float(v.x), __uint_as_float(v.y)),
+                 fmaxf(__uint_as_float(v.z), __uint_as_float(v.w)));
+}
+template <> __device__ __forceinline__ float vec_max<__nv_bfloat16>(const uint4& v) {
+    __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&v.x);
+    __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&v.y);
+    __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&v.z);
+    __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162*>(&v.w);
+    __nv_bfloat162 m = __hmax2(__hmax2(a, b), __hmax2(c, d));
+    return fmaxf(__low2float(m), __high2float(m));
+}
+
+// ---------------------------------------------------------------- warps
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ int warp_min(int v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+// Inclusive prefix sum over the lanes of a warp.
+__device__ __forceinline__ float warp_incl_scan(float v, int lane) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        float n = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += n;
+    }
+    return v;
+}
+__device__ __forceinline__ double warp_incl_scan(double v, int lane) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        double n = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += n;
+    }
+    return v;
+}
+
+}  // namespace vsd

@@ -1,0 +1,35 @@
+// vsd_launch.h -- host-side launchers of the VSD kernels, one set per logit
+// dtype (defined in vsd_kernels_f32.cu and vsd_kernels_bf16.cu).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "vsd_passes.cuh"
+
+namespace vsd {
+
+template <typename T> struct Launch {
+    // z~ ~ q per row, tokens/logq/row_stats written from the row records
+    static cudaError_t sample(const Problem<T>& P, bool vec, cudaStream_t s);
+    // row statistics of draft+target with given tokens (linear) or none (tree)
+    static cudaError_t rows_verify(const Problem<T>& P, bool vec, bool tree, cudaStream_t s);
+    // accepted lengths, residual draws, corrected paths, log-kappa (linear)
+    static cudaError_t paths(const Problem<T>& P, bool vec, cudaStream_t s);
+    // tree acceptance scan, residual draws, deepest node, bonus
+    static cudaError_t tree(const Problem<T>& P, bool vec, cudaStream_t s);
+    // M-step weights and loss from an E-step view
+    static cudaError_t weights(const Problem<T>& P, const EStepView& E, float* weights,
+                              float* loss, cudaStream_t s);
+    // gradient rows from coefficients and row statistics
+    static cudaError_t grad(const Problem<T>& P, bool vec, const float4* rstats, void* grad,
+                            bool grad_bf16, cudaStream_t s);
+    // the fused persistent E-step + M-step kernel
+    static cudaError_t fused(const Problem<T>& P, bool vec, void* grad, bool grad_bf16,
+                             int ctas, cudaStream_t s);
+    // resident blocks per SM of the fused kernel
+    static int fused_blocks_per_sm(const Problem<T>& P, bool vec, bool grad_bf16);
+};
+
+inline size_t table_smem_bytes(int nch) { return (size_t)nch * sizeof(float4); }
+
+}  // namespace vsd

@@ -1,0 +1,355 @@
+"""Python binding of libvsd (include/vsd.h): argument marshalling only.
+
+Every step of the E-step / M-step runs in the library's CUDA kernels; this
+module checks tensor shapes and dtypes, allocates output tensors when the
+caller gives none, passes raw device pointers and the current CUDA stream, and
+turns status codes into exceptions.  PyTorch provides device memory and
+streams.  There is no CPU fallback: if libvsd.so is missing or fails to load,
+every call raises.
+"""
+import ctypes as C
+import os
+
+import torch
+
+from . import build as _build
+
+VSD_F32, VSD_BF16 = 0, 1
+STATUS_BAD_ROW, STATUS_TIMEOUT, STATUS_BAD_TREE, STATUS_BAD_TOKEN = 1, 2, 4, 8
+_STATUS_NAMES = {0: "VSD_OK", 1: "VSD_ERR_INVALID_ARG", 2: "VSD_ERR_UNSUPPORTED",
+                 3: "VSD_ERR_CUDA", 4: "VSD_ERR_TIMEOUT", 5: "VSD_ERR_WORKSPACE",
+                 6: "VSD_ERR_DEVICE_DATA"}
+
+SYMBOLS = ("vsd_workspace_bytes", "vsd_sample_paths", "vsd_verify_paths",
+           "vsd_weighted_loss_fwd_bwd", "vsd_estep_mstep", "vsd_device_status",
+           "vsd_status_string", "vsd_version")
+
+
+class VsdError(RuntimeError):
+    def __init__(self, code, where):
+        self.code = code
+        msg = _lib().vsd_status_string(code).decode() if _LIB is not None else "?"
+        super().__init__("%s: %s (%s)" % (where, _STATUS_NAMES.get(code, code), msg))
+
+
+class Layout(C.Structure):
+    _fields_ = [("B", C.c_int32), ("K", C.c_int32), ("D", C.c_int32), ("V", C.c_int32),
+                ("N", C.c_int32), ("parent", C.c_void_p)]
+
+
+class Params(C.Structure):
+    _fields_ = [("w_base", C.c_float), ("tau_car", C.c_float), ("zeta_mode", C.c_int32),
+                ("grad_dtype", C.c_int32), ("wait_timeout_ns", C.c_uint64),
+                ("test_never_publish", C.c_int32)]
+
+
+LINEAR_FIELDS = ("tokens", "logq_tok", "alpha", "accept", "accept_len", "corr_tokens",
+                 "logq_corr", "alpha_corr", "logkappa", "logkappa_corr", "logkappa_ref",
+                 "ref_tokens", "expected_len", "row_stats", "weights", "loss", "grad")
+TREE_FIELDS = ("alpha", "accept", "path_accept", "logkappa", "corr_tokens", "deepest",
+               "accept_len", "bonus", "row_stats")
+
+
+class LinearOutputs(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in LINEAR_FIELDS]
+
+
+class TreeOutputs(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in TREE_FIELDS]
+
+
+_LIB = None
+
+
+def library_path():
+    return _build.LIB
+
+
+def _lib():
+    global _LIB
+    if _LIB is None:
+        path = library_path()
+        if not os.path.exists(path):
+            raise RuntimeError("libvsd.so is not built (%s); run __graft_entry__.build()" % path)
+        lib = C.CDLL(path)
+        vp = C.c_void_p
+        lib.vsd_workspace_bytes.argtypes = [Layout]
+        lib.vsd_workspace_bytes.restype = C.c_size_t
+        lib.vsd_sample_paths.argtypes = [vp, C.c_int, Layout, C.c_float, vp, vp, vp, vp, vp,
+                                         C.c_size_t, vp]
+        lib.vsd_verify_paths.argtypes = [vp, vp, C.c_int, Layout, C.c_float, vp, vp, vp, vp,
+                                         C.POINTER(LinearOutputs), C.POINTER(TreeOutputs), vp,
+                                         C.c_size_t, vp]
+        lib.vsd_weighted_loss_fwd_bwd.argtypes = [vp, C.c_int, Layout, C.c_float,
+                                                  C.POINTER(LinearOutputs), C.POINTER(Params),
+                                                  vp, vp, vp, vp, C.c_size_t, vp]
+        lib.vsd_estep_mstep.argtypes = [vp, vp, C.c_int, Layout, C.c_float, vp, vp, vp, vp,
+                                        C.POINTER(Params), C.POINTER(LinearOutputs), vp,
+                                        C.c_size_t, vp]
+        lib.vsd_device_status.argtypes = [vp, vp, C.POINTER(C.c_int32)]
+        lib.vsd_status_string.argtypes = [C.c_int]
+        lib.vsd_status_string.restype = C.c_char_p
+        lib.vsd_version.restype = C.c_char_p
+        for name in ("vsd_sample_paths", "vsd_verify_paths", "vsd_weighted_loss_fwd_bwd",
+                     "vsd_estep_mstep", "vsd_device_status"):
+            getattr(lib, name).restype = C.c_int
+        _LIB = lib
+    return _LIB
+
+
+def load():
+    """Load libvsd.so (raises if it is missing); returns the ctypes handle."""
+    return _lib()
+
+
+def _check(code, where):
+    if code != 0:
+        raise VsdError(code, where)
+
+
+def _dtype_code(t):
+    if t.dtype == torch.float32:
+        return VSD_F32
+    if t.dtype == torch.bfloat16:
+        return VSD_BF16
+    raise TypeError("logits must be float32 or bfloat16, got %s" % t.dtype)
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _stream(device):
+    return C.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _need_cuda(*ts):
+    for t in ts:
+        if t is not None:
+            if not t.is_cuda:
+                raise ValueError("tensors must live on a CUDA device")
+            if not t.is_contiguous():
+                raise ValueError("tensors must be contiguous")
+
+
+def layout(B, K=1, D=1, V=1, N=0, parent=None):
+    return Layout(int(B), int(K), int(D), int(V), int(N),
+                  None if parent is None else parent.data_ptr())
+
+
+def workspace_bytes(lay):
+    n = _lib().vsd_workspace_bytes(lay)
+    if n == 0:
+        raise ValueError("invalid layout")
+    return n
+
+
+def new_workspace(lay, device):
+    return torch.empty(workspace_bytes(lay), dtype=torch.uint8, device=device)
+
+
+def params(w_base=1.05, tau_car=0.2, zeta_mode=0, grad_dtype=None, wait_timeout_ns=0,
+           test_never_publish=0, like=None):
+    if grad_dtype is None:
+        grad_dtype = VSD_BF16 if (like is not None and like.dtype == torch.bfloat16) else VSD_F32
+    elif isinstance(grad_dtype, torch.dtype):
+        grad_dtype = VSD_BF16 if grad_dtype == torch.bfloat16 else VSD_F32
+    return Params(float(w_base), float(tau_car), int(zeta_mode), int(grad_dtype),
+                  int(wait_timeout_ns), int(test_never_publish))
+
+
+def _ws(ws, lay, device):
+    if ws is None:
+        ws = new_workspace(lay, device)
+    elif ws.numel() < workspace_bytes(lay):
+        raise ValueError("workspace too small")
+    return ws
+
+
+def _rows(x, V):
+    if x.numel() % V:
+        raise ValueError("logit tensor size is not a multiple of V")
+    return x.numel() // V
+
+
+def linear_outputs(B, K, D, V, device, grad_dtype=torch.bfloat16, grad=True, full=True):
+    """Allocate the output tensors of the linear E-step / M-step."""
+    R = B * K * D
+    f = dict(device=device)
+    o = dict(tokens=torch.empty(R, dtype=torch.int32, **f),
+             accept_len=torch.empty(B * K, dtype=torch.int32, **f),
+             corr_tokens=torch.empty(R, dtype=torch.int32, **f),
+             logkappa=torch.empty(R, dtype=torch.float32, **f),
+             loss=torch.empty(B + 1, dtype=torch.float32, **f))
+    if full:
+        o.update(logq_tok=torch.empty(R, dtype=torch.float32, **f),
+                 alpha=torch.empty(R, dtype=torch.float32, **f),
+                 accept=torch.empty(R, dtype=torch.uint8, **f),
+                 logq_corr=torch.empty(R, dtype=torch.float32, **f),
+                 alpha_corr=torch.empty(R, dtype=torch.float32, **f),
+                 logkappa_corr=torch.empty(R, dtype=torch.float32, **f),
+                 logkappa_ref=torch.empty(R, dtype=torch.float32, **f),
+                 ref_tokens=torch.empty(R, dtype=torch.int32, **f),
+                 expected_len=torch.empty(B * K, dtype=torch.float32, **f),
+                 row_stats=torch.empty(R, 4, dtype=torch.float32, **f),
+                 weights=torch.empty(B, D, K, 4, dtype=torch.float32, **f))
+    if grad:
+        o["grad"] = torch.empty(R, V, dtype=grad_dtype, **f)
+    return o
+
+
+def _linear_struct(o):
+    return LinearOutputs(*[(o[n].data_ptr() if o.get(n) is not None else None)
+                           for n in LINEAR_FIELDS])
+
+
+def sample_paths(draft, u_draft, K, D, T, workspace=None):
+    """z~ ~ q for every row (Algorithm 1): tokens, log q(z~), row statistics."""
+    _need_cuda(draft, u_draft)
+    V = draft.shape[-1]
+    R = _rows(draft, V)
+    B = R // (K * D)
+    lay = layout(B, K, D, V)
+    dev = draft.device
+    ws = _ws(workspace, lay, dev)
+    out = dict(tokens=torch.empty(R, dtype=torch.int32, device=dev),
+               logq_tok=torch.empty(R, dtype=torch.float32, device=dev),
+               row_stats=torch.empty(R, 4, dtype=torch.float32, device=dev))
+    _check(_lib().vsd_sample_paths(_ptr(draft), _dtype_code(draft), lay, float(T), _ptr(u_draft),
+                                   _ptr(out["tokens"]), _ptr(out["logq_tok"]),
+                                   _ptr(out["row_stats"]), _ptr(ws), ws.numel(), _stream(dev)),
+           "vsd_sample_paths")
+    return out
+
+
+def verify_paths(draft, target, tokens, u_accept, u_correct, K, D, T, ref_logkappa=None,
+                 workspace=None):
+    """Eq. 1 per token, accepted lengths, residual correction, log-kappas."""
+    _need_cuda(draft, target, tokens, u_accept, u_correct, ref_logkappa)
+    V = draft.shape[-1]
+    R = _rows(draft, V)
+    B = R // (K * D)
+    lay = layout(B, K, D, V)
+    dev = draft.device
+    ws = _ws(workspace, lay, dev)
+    o = linear_outputs(B, K, D, V, dev, grad=False)
+    del o["loss"], o["weights"]
+    o["tokens"] = torch.empty(R, dtype=torch.int32, device=dev)
+    st = _linear_struct(o)
+    _check(_lib().vsd_verify_paths(_ptr(draft), _ptr(target), _dtype_code(draft), lay, float(T),
+                                   _ptr(tokens), _ptr(u_accept), _ptr(u_correct),
+                                   _ptr(ref_logkappa), C.byref(st), None, _ptr(ws), ws.numel(),
+                                   _stream(dev)), "vsd_verify_paths")
+    return o
+
+
+def verify_tree(draft, target, parent, tokens, u_accept, u_correct, T, workspace=None):
+    """Tree verification (App. E tree, Eq. 1 per node, Sec. 3 residual)."""
+    _need_cuda(draft, target, parent, tokens, u_accept, u_correct)
+    V = draft.shape[-1]
+    B, N = parent.shape
+    lay = layout(B, V=V, N=N, parent=parent)
+    dev = draft.device
+    ws = _ws(workspace, lay, dev)
+    f = dict(device=dev)
+    o = dict(alpha=torch.empty(B, N, dtype=torch.float32, **f),
+             accept=torch.empty(B, N, dtype=torch.uint8, **f),
+             path_accept=torch.empty(B, N, dtype=torch.uint8, **f),
+             logkappa=torch.empty(B, N, dtype=torch.float32, **f),
+             corr_tokens=torch.empty(B, N, dtype=torch.int32, **f),
+             deepest=torch.empty(B, dtype=torch.int32, **f),
+             accept_len=torch.empty(B, dtype=torch.int32, **f),
+             bonus=torch.empty(B, dtype=torch.int32, **f),
+             row_stats=torch.empty(B * N, 4, dtype=torch.float32, **f))
+    st = TreeOutputs(*[o[n].data_ptr() for n in TREE_FIELDS])
+    _check(_lib().vsd_verify_paths(_ptr(draft), _ptr(target), _dtype_code(draft), lay, float(T),
+                                   _ptr(tokens), _ptr(u_accept), _ptr(u_correct), None, None,
+                                   C.byref(st), _ptr(ws), ws.numel(), _stream(dev)),
+           "vsd_verify_paths(tree)")
+    return o
+
+
+def weighted_loss_fwd_bwd(draft, estep, K, D, T, prm=None, workspace=None, grad=None,
+                          weights=True):
+    """M-step: o~, o', beta, zeta, loss and gradient from E-step results."""
+    _need_cuda(draft)
+    V = draft.shape[-1]
+    R = _rows(draft, V)
+    B = R // (K * D)
+    lay = layout(B, K, D, V)
+    dev = draft.device
+    ws = _ws(workspace, lay, dev)
+    prm = prm or params(like=draft)
+    if grad is None:
+        grad = torch.empty(R, V, dtype=torch.bfloat16 if prm.grad_dtype == VSD_BF16
+                           else torch.float32, device=dev)
+    loss = torch.empty(B + 1, dtype=torch.float32, device=dev)
+    w = torch.empty(B, D, K, 4, dtype=torch.float32, device=dev) if weights else None
+    st = _linear_struct(estep)
+    _check(_lib().vsd_weighted_loss_fwd_bwd(_ptr(draft), _dtype_code(draft), lay, float(T),
+                                            C.byref(st), C.byref(prm), _ptr(loss), _ptr(grad),
+                                            _ptr(w), _ptr(ws), ws.numel(), _stream(dev)),
+           "vsd_weighted_loss_fwd_bwd")
+    return dict(loss=loss, grad=grad, weights=w)
+
+
+def estep_mstep(draft, target, u_draft, u_accept, u_correct, K, D, T, ref_logkappa=None,
+                prm=None, workspace=None, out=None, full=True):
+    """The fused E-step + M-step (one persistent kernel).  Returns the outputs."""
+    _need_cuda(draft, target, u_draft, u_accept, u_correct, ref_logkappa)
+    V = draft.shape[-1]
+    R = _rows(draft, V)
+    B = R // (K * D)
+    lay = layout(B, K, D, V)
+    dev = draft.device
+    ws = _ws(workspace, lay, dev)
+    prm = prm or params(like=draft)
+    if out is None:
+        gdt = torch.bfloat16 if prm.grad_dtype == VSD_BF16 else torch.float32
+        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full)
+    st = _linear_struct(out)
+    _check(_lib().vsd_estep_mstep(_ptr(draft), _ptr(target), _dtype_code(draft), lay, float(T),
+                                  _ptr(u_draft), _ptr(u_accept), _ptr(u_correct),
+                                  _ptr(ref_logkappa), C.byref(prm), C.byref(st), _ptr(ws),
+                                  ws.numel(), _stream(dev)), "vsd_estep_mstep")
+    return out
+
+
+def device_status(workspace):
+    """(status code, status bits) of the last call on this workspace; synchronises."""
+    bits = C.c_int32(0)
+    code = _lib().vsd_device_status(_ptr(workspace), _stream(workspace.device), C.byref(bits))
+    return code, bits.value
+
+
+class HostStep:
+    """End-to-end E-step + M-step from pinned host tensors: per call, copy the
+    inputs to the device, run the fused kernel, read the loss back."""
+
+    def __init__(self, B, K, D, V, dtype, device, prm=None, full=False):
+        self.B, self.K, self.D, self.V = B, K, D, V
+        R = B * K * D
+        self.dev = torch.device(device)
+        self.draft = torch.empty(R, V, dtype=dtype, device=self.dev)
+        self.target = torch.empty(R, V, dtype=dtype, device=self.dev)
+        self.u = torch.empty(3, R, dtype=torch.float32, device=self.dev)
+        self.prm = prm or params(like=self.draft)
+        gdt = torch.bfloat16 if self.prm.grad_dtype == VSD_BF16 else torch.float32
+        self.out = linear_outputs(B, K, D, V, self.dev, grad_dtype=gdt, full=full)
+        self.ws = new_workspace(layout(B, K, D, V), self.dev)
+        self.loss_host = torch.empty(B + 1, dtype=torch.float32).pin_memory()
+
+    def h2d_bytes(self):
+        return (self.draft.numel() * self.draft.element_size() * 2 + self.u.numel() * 4)
+
+    def d2h_bytes(self):
+        return self.loss_host.numel() * 4
+
+    def __call__(self, h_draft, h_target, h_u, T):
+        self.draft.copy_(h_draft, non_blocking=True)
+        self.target.copy_(h_target, non_blocking=True)
+        self.u.copy_(h_u, non_blocking=True)
+        estep_mstep(self.draft, self.target, self.u[0], self.u[1], self.u[2], self.K, self.D, T,
+                    prm=self.prm, workspace=self.ws, out=self.out)
+        self.loss_host.copy_(self.out["loss"], non_blocking=True)
+        return self.loss_host

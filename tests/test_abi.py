@@ -1,0 +1,100 @@
+"""CPU checks of the C ABI: the library builds, loads and exports every symbol
+that include/vsd.h declares; host-side argument checks return the documented
+codes before anything touches a GPU (no compute call is made here)."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def vsd():
+    from paper_2602_05774_gb300 import build, vsd as v
+    build.build_library()
+    v.load()
+    return v
+
+
+def declared_symbols():
+    src = open(os.path.join(ROOT, "include", "vsd.h")).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[\w\s\*]+?\b(vsd_\w+)\s*\(", src, re.M)))
+
+
+def test_header_symbols_exported(vsd):
+    names = declared_symbols()
+    assert len(names) >= 8, names
+    lib = vsd.load()
+    for n in names:
+        assert hasattr(lib, n), "missing export %s" % n
+    assert set(vsd.SYMBOLS) <= set(names)
+
+
+def test_version_and_status_strings(vsd):
+    lib = vsd.load()
+    assert lib.vsd_version().decode().count(".") == 2
+    for code in range(7):
+        assert len(lib.vsd_status_string(code)) > 0
+    assert lib.vsd_status_string(99) == b"unknown status"
+
+
+def test_workspace_bytes(vsd):
+    lay = vsd.layout(32, 16, 8, 128256)
+    n = vsd.workspace_bytes(lay)
+    R = 32 * 16 * 8
+    assert R * 64 < n < R * 400
+    small = vsd.workspace_bytes(vsd.layout(2, 4, 4, 1024))
+    assert 0 < small < n
+    lib = vsd.load()
+    for bad in (vsd.layout(0, 1, 1, 8), vsd.layout(1, 0, 1, 8), vsd.layout(1, 1, 65, 8),
+                vsd.layout(1, 257, 1, 8), vsd.layout(1, 1, 1, (1 << 20) + 1),
+                vsd.layout(1, 1, 1, 0)):
+        assert lib.vsd_workspace_bytes(bad) == 0
+
+
+def test_argument_checks_before_any_launch(vsd):
+    lib = vsd.load()
+    lay = vsd.layout(2, 4, 4, 1024)
+    fake = C.c_void_p(0x1000)  # never dereferenced: every call below fails its checks
+    big = 1 << 30
+    outs = vsd.LinearOutputs()
+    # null pointers
+    assert lib.vsd_sample_paths(None, 0, lay, 1.0, fake, fake, fake, None, fake, big, None) == 1
+    # temperature 0 is unsupported, negative / nan invalid
+    assert lib.vsd_sample_paths(fake, 0, lay, 0.0, fake, fake, fake, None, fake, big, None) == 2
+    assert lib.vsd_sample_paths(fake, 0, lay, -1.0, fake, fake, fake, None, fake, big, None) == 1
+    assert lib.vsd_sample_paths(fake, 0, lay, float("nan"), fake, fake, fake, None, fake, big,
+                                None) == 1
+    # bad dtype
+    assert lib.vsd_sample_paths(fake, 7, lay, 1.0, fake, fake, fake, None, fake, big, None) == 1
+    # workspace too small / missing / misaligned
+    assert lib.vsd_sample_paths(fake, 0, lay, 1.0, fake, fake, fake, None, fake, 16, None) == 5
+    assert lib.vsd_sample_paths(fake, 0, lay, 1.0, fake, fake, fake, None, None, big, None) == 5
+    assert lib.vsd_sample_paths(fake, 0, lay, 1.0, fake, fake, fake, None, C.c_void_p(0x1004),
+                                big, None) == 5
+    # fused: required outputs missing
+    assert lib.vsd_estep_mstep(fake, fake, 1, lay, 1.0, fake, fake, fake, None, None,
+                               C.byref(outs), fake, big, None) == 1
+    # bad M-step parameters
+    o = vsd.LinearOutputs(*([0x1000] * len(vsd.LINEAR_FIELDS)))
+    for prm in (vsd.params(w_base=0.0), vsd.params(tau_car=0.0), vsd.params(zeta_mode=3),
+                vsd.params(grad_dtype=5)):
+        assert lib.vsd_estep_mstep(fake, fake, 1, lay, 1.0, fake, fake, fake, None, C.byref(prm),
+                                   C.byref(o), fake, big, None) == 1
+    # tree layout: reference log-kappa is not accepted, outputs required
+    tlay = vsd.Layout(2, 1, 1, 1024, 60, 0x1000)
+    to = vsd.TreeOutputs()
+    assert lib.vsd_verify_paths(fake, fake, 1, tlay, 1.0, fake, fake, fake, None, None,
+                                C.byref(to), fake, big, None) == 1
+    # linear-only entry points reject a tree layout
+    assert lib.vsd_sample_paths(fake, 1, tlay, 1.0, fake, fake, fake, None, fake, big, None) == 1
+
+
+def test_binding_refuses_cpu_tensors(vsd):
+    torch = pytest.importorskip("torch")
+    x = torch.zeros(4, 8)
+    u = torch.zeros(4)
+    with pytest.raises(ValueError):
+        vsd.sample_paths(x, u, 1, 4, 1.0)

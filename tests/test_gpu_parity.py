@@ -1,0 +1,231 @@
+"""GPU parity: the CUDA path against the CPU oracle on the same seeded inputs.
+
+Runs through the C ABI (Python binding).  Sizes span several chunks and a
+ragged tail; the full vocab128k workload is checked on sampled prefixes, in
+the launch configuration the benchmark times.
+"""
+import numpy as np
+import pytest
+import torch
+
+from tests.parity import compare_linear, compare_tree, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def vsd():
+    from paper_2602_05774_gb300 import build, vsd as v
+    build.build_library()
+    v.load()
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    return v
+
+
+def _np32(t):
+    return t.detach().float().cpu().numpy()
+
+
+def run_oracle(oracle, prob, T, **kw):
+    return oracle.linear(_np32(prob["draft"]), _np32(prob["target"]), T,
+                         _np32(prob["u_draft"]), _np32(prob["u_accept"]),
+                         _np32(prob["u_correct"]), prob["K"], prob["D"], **kw)
+
+
+def to_cuda(prob):
+    return {k: (v.cuda() if torch.is_tensor(v) else v) for k, v in prob.items()}
+
+
+def fused(vsd, p, T, **kw):
+    out = vsd.estep_mstep(p["draft"], p["target"], p["u_draft"], p["u_accept"], p["u_correct"],
+                          p["K"], p["D"], T, **kw)
+    torch.cuda.synchronize()
+    return out
+
+
+@pytest.mark.parametrize("T", [1.0, 0.7])
+def test_tiny_fused_matches_oracle(vsd, oracle, T):
+    from paper_2602_05774_gb300 import inputs
+    prob = inputs.config("tiny")
+    orc = run_oracle(oracle, prob, T)
+    g = fused(vsd, to_cuda(prob), T)
+    compare_linear(g, orc, prob["B"], prob["K"], prob["D"], prob["V"], T, grad_dtype="f32")
+
+
+def test_vocab32k_fused_matches_oracle(vsd, oracle):
+    from paper_2602_05774_gb300 import inputs
+    prob = inputs.config("vocab32k")
+    orc = run_oracle(oracle, prob, 1.0)
+    g = fused(vsd, to_cuda(prob), 1.0)
+    rep = {}
+    compare_linear(g, orc, prob["B"], prob["K"], prob["D"], prob["V"], 1.0, grad_dtype="bf16",
+                   report=rep)
+
+
+SHAPES = [
+    # B, K, D, V, dtype, kind, T
+    (1, 1, 1, 1, "f32", "gauss", 1.0),
+    (2, 3, 2, 2, "f32", "gauss", 0.25),
+    (3, 2, 3, 3, "bf16", "gauss", 2.0),
+    (2, 5, 3, 7, "f32", "gauss", 1.0),
+    (2, 4, 2, 8, "bf16", "gauss", 0.7),
+    (1, 3, 5, 33, "f32", "gauss", 1.0),
+    (2, 2, 3, 1000, "bf16", "gauss", 1.0),
+    (2, 3, 4, 4097, "f32", "gauss", 0.7),
+    (2, 3, 4, 4097, "bf16", "spiked", 1.0),
+    (1, 7, 3, 5000, "bf16", "zipf", 1.0),
+    (3, 1, 6, 2048, "bf16", "spiked", 1.0),
+    (2, 16, 1, 1536, "f32", "gauss", 1.0),
+]
+
+
+@pytest.mark.parametrize("B,K,D,V,dtype,kind,T", SHAPES)
+def test_random_shapes_fused(vsd, oracle, B, K, D, V, dtype, kind, T):
+    from paper_2602_05774_gb300 import inputs
+    prob = inputs.linear_problem(B, K, D, V, dtype, kind, seed=1000 + V + 7 * K + D)
+    orc = run_oracle(oracle, prob, T)
+    g = fused(vsd, to_cuda(prob), T)
+    compare_linear(g, orc, B, K, D, V, T, grad_dtype=dtype)
+
+
+@pytest.mark.parametrize("zeta_mode,ref", [(1, False), (0, True)])
+def test_params_and_reference_input(vsd, oracle, zeta_mode, ref):
+    from paper_2602_05774_gb300 import inputs
+    prob = inputs.linear_problem(3, 4, 3, 3000, "bf16", "spiked", seed=77)
+    refk = None
+    if ref:
+        refk = torch.linspace(-0.5, -3.0, 9).reshape(3, 3).float()
+    orc = run_oracle(oracle, prob, 1.0, zeta_mode=zeta_mode, tau_car=0.5, w_base=1.2,
+                     ref_logkappa=None if refk is None else refk.numpy())
+    p = to_cuda(prob)
+    prm = vsd.params(w_base=1.2, tau_car=0.5, zeta_mode=zeta_mode, grad_dtype=torch.float32)
+    g = fused(vsd, p, 1.0, prm=prm, ref_logkappa=None if refk is None else refk.cuda())
+    compare_linear(g, orc, 3, 4, 3, 3000, 1.0, grad_dtype="f32")
+
+
+def test_draft_equals_target(vsd, oracle):
+    from paper_2602_05774_gb300 import inputs
+    prob = inputs.linear_problem(2, 4, 4, 2500, "bf16", "gauss", seed=5)
+    prob["target"] = prob["draft"].clone()
+    orc = run_oracle(oracle, prob, 1.0)
+    g = fused(vsd, to_cuda(prob), 1.0)
+    assert np.all(to_np(g["alpha"]) == 1.0)
+    assert np.all(to_np(g["accept_len"]) == 4)
+    compare_linear(g, orc, 2, 4, 4, 2500, 1.0, grad_dtype="bf16")
+
+
+def test_one_token_rows(vsd, oracle):
+    """All -inf logits but one token per row (and a few two-token rows)."""
+    B, K, D, V = 2, 3, 3, 3000
+    R = B * K * D
+    gen = torch.Generator().manual_seed(3)
+    draft = torch.full((R, V), float("-inf"))
+    target = torch.full((R, V), float("-inf"))
+    idx = torch.randint(0, V, (R,), generator=gen)
+    draft[torch.arange(R), idx] = 1.0
+    target[torch.arange(R), idx] = 2.0
+    idx2 = torch.randint(0, V, (R,), generator=gen)
+    target[torch.arange(R)[::2], idx2[::2]] = 1.5
+    draft[torch.arange(R)[::3], idx2[::3]] = 0.5
+    prob = dict(B=B, K=K, D=D, V=V, draft=draft, target=target,
+                u_draft=torch.rand(R, generator=gen), u_accept=torch.rand(R, generator=gen),
+                u_correct=torch.rand(R, generator=gen))
+    orc = run_oracle(oracle, prob, 1.0)
+    g = fused(vsd, to_cuda(prob), 1.0, prm=vsd.params(grad_dtype=torch.float32))
+    compare_linear(g, orc, B, K, D, V, 1.0, grad_dtype="f32")
+
+
+def test_separate_entry_points(vsd, oracle):
+    """sample -> verify -> weighted loss, each fed the oracle's own E-step results."""
+    from paper_2602_05774_gb300 import inputs
+    B, K, D, V, T = 3, 4, 3, 5000, 0.8
+    prob = inputs.linear_problem(B, K, D, V, "bf16", "spiked", seed=11)
+    orc = run_oracle(oracle, prob, T)
+    p = to_cuda(prob)
+    s = vsd.sample_paths(p["draft"], p["u_draft"], K, D, T)
+    torch.cuda.synchronize()
+    m = orc["margins"][:, 0] >= 1e-6
+    assert np.array_equal(to_np(s["tokens"])[m], orc["tokens"][m])
+    assert np.allclose(to_np(s["logq_tok"]), orc["logq_tok"], atol=2e-5, rtol=1e-6)
+    tok = torch.from_numpy(orc["tokens"]).cuda()
+    v = vsd.verify_paths(p["draft"], p["target"], tok, p["u_accept"], p["u_correct"], K, D, T)
+    torch.cuda.synchronize()
+    compare_linear(v, orc, B, K, D, V, T, check_grad=False)
+    es = {n: torch.from_numpy(np.ascontiguousarray(orc[n])).cuda() for n in
+          ("tokens", "corr_tokens")}
+    for n in ("logq_tok", "logq_corr", "logkappa", "logkappa_corr", "logkappa_ref"):
+        es[n] = torch.from_numpy(orc[n].astype(np.float32)).cuda()
+    rs = to_np(v["row_stats"])  # statistics of the draft rows (inputs, not decisions)
+    es["row_stats"] = torch.from_numpy(rs).cuda()
+    lo = vsd.weighted_loss_fwd_bwd(p["draft"], es, K, D, T,
+                                   prm=vsd.params(grad_dtype=torch.float32))
+    torch.cuda.synchronize()
+    res = dict(loss=lo["loss"], grad=lo["grad"], weights=lo["weights"],
+               accept_len=torch.from_numpy(orc["accept_len"]),
+               corr_tokens=torch.from_numpy(orc["corr_tokens"]),
+               logkappa=torch.from_numpy(orc["logkappa"].astype(np.float32)))
+    compare_linear(res, orc, B, K, D, V, T, grad_dtype="f32")
+
+
+def test_tree60_matches_oracle(vsd, oracle):
+    from paper_2602_05774_gb300 import inputs
+    prob = inputs.config("tree60")
+    B, N, V = prob["B"], prob["N"], prob["V"]
+    orc = oracle.tree(_np32(prob["draft"]), _np32(prob["target"]), 1.0, prob["parent"].numpy(),
+                      prob["tokens"].numpy(), _np32(prob["u_accept"]), _np32(prob["u_correct"]))
+    p = to_cuda(prob)
+    g = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"], p["u_accept"],
+                        p["u_correct"], 1.0)
+    torch.cuda.synchronize()
+    compare_tree(g, orc)
+
+
+def test_small_trees_matches_oracle(vsd, oracle):
+    from paper_2602_05774_gb300 import inputs
+    for (B, N, depth, topk, V, seed) in [(3, 12, 4, 3, 777, 1), (2, 30, 6, 5, 4096, 2),
+                                         (1, 2, 1, 1, 9, 3)]:
+        prob = inputs.tree_problem(B, N, depth, topk, V, seed=seed)
+        orc = oracle.tree(_np32(prob["draft"]), _np32(prob["target"]), 0.9,
+                          prob["parent"].numpy(), prob["tokens"].numpy(),
+                          _np32(prob["u_accept"]), _np32(prob["u_correct"]))
+        p = to_cuda(prob)
+        g = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"], p["u_accept"],
+                            p["u_correct"], 0.9)
+        torch.cuda.synchronize()
+        compare_tree(g, orc)
+
+
+@pytest.mark.parametrize("T", [1.0, 0.7])
+def test_vocab128k_full_size_sampled_prefixes(vsd, oracle, T):
+    """The benchmark's workload and launch; the oracle checks two sampled prefixes."""
+    from paper_2602_05774_gb300 import inputs
+    prob = inputs.config("vocab128k", device="cuda")
+    B, K, D, V = prob["B"], prob["K"], prob["D"], prob["V"]
+    g = fused(vsd, prob, T)
+    P = K * D
+    # properties at full size: gradient rows sum to ~0, loss finite
+    grad = g["grad"]
+    rs = grad.float().sum(dim=1)
+    assert torch.isfinite(g["loss"]).all()
+    assert rs.abs().max().item() < 1e-3
+    for b in (0, B - 1) if T == 1.0 else (B // 2,):
+        rows = slice(b * P, (b + 1) * P)
+        sub = dict(B=1, K=K, D=D, V=V, draft=prob["draft"][rows], target=prob["target"][rows],
+                   u_draft=prob["u_draft"][rows], u_accept=prob["u_accept"][rows],
+                   u_correct=prob["u_correct"][rows])
+        orc = run_oracle(oracle, sub, T)
+        # the oracle's loss normalises over its own batch of 1: rescale the grad
+        orc["grad"] = orc["grad"] / B
+        gsub = {}
+        for n, t in g.items():
+            if t is None:
+                continue
+            if n in ("accept_len", "expected_len"):
+                gsub[n] = t[b * K:(b + 1) * K]
+            elif n == "weights":
+                gsub[n] = t[b:b + 1]
+            elif n == "loss":
+                gsub[n] = torch.stack([t[b], t[b]])
+            elif t.shape[0] == B * P:
+                gsub[n] = t[rows]
+        compare_linear(gsub, orc, 1, K, D, V, T, grad_dtype="bf16")
