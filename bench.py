@@ -37,6 +37,9 @@ def parse():
     ap.add_argument("--config", default="vocab128k", choices=WORKLOADS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--prefixes", type=int, default=0,
+                    help="run only the first B prefixes of the workload (small profiling "
+                         "captures); 0 = all")
     return ap.parse_args()
 
 
@@ -210,6 +213,12 @@ def run_ours(args):
     c = inputs.CONFIGS[args.config]
     seed = inputs.BASE_SEED + list(inputs.CONFIGS).index(args.config) + 1000 * rank
     prob = inputs.config(args.config, device=dev, seed=seed)
+    if args.prefixes and args.prefixes < prob["B"]:
+        P = prob["K"] * prob["D"]
+        n = args.prefixes * P
+        for k in ("draft", "target", "u_draft", "u_accept", "u_correct"):
+            prob[k] = prob[k][:n].contiguous()
+        prob["B"] = args.prefixes
     B, K, D, V = prob["B"], prob["K"], prob["D"], prob["V"]
     R = B * K * D
     temps = c["T"]

@@ -130,8 +130,9 @@ typedef struct {
 /* margins[r][0]: draft sample, |u - nearest CDF boundary| of q
  * margins[r][1]: accept, |u_accept - alpha|
  * margins[r][2]: correction sample of z'_d (residual or p), +inf if none
- * margins[r][3]: o~ at l=d+1, |log k(z~) - log k(z-bar)|
- * margins[r][4]: o' at l=d+1 when o~=0, |log k(z') - log k(z-bar)|, else +inf
+ * margins[r][3]: o~ at l=d+1: decision_margin(log k(z~), log k(z-bar))
+ * margins[r][4]: o' at l=d+1 when o~=0: decision_margin(log k(z'), log k(z-bar)),
+ *                else +inf
  * margins[r][5]: alpha of the correction token, |alpha' - 1| is not a
  *                decision; kept +inf (reserved) */
 
@@ -268,6 +269,31 @@ double vso_prefix_objective(const float* draft, int K, int D, int64_t V, double 
     return J;
 }
 
+/* Margin of the decision log k(a_{<=l}) >= log k(b_{<=l}) (Algorithm 2), for
+ * counting near-boundary decisions in tests.  log k is a sum of clipped
+ * log-ratios min(0, r_i).  Unequal sums: the gap.  Equal sums: the decision
+ * is exact when, at every position where the two paths hold different
+ * tokens, both log-ratios are clipped (r >= 0); its margin is then the
+ * smallest such r; any other equality is a coincidence (margin 0).  With an
+ * input reference (rb == NULL) the sum b is a constant. */
+static double decision_margin(double a, double b, int n, const double* ra, const int32_t* ta,
+                              const double* rb, const int32_t* tb)
+{
+    if (a != b) return fabs(a - b);
+    double m = INFINITY;
+    for (int i = 0; i < n; ++i) {
+        if (rb && ta[i] == tb[i]) continue; /* identical terms cancel exactly */
+        if (ra[i] < 0.0) return 0.0;
+        if (ra[i] < m) m = ra[i];
+        if (rb) {
+            if (rb[i] < 0.0) return 0.0;
+            if (rb[i] < m) m = rb[i];
+        }
+    }
+    if (!rb && b != 0.0) return 0.0;
+    return m;
+}
+
 /* ------------------------------------------------------------------ */
 /* Public: the whole E-step + M-step for linear paths.  Returns 0 on success,
  * nonzero on an invalid argument. */
@@ -287,6 +313,10 @@ int vso_linear(const vso_linear_in* in, vso_linear_out* out)
     double* lkc = (double*)malloc(sizeof(double) * (size_t)(K * D));
     double* lkr = (double*)malloc(sizeof(double) * (size_t)(K * D));
     double* lqpath = (double*)malloc(sizeof(double) * (size_t)(K * D));
+    /* unclipped log-ratios log(p/q) at z~, z', v-bar (for decision margins) */
+    double* rt = (double*)malloc(sizeof(double) * (size_t)(K * D));
+    double* rc = (double*)malloc(sizeof(double) * (size_t)(K * D));
+    double* rr = (double*)malloc(sizeof(double) * (size_t)(K * D));
     double loss_sum = 0.0;
 
     for (int b = 0; b < B; ++b) {
@@ -328,6 +358,8 @@ int vso_linear(const vso_linear_in* in, vso_linear_out* out)
                 double ab = p[vb] / q[vb];
                 if (ab > 1.0) ab = 1.0;
                 out->ref_tokens[r] = (int32_t)vb;
+                rt[s * D + d] = log(p[zt] / q[zt]);
+                rr[s * D + d] = log(p[vb] / q[vb]);
                 /* prefix sums over l: log k(z~_{<=l}) = sum_{i<=l} log alpha_i (Eq. 2) */
                 double prev = d ? lk[s * D + d - 1] : 0.0;
                 lk[s * D + d] = prev + log(alpha);
@@ -375,6 +407,7 @@ int vso_linear(const vso_linear_in* in, vso_linear_out* out)
                 out->corr_tokens[r] = (int32_t)zc;
                 out->logq_corr[r] = lq[zc];
                 out->alpha_corr[r] = ac;
+                rc[s * D + d] = log(p[zc] / q[zc]);
                 if (out->margins) out->margins[6 * r + 2] = mg;
                 double prev = d ? lkc[s * D + d - 1] : 0.0;
                 lkc[s * D + d] = prev + log(ac);
@@ -395,13 +428,22 @@ int vso_linear(const vso_linear_in* in, vso_linear_out* out)
         double N = vso_prefix_weights(K, D, lk, lkc, lkr, lqpath, in->w_base, in->tau_car,
                                       in->zeta_mode, wb);
         if (out->margins) {
+            const int32_t* tz = out->tokens + (size_t)b * K * D;
+            const int32_t* tc = out->corr_tokens + (size_t)b * K * D;
+            const int32_t* tr = out->ref_tokens + (size_t)b * K * D;
+            const int refin = in->ref_logkappa != NULL;
             for (int s = 0; s < K; ++s)
                 for (int d = 0; d < D; ++d) {
                     const size_t r = ((size_t)b * K + s) * D + d;
-                    out->margins[6 * r + 3] = fabs(lk[s * D + d] - lkr[s * D + d]);
-                    out->margins[6 * r + 4] = wb[((size_t)d * K + s) * 4 + 0] > 0.0
-                                                  ? INFINITY
-                                                  : fabs(lkc[s * D + d] - lkr[s * D + d]);
+                    const int o = s * D;
+                    out->margins[6 * r + 3] =
+                        decision_margin(lk[o + d], lkr[o + d], d + 1, rt + o, tz + o,
+                                        refin ? NULL : rr + o, tr + o);
+                    out->margins[6 * r + 4] =
+                        wb[((size_t)d * K + s) * 4 + 0] > 0.0
+                            ? INFINITY
+                            : decision_margin(lkc[o + d], lkr[o + d], d + 1, rc + o, tc + o,
+                                              refin ? NULL : rr + o, tr + o);
                 }
         }
         const size_t rb = (size_t)b * K * D;
@@ -414,7 +456,7 @@ int vso_linear(const vso_linear_in* in, vso_linear_out* out)
     }
     out->loss[B] = loss_sum / (double)B;
     free(lq); free(lp); free(q); free(p); free(res);
-    free(lk); free(lkc); free(lkr); free(lqpath);
+    free(lk); free(lkc); free(lkr); free(lqpath); free(rt); free(rc); free(rr);
     return 0;
 }
 

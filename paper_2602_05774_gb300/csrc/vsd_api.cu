@@ -23,7 +23,7 @@ constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct WsLayout {
-    size_t status, ticket, prefix_done, path_cnt, prefix_cnt, ready, zero_end;
+    size_t status, ticket, prefix_done, grad_head, path_cnt, prefix_cnt, ready, grad_cnt, zero_end;
     size_t rows, rstats, es_tok, es_corr, es_lq_tok, es_lq_corr, es_lk, es_lkc, es_lkr;
     size_t coef, wscr, total;
 };
@@ -50,10 +50,12 @@ WsLayout ws_layout(const vsd_layout& L) {
     w.status = 0;
     w.ticket = 4;
     w.prefix_done = 8;
+    w.grad_head = 12;
     o = 256;
     w.path_cnt = o; o = align256(o + 4 * npath);
     w.prefix_cnt = o; o = align256(o + 4 * (size_t)L.B);
     w.ready = o; o = align256(o + 4 * (size_t)L.B);
+    w.grad_cnt = o; o = align256(o + 4 * (size_t)L.B);
     w.zero_end = o;
     w.rows = o; o = align256(o + sizeof(RowRec) * R);
     w.rstats = o; o = align256(o + sizeof(float4) * R);
@@ -81,13 +83,6 @@ int num_sms() {
     if (cudaGetDevice(&dev) != cudaSuccess) return 1;
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 1;
     return n > 0 ? n : 1;
-}
-
-size_t l2_bytes() {
-    int dev = 0, n = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrL2CacheSize, dev) != cudaSuccess) return 0;
-    return (size_t)n;
 }
 
 vsd_status check_temperature(float T) {
@@ -153,6 +148,8 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.path_cnt = at<int>(ws, w.path_cnt);
     P.prefix_cnt = at<int>(ws, w.prefix_cnt);
     P.ready = at<int>(ws, w.ready);
+    P.grad_cnt = at<int>(ws, w.grad_cnt);
+    P.grad_head = at<int>(ws, w.grad_head);
     P.rows = at<RowRec>(ws, w.rows);
     P.rstats = at<float4>(ws, w.rstats);
     P.es.tok = at<int32_t>(ws, w.es_tok);
@@ -266,19 +263,6 @@ vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float
     if ((int64_t)ctas > tickets) ctas = (int)tickets;
     const char* env_ctas = getenv("VSD_FUSED_CTAS");
     if (env_ctas && atoi(env_ctas) > 0 && atoi(env_ctas) < ctas) ctas = atoi(env_ctas);
-    // Rows of `lag` prefixes are scheduled ahead of a prefix's gradient rows:
-    // enough independent work to cover the blocks in flight, capped so that
-    // the draft rows still to be re-read fit comfortably in L2.
-    const int Pp = P.K * P.D;
-    int lag = (2 * ctas + Pp - 1) / Pp;
-    const size_t l2 = l2_bytes();
-    const size_t prefix_bytes = (size_t)Pp * (size_t)L.V * sizeof(T);
-    while (lag > 1 && l2 && (size_t)(lag + 1) * prefix_bytes > (l2 * 3) / 5) --lag;
-    if (lag < 1) lag = 1;
-    const char* env_lag = getenv("VSD_FUSED_LAG");
-    if (env_lag && atoi(env_lag) > 0) lag = atoi(env_lag);
-    if (lag > P.B - 1) lag = P.B - 1 > 0 ? P.B - 1 : 0;
-    P.lag = lag;
     cudaError_t e = clear_counters(ws, L, s);
     if (e == cudaSuccess) e = Launch<T>::fused(P, vec, out->grad, P.grad_bf16, ctas, s);
     return from_cuda(e);

@@ -83,13 +83,16 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int* status, uint64_t
     }
 }
 
-// Persistent E-step + M-step.  Blocks take tickets in order (schedule_block):
-// a row ticket streams one logit row; the block that completes the last row
-// of a path runs its path pass, the block that completes the last path of a
-// prefix runs the prefix's M-step and publishes it; a gradient ticket waits
-// (bounded) for its prefix and writes one gradient row.  Every wait is on
-// work claimed by an earlier ticket, and no such work waits, so progress does
-// not depend on how many blocks are resident.
+// Persistent E-step + M-step.  Each block repeatedly takes the next work item:
+// a gradient row of the oldest prefix whose M-step is already published, if
+// any is left; otherwise the next logit row (rows in prefix order).  A row item
+// streams one draft/target row; the block that completes the last row of a
+// path runs its path pass; the block that completes the last path of a
+// prefix runs the prefix's M-step and publishes it.  A block waits (bounded)
+// only once every row has been claimed; claimed rows are finished by running
+// blocks that never wait, so progress does not depend on residency.  Gradient
+// rows follow their prefix closely, so the draft rows they re-read are still
+// in L2.
 template <typename T, bool VEC, typename G>
 __global__ void __launch_bounds__(kThreads, 2) k_fused(Problem<T> P, G* grad) {
     extern __shared__ float4 tab[];
@@ -98,20 +101,40 @@ __global__ void __launch_bounds__(kThreads, 2) k_fused(Problem<T> P, G* grad) {
         PathShared path;
         WeightsShared w;
     } sh;
-    __shared__ int s_ticket, s_flag;
+    __shared__ int s_kind, s_idx, s_flag;
     const int Pp = P.K * P.D;
-    const int total = 2 * P.B * Pp;
+    const int B = P.B;
     const EStepView E{P.es.tok, P.es.corr, P.es.lq_tok, P.es.lq_corr,
                       P.es.lk, P.es.lkc, P.es.lkr};
     for (;;) {
-        if (threadIdx.x == 0) s_ticket = atomicAdd(P.ticket, 1);
+        if (threadIdx.x == 0) {
+            int kind = 0, idx = 0;  // 0: finished, 1: logit row, 2: gradient row
+            int g = *(volatile int*)P.grad_head;
+            for (;;) {
+                while (g < B && ld_acquire(P.ready + g)) {
+                    const int t = atomicAdd(P.grad_cnt + g, 1);
+                    if (t < Pp) { kind = 2; idx = g * Pp + t; break; }
+                    atomicMax(P.grad_head, g + 1);
+                    ++g;
+                }
+                if (kind) break;
+                const int t = atomicAdd(P.ticket, 1);
+                if (t < P.R) { kind = 1; idx = t; break; }
+                if (g >= B) break;
+                if (!wait_flag(P.ready + g, P.status, P.timeout_ns)) {
+                    atomicOr(P.status, VSD_STATUS_TIMEOUT);
+                    break;
+                }
+            }
+            s_kind = kind;
+            s_idx = idx;
+        }
         __syncthreads();
-        const int t = s_ticket;
+        const int kind = s_kind, r = s_idx;
         __syncthreads();
-        if (t >= total) break;
-        const Item it = schedule_block(t / Pp, P.B, P.lag);
-        const int r = it.prefix * Pp + (t % Pp);
-        if (!it.grad) {
+        if (kind == 0) break;
+        if (kind == 1) {
+            const int prefix = r / Pp;
             row_pass<T, VEC, true, kSampleToken, true>(P, r, tab, sh.row);
             const int path = r / P.D;
             if (threadIdx.x == 0) {
@@ -125,16 +148,16 @@ __global__ void __launch_bounds__(kThreads, 2) k_fused(Problem<T> P, G* grad) {
                 __syncthreads();
                 if (threadIdx.x == 0) {
                     __threadfence();
-                    s_flag = atomicAdd(P.prefix_cnt + it.prefix, 1) == P.K - 1;
+                    s_flag = atomicAdd(P.prefix_cnt + prefix, 1) == P.K - 1;
                     if (s_flag) __threadfence();
                 }
                 __syncthreads();
                 if (s_flag) {
-                    weights_pass<T>(P, E, it.prefix, P.out.weights, P.out.loss, sh.w);
+                    weights_pass<T>(P, E, prefix, P.out.weights, P.out.loss, sh.w);
                     __syncthreads();
                     if (threadIdx.x == 0) {
                         __threadfence();
-                        if (!P.inject_wait_fault) st_release(P.ready + it.prefix, 1);
+                        if (!P.inject_wait_fault) st_release(P.ready + prefix, 1);
                         if (atomicAdd(P.prefix_done, 1) == P.B - 1) {
                             __threadfence();
                             loss_mean(P.out.loss, P.B);
@@ -143,13 +166,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_fused(Problem<T> P, G* grad) {
                 }
             }
         } else {
-            if (threadIdx.x == 0) {
-                const bool ok = wait_flag(P.ready + it.prefix, P.status, P.timeout_ns);
-                if (!ok) atomicOr(P.status, VSD_STATUS_TIMEOUT);
-                s_flag = ok;
-            }
-            __syncthreads();
-            if (s_flag) grad_pass<T, VEC, G>(P, r, P.rstats, grad);
+            grad_pass<T, VEC, G>(P, r, P.rstats, grad);
         }
         __syncthreads();
     }

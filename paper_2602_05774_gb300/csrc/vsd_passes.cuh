@@ -114,12 +114,13 @@ struct Problem {
     int* path_cnt;                // [B*K]
     int* prefix_cnt;              // [B]
     int* ready;                   // [B]
+    int* grad_cnt;                // [B] gradient rows claimed per prefix
+    int* grad_head;               // oldest prefix that may have unclaimed gradient rows
     RowRec* rows;                 // [R]
     float4* rstats;               // [R] m_q, logZ_q, m_p, logZ_p (float copy of rows[])
     EStepStore es;                // [R] each
     Coef* coef;                   // [R]
     double2* wscr;                // [R] M-step scratch
-    int lag;                      // fused schedule: prefixes of rows ahead of gradients
     // outputs (device, caller-owned; null = not written)
     vsd_linear_outputs out;
     vsd_tree_outputs tout;
@@ -395,6 +396,7 @@ struct RowShared {
     float Mx, My;
     double Zx, Zy;
     int tok, ps, ref;
+    float lq[3], la[3];
 };
 
 enum XMode { kNoToken = 0, kSampleToken = 1, kGivenToken = 2 };
@@ -444,43 +446,55 @@ __device__ void row_pass(const Problem<T>& P, int r, float4* tab, RowShared& sh)
         if (lane == 0) sh.ref = ref < V ? ref : -1;
     }
     __syncthreads();
+    // log q and log alpha of z~, of the p-draw and of the argmax: one lane each.
+    const double Td = P.ts.Td;
+    const bool okx = row_ok(sh.Mx, sh.Zx);
+    const bool oky = HAS_Y ? row_ok(sh.My, sh.Zy) : true;
+    const bool ok = okx && oky;
+    const int tok = XMODE == kNoToken ? -1 : sh.tok;
+    const bool tok_ok = tok >= 0 && tok < V;
+    if (threadIdx.x < 3) {
+        const int which = threadIdx.x;
+        const int v = which == 0 ? tok : (which == 1 ? sh.ps : sh.ref);
+        float lq = -INFINITY, la = -INFINITY;
+        const bool want = which == 0 || (HAS_Y && (which == 1 || ARGMAX));
+        if (want && ok && v >= 0 && v < V) {
+            RowRec tmp;
+            tmp.mx = sh.Mx;
+            tmp.lzx = log(sh.Zx);
+            tmp.my = HAS_Y ? sh.My : 0.f;
+            tmp.lzy = HAS_Y ? log(sh.Zy) : 0.0;
+            if (HAS_Y)
+                token_logs(x, y, v, tmp, Td, &lq, &la);
+            else
+                lq = (float)(((double)elem_value(x, v) - (double)tmp.mx) / Td - tmp.lzx);
+        }
+        sh.lq[which] = lq;
+        sh.la[which] = la;
+    }
+    __syncthreads();
     if (threadIdx.x == 0) {
         RowRec rec;
-        const double Td = P.ts.Td;
-        const bool okx = row_ok(sh.Mx, sh.Zx);
-        const bool oky = HAS_Y ? row_ok(sh.My, sh.Zy) : true;
-        const bool ok = okx && oky;
         rec.mx = sh.Mx;
         rec.lzx = okx ? log(sh.Zx) : 0.0;
         rec.my = HAS_Y ? sh.My : 0.f;
         rec.lzy = (HAS_Y && oky) ? log(sh.Zy) : 0.0;
         rec.flags = ok ? 0 : 1;
         if (!ok) atomicOr(P.status, VSD_STATUS_BAD_ROW);
-        int tok = XMODE == kNoToken ? -1 : sh.tok;
-        if (XMODE == kGivenToken && (tok < 0 || tok >= V)) {
+        int t = tok;
+        if (XMODE == kGivenToken && !tok_ok) {
             atomicOr(P.status, VSD_STATUS_BAD_TOKEN);
-            tok = -1;
+            t = -1;
             rec.flags |= 2;
         }
-        rec.tok = tok;
-        rec.lq_tok = rec.la_tok = rec.lq_ps = rec.la_ps = rec.la_ref = -INFINITY;
-        rec.ps = -1;
-        rec.ref = -1;
-        if (ok && tok >= 0) {
-            if (HAS_Y)
-                token_logs(x, y, tok, rec, Td, &rec.lq_tok, &rec.la_tok);
-            else
-                rec.lq_tok = (float)(((double)elem_value(x, tok) - (double)rec.mx) / Td - rec.lzx);
-        }
-        if (HAS_Y && ok) {
-            rec.ps = sh.ps;
-            if (sh.ps >= 0) token_logs(x, y, sh.ps, rec, Td, &rec.lq_ps, &rec.la_ps);
-            if (ARGMAX) {
-                rec.ref = sh.ref;
-                float lqr;
-                if (sh.ref >= 0) token_logs(x, y, sh.ref, rec, Td, &lqr, &rec.la_ref);
-            }
-        }
+        rec.tok = t;
+        rec.lq_tok = (ok && t >= 0) ? sh.lq[0] : -INFINITY;
+        rec.la_tok = (ok && t >= 0) ? sh.la[0] : -INFINITY;
+        rec.ps = (HAS_Y && ok) ? sh.ps : -1;
+        rec.lq_ps = (HAS_Y && ok) ? sh.lq[1] : -INFINITY;
+        rec.la_ps = (HAS_Y && ok) ? sh.la[1] : -INFINITY;
+        rec.ref = (HAS_Y && ARGMAX && ok) ? sh.ref : -1;
+        rec.la_ref = (HAS_Y && ARGMAX && ok) ? sh.la[2] : -INFINITY;
         P.rows[r] = rec;
         P.rstats[r] = make_float4(rec.mx, (float)rec.lzx, rec.my, (float)rec.lzy);
     }
@@ -495,11 +509,20 @@ __device__ void stream_residual(const T* x, const T* y, int64_t V, int nch, floa
     constexpr int PV = Traits<T>::kPerVec;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint64_t pol = policy_evict_normal();
-    for (int ch = warp; ch < nch; ch += kWarps) {
-        uint4 bx[kLoads], by[kLoads];
+    int ch = warp;
+    uint4 bx[kLoads], by[kLoads];
+    if (ch < nch) {
         load_chunk<T, VEC>(x, V, ch, lane, pol, bx);
         load_chunk<T, VEC>(y, V, ch, lane, pol, by);
-        float s[kLoads];
+    }
+    while (ch < nch) {
+        const int cn = ch + kWarps;
+        uint4 nx[kLoads], ny[kLoads];
+        if (cn < nch) {
+            load_chunk<T, VEC>(x, V, cn, lane, pol, nx);
+            load_chunk<T, VEC>(y, V, cn, lane, pol, ny);
+        }
+        float s4[kLoads];
 #pragma unroll
         for (int k = 0; k < kLoads; ++k) {
             float fx[PV], fy[PV];
@@ -508,10 +531,16 @@ __device__ void stream_residual(const T* x, const T* y, int64_t V, int nch, floa
             float a = 0.f;
 #pragma unroll
             for (int e = 0; e < PV; ++e) a += mr(fx[e], fy[e]);
-            s[k] = a;
+            s4[k] = a;
         }
-        const float t = warp_sum((s[0] + s[1]) + (s[2] + s[3]));
+        const float t = warp_sum((s4[0] + s4[1]) + (s4[2] + s4[3]));
         if (lane == 0) tab[ch] = make_float4(0.f, t, 0.f, 0.f);
+#pragma unroll
+        for (int k = 0; k < kLoads; ++k) {
+            bx[k] = nx[k];
+            by[k] = ny[k];
+        }
+        ch = cn;
     }
 }
 
@@ -577,22 +606,31 @@ struct PathShared {
     RowRec rec;
 };
 
-// Linear proposal path (b, s) = path: rows path*D .. path*D + D - 1.
+// Linear proposal path (b, s) = path: rows path*D .. path*D + D - 1.  Warp 0
+// handles the rows lane-parallel (two rounds when D > 32) with warp scans for
+// the prefix sums over l; the whole block streams the residual row.
 template <typename T, bool VEC>
 __device__ void path_pass(const Problem<T>& P, int path, float4* tab, PathShared& sh) {
     const int D = P.D;
     const int r0 = path * D;
-    if (threadIdx.x == 0) {
-        int A = 0;
-        bool still = true;
-        for (int d = 0; d < D; ++d) {
-            const RowRec rec = ld_cg(P.rows + r0 + d);
-            const double a = rec.flags ? 0.0 : exp((double)rec.la_tok);
-            const bool acc = !rec.flags && (double)__ldg(P.u_accept + r0 + d) <= a;
-            if (still && acc) A = d + 1; else still = false;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (warp == 0) {
+        int A = D;
+        for (int d0 = 0; d0 < D; d0 += 32) {
+            const int d = d0 + lane;
+            bool rej = false;
+            if (d < D) {
+                const RowRec rec = ld_cg(P.rows + r0 + d);
+                const double a = rec.flags ? 0.0 : exp((double)rec.la_tok);
+                rej = rec.flags || !((double)__ldg(P.u_accept + r0 + d) <= a);
+            }
+            const unsigned bal = __ballot_sync(0xffffffffu, rej);
+            if (bal && A == D) A = d0 + __ffs(bal) - 1;
         }
-        sh.A = A;
-        if (A < D) sh.rec = ld_cg(P.rows + r0 + A);
+        if (lane == 0) {
+            sh.A = A;
+            if (A < D) sh.rec = ld_cg(P.rows + r0 + A);
+        }
     }
     __syncthreads();
     const int A = sh.A;
@@ -600,64 +638,81 @@ __device__ void path_pass(const Problem<T>& P, int path, float4* tab, PathShared
     if (A < D && !sh.rec.flags)
         resid = residual_draw<T, VEC>(P, r0 + A, sh.rec, __ldg(P.u_correct + r0 + A), tab,
                                       &sh.resid);
-    if (threadIdx.x == 0) {
+    if (warp == 0) {
         const int b = path / P.K;
         const double NEG = -INFINITY;
-        double lk = 0.0, lkc = 0.0, lkr = 0.0, EA = 0.0;
         const int64_t V = P.V;
         const vsd_linear_outputs& o = P.out;
-        for (int d = 0; d < D; ++d) {
-            const int r = r0 + d;
-            const RowRec rec = ld_cg(P.rows + r);
-            const double a = rec.flags ? 0.0 : exp((double)rec.la_tok);
-            const bool acc = !rec.flags && (double)__ldg(P.u_accept + r) <= a;
-            int zc;
-            float lqc, lac;
-            if (d < A) {
-                zc = rec.tok; lqc = rec.lq_tok; lac = rec.la_tok;
-            } else if (d == A) {
-                zc = resid >= 0 ? resid : rec.ps;  // no residual mass: draw from p (R10)
-                if (zc == rec.ps) {
-                    lqc = rec.lq_ps; lac = rec.la_ps;
+        double ck = 0.0, ckc = 0.0, ckr = 0.0, EA = 0.0;
+        for (int d0 = 0; d0 < D; d0 += 32) {
+            const int d = d0 + lane;
+            const bool act = d < D;
+            const int r = r0 + (act ? d : 0);
+            RowRec rec;
+            if (act) rec = ld_cg(P.rows + r);
+            double a = 0.0, tk = 0.0, tkc = 0.0, tkr = 0.0;
+            bool acc = false;
+            int zc = -1;
+            float lqc = -INFINITY, lac = -INFINITY;
+            if (act) {
+                a = rec.flags ? 0.0 : exp((double)rec.la_tok);
+                acc = !rec.flags && (double)__ldg(P.u_accept + r) <= a;
+                if (d < A) {
+                    zc = rec.tok; lqc = rec.lq_tok; lac = rec.la_tok;
+                } else if (d == A) {
+                    zc = resid >= 0 ? resid : rec.ps;  // no residual mass: draw from p (R10)
+                    if (zc == rec.ps) {
+                        lqc = rec.lq_ps; lac = rec.la_ps;
+                    } else {
+                        token_logs(P.draft + (int64_t)r * V, P.target + (int64_t)r * V, zc, rec,
+                                   P.ts.Td, &lqc, &lac);
+                    }
                 } else {
-                    token_logs(P.draft + (int64_t)r * V, P.target + (int64_t)r * V, zc, rec,
-                               P.ts.Td, &lqc, &lac);
+                    zc = rec.ps; lqc = rec.lq_ps; lac = rec.la_ps;
                 }
-            } else {
-                zc = rec.ps; lqc = rec.lq_ps; lac = rec.la_ps;
+                if (rec.flags) { zc = -1; lqc = lac = -INFINITY; }
+                tk = rec.flags ? NEG : (double)rec.la_tok;
+                tkc = zc >= 0 ? (double)lac : NEG;
+                tkr = rec.ref >= 0 ? (double)rec.la_ref : NEG;
             }
-            if (rec.flags) { zc = -1; lqc = lac = -INFINITY; }
-            lk += rec.flags ? NEG : (double)rec.la_tok;
-            lkc += zc >= 0 ? (double)lac : NEG;
-            if (P.ref_logkappa)
-                lkr = (double)__ldg(P.ref_logkappa + (int64_t)b * D + d);
-            else
-                lkr += rec.ref >= 0 ? (double)rec.la_ref : NEG;
-            EA += exp(lk);
-            P.es.tok[r] = rec.tok;
-            P.es.corr[r] = zc;
-            P.es.lq_tok[r] = rec.lq_tok;
-            P.es.lq_corr[r] = lqc;
-            P.es.lk[r] = (float)lk;
-            P.es.lkc[r] = (float)lkc;
-            P.es.lkr[r] = (float)lkr;
-            if (o.tokens) o.tokens[r] = rec.tok;
-            if (o.logq_tok) o.logq_tok[r] = rec.lq_tok;
-            if (o.alpha) o.alpha[r] = (float)a;
-            if (o.accept) o.accept[r] = acc ? 1 : 0;
-            if (o.corr_tokens) o.corr_tokens[r] = zc;
-            if (o.logq_corr) o.logq_corr[r] = lqc;
-            if (o.alpha_corr) o.alpha_corr[r] = zc >= 0 ? (float)exp((double)lac) : 0.f;
-            if (o.logkappa) o.logkappa[r] = (float)lk;
-            if (o.logkappa_corr) o.logkappa_corr[r] = (float)lkc;
-            if (o.logkappa_ref) o.logkappa_ref[r] = (float)lkr;
-            if (o.ref_tokens) o.ref_tokens[r] = rec.ref;
-            if (o.row_stats)
-                reinterpret_cast<float4*>(o.row_stats)[r] =
-                    make_float4(rec.mx, (float)rec.lzx, rec.my, (float)rec.lzy);
+            // prefix sums over l (Eq. 2): log kappa of z~, z' and the reference
+            const double lk = ck + warp_incl_scan(tk, lane);
+            const double lkc = ckc + warp_incl_scan(tkc, lane);
+            double lkr = ckr + warp_incl_scan(tkr, lane);
+            if (P.ref_logkappa && act) lkr = (double)__ldg(P.ref_logkappa + (int64_t)b * D + d);
+            EA += warp_sum(act ? exp(lk) : 0.0);  // Eq. 11
+            const int lastl = min(31, D - 1 - d0);
+            ck = __shfl_sync(0xffffffffu, lk, lastl);
+            ckc = __shfl_sync(0xffffffffu, lkc, lastl);
+            ckr = __shfl_sync(0xffffffffu, ckr + warp_incl_scan(tkr, lane), lastl);
+            if (act) {
+                P.es.tok[r] = rec.tok;
+                P.es.corr[r] = zc;
+                P.es.lq_tok[r] = rec.lq_tok;
+                P.es.lq_corr[r] = lqc;
+                P.es.lk[r] = (float)lk;
+                P.es.lkc[r] = (float)lkc;
+                P.es.lkr[r] = (float)lkr;
+                if (o.tokens) o.tokens[r] = rec.tok;
+                if (o.logq_tok) o.logq_tok[r] = rec.lq_tok;
+                if (o.alpha) o.alpha[r] = (float)a;
+                if (o.accept) o.accept[r] = acc ? 1 : 0;
+                if (o.corr_tokens) o.corr_tokens[r] = zc;
+                if (o.logq_corr) o.logq_corr[r] = lqc;
+                if (o.alpha_corr) o.alpha_corr[r] = zc >= 0 ? (float)exp((double)lac) : 0.f;
+                if (o.logkappa) o.logkappa[r] = (float)lk;
+                if (o.logkappa_corr) o.logkappa_corr[r] = (float)lkc;
+                if (o.logkappa_ref) o.logkappa_ref[r] = (float)lkr;
+                if (o.ref_tokens) o.ref_tokens[r] = rec.ref;
+                if (o.row_stats)
+                    reinterpret_cast<float4*>(o.row_stats)[r] =
+                        make_float4(rec.mx, (float)rec.lzx, rec.my, (float)rec.lzy);
+            }
         }
-        if (o.accept_len) o.accept_len[path] = A;
-        if (o.expected_len) o.expected_len[path] = (float)EA;
+        if (lane == 0) {
+            if (o.accept_len) o.accept_len[path] = A;
+            if (o.expected_len) o.expected_len[path] = (float)EA;
+        }
     }
 }
 
@@ -763,9 +818,34 @@ __device__ __forceinline__ void loss_mean(float* loss, int B) {
 
 // --------------------------------------------------------------- gradient
 // grad[r][v] = g q_r(v) - c0 [v = t0] - c1 [v = t1], q_r(v) = 2^{(x_v - m) c} / Z.
+template <typename T, typename G, int PV>
+__device__ __forceinline__ void grad_store(G* g, int64_t v0, const float (&o)[PV], uint64_t pol) {
+    if constexpr (sizeof(G) == 2) {
+        uint32_t w[PV / 2];
+#pragma unroll
+        for (int e = 0; e < PV / 2; ++e) {
+            __nv_bfloat162 h = __floats2bfloat162_rn(o[2 * e], o[2 * e + 1]);
+            w[e] = *reinterpret_cast<uint32_t*>(&h);
+        }
+        if constexpr (PV == 8)
+            st_stream(g + v0, make_uint4(w[0], w[1], w[2], w[3]), pol);
+        else  // f32 logits, bf16 gradient: 8 bytes per vector
+            *reinterpret_cast<uint2*>(g + v0) = make_uint2(w[0], w[1]);
+    } else {
+        st_stream(g + v0, make_uint4(__float_as_uint(o[0]), __float_as_uint(o[1]),
+                                     __float_as_uint(o[2]), __float_as_uint(o[3])),
+                  pol);
+        if constexpr (PV == 8)  // bf16 logits, f32 gradient: a second store
+            st_stream(g + v0 + 4, make_uint4(__float_as_uint(o[4]), __float_as_uint(o[5]),
+                                             __float_as_uint(o[6]), __float_as_uint(o[7])),
+                      pol);
+    }
+}
+
 template <typename T, bool VEC, typename G>
 __device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* grad) {
     constexpr int PV = Traits<T>::kPerVec;
+    constexpr int U = 4;  // vectors in flight per thread
     const int64_t V = P.V;
     const T* x = P.draft + (int64_t)r * V;
     G* g = grad + (int64_t)r * V;
@@ -777,39 +857,29 @@ __device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* g
     const uint64_t pol = policy_evict_first();
     if constexpr (VEC) {
         const int64_t nvec = V / PV;
-        for (int64_t i = threadIdx.x; i < nvec; i += kThreads) {
-            const int64_t v0 = i * PV;
-            const uint4 raw = ld_stream(x + v0, pol);
-            float f[PV], o[PV];
-            unpack<T>(raw, f);
+        for (int64_t i0 = threadIdx.x; i0 < nvec; i0 += (int64_t)kThreads * U) {
+            uint4 raw[U];
 #pragma unroll
-            for (int e = 0; e < PV; ++e) {
-                float val = gq * ex2((f[e] - mx) * c);
-                const int64_t v = v0 + e;
-                if (v == cf.t0) val -= cf.c0;
-                if (v == cf.t1) val -= cf.c1;
-                o[e] = val;
+            for (int u = 0; u < U; ++u) {
+                const int64_t i = i0 + (int64_t)u * kThreads;
+                if (i < nvec) raw[u] = ld_stream(x + i * PV, pol);
             }
-            if constexpr (sizeof(G) == 2) {
-                uint32_t w[PV / 2];
 #pragma unroll
-                for (int e = 0; e < PV / 2; ++e) {
-                    __nv_bfloat162 h = __floats2bfloat162_rn(o[2 * e], o[2 * e + 1]);
-                    w[e] = *reinterpret_cast<uint32_t*>(&h);
+            for (int u = 0; u < U; ++u) {
+                const int64_t i = i0 + (int64_t)u * kThreads;
+                if (i >= nvec) break;
+                const int64_t v0 = i * PV;
+                float f[PV], o[PV];
+                unpack<T>(raw[u], f);
+#pragma unroll
+                for (int e = 0; e < PV; ++e) {
+                    float val = gq * ex2((f[e] - mx) * c);
+                    const int64_t v = v0 + e;
+                    if (v == cf.t0) val -= cf.c0;
+                    if (v == cf.t1) val -= cf.c1;
+                    o[e] = val;
                 }
-                if constexpr (PV == 8)
-                    st_stream(g + v0, make_uint4(w[0], w[1], w[2], w[3]), pol);
-                else  // f32 logits, bf16 gradient: 8 bytes per step
-                    *reinterpret_cast<uint2*>(g + v0) = make_uint2(w[0], w[1]);
-            } else {
-                st_stream(g + v0, make_uint4(__float_as_uint(o[0]), __float_as_uint(o[1]),
-                                             __float_as_uint(o[2]), __float_as_uint(o[3])),
-                          pol);
-                if constexpr (PV == 8)  // bf16 logits, f32 gradient: a second store
-                    st_stream(g + v0 + 4,
-                              make_uint4(__float_as_uint(o[4]), __float_as_uint(o[5]),
-                                         __float_as_uint(o[6]), __float_as_uint(o[7])),
-                              pol);
+                grad_store<T, G, PV>(g, v0, o, pol);
             }
         }
     } else {
@@ -964,23 +1034,6 @@ __device__ void tree_pass(const Problem<T>& P, int b, float4* tab, TreeShared& s
         if (!has_child) bonus = ld_cg(P.rows + n0 + best).ps;  // leaf: p-draw at its row
         o.bonus[b] = bonus;
     }
-}
-
-// --------------------------------------------------------------- fused schedule
-// Ticket order of the fused kernel, in blocks of P = K*D items: the rows of
-// prefixes 0..lag, then alternately the gradient rows of prefix g and the
-// rows of prefix g+lag+1, then the remaining gradients.  A gradient block
-// is never claimed before every row block it depends on has been claimed.
-struct Item { int grad; int prefix; };
-__device__ __forceinline__ Item schedule_block(int j, int B, int lag) {
-    if (lag >= B - 1) {  // all rows, then all gradients
-        return j < B ? Item{0, j} : Item{1, j - B};
-    }
-    if (j <= lag) return Item{0, j};
-    const int k = j - (lag + 1);
-    const int rows_left = B - (lag + 1);
-    if (k < 2 * rows_left) return (k & 1) ? Item{0, lag + 1 + (k >> 1)} : Item{1, k >> 1};
-    return Item{1, rows_left + (k - 2 * rows_left)};
 }
 
 }  // namespace vsd
