@@ -212,13 +212,8 @@ def run_ours(args):
     vsd.load()
     c = inputs.CONFIGS[args.config]
     seed = inputs.BASE_SEED + list(inputs.CONFIGS).index(args.config) + 1000 * rank
-    prob = inputs.config(args.config, device=dev, seed=seed)
-    if args.prefixes and args.prefixes < prob["B"]:
-        P = prob["K"] * prob["D"]
-        n = args.prefixes * P
-        for k in ("draft", "target", "u_draft", "u_accept", "u_correct"):
-            prob[k] = prob[k][:n].contiguous()
-        prob["B"] = args.prefixes
+    prob = inputs.config(args.config, device=dev, seed=seed, B=args.prefixes or None)
+    torch.cuda.empty_cache()
     B, K, D, V = prob["B"], prob["K"], prob["D"], prob["V"]
     R = B * K * D
     temps = c["T"]

@@ -103,9 +103,12 @@ def linear_problem(B, K, D, V, dtype="bf16", kind="gauss", device="cpu", seed=BA
                 u_correct=uniforms(R, device, seed + 5))
 
 
-def config(name, device="cpu", seed=None):
-    """The named workload (see the module docstring)."""
-    c = CONFIGS[name]
+def config(name, device="cpu", seed=None, B=None):
+    """The named workload (see the module docstring); B overrides the number of
+    prefixes (trees) for small profiling runs of the same shapes."""
+    c = dict(CONFIGS[name])
+    if B is not None:
+        c["B"] = int(B)
     idx = list(CONFIGS).index(name)
     seed = BASE_SEED + idx if seed is None else seed
     if name == "tiny":
