@@ -76,8 +76,8 @@ typedef struct {
 
 /* M-step parameters (App. F: w(l) = 1.05^l, tau = 0.2). */
 typedef struct {
-    float w_base;      /* w(l) = w_base^l, l = 1..D                                */
-    float tau_car;     /* CAR temperature tau of Eq. zeta                          */
+    double w_base;     /* w(l) = w_base^l, l = 1..D                                */
+    double tau_car;    /* CAR temperature tau of Eq. zeta                          */
     int32_t zeta_mode; /* 0: softmax of q(z~_{<=l})/tau (as printed); 1: log q      */
     int32_t grad_dtype;/* vsd_dtype of the gradient output                         */
     uint64_t wait_timeout_ns; /* bound of every device wait; 0 = 2 s              */

@@ -102,8 +102,8 @@ vsd_status from_cuda(cudaError_t e) { return e == cudaSuccess ? VSD_OK : VSD_ERR
 
 vsd_params default_params(vsd_dtype dtype) {
     vsd_params p;
-    p.w_base = 1.05f;
-    p.tau_car = 0.2f;
+    p.w_base = 1.05;
+    p.tau_car = 0.2;
     p.zeta_mode = 0;
     p.grad_dtype = dtype;
     p.wait_timeout_ns = kDefaultTimeoutNs;
@@ -112,8 +112,8 @@ vsd_params default_params(vsd_dtype dtype) {
 }
 
 vsd_status check_params(const vsd_params& p) {
-    if (!(p.w_base > 0.f) || !isfinite(p.w_base)) return VSD_ERR_INVALID_ARG;
-    if (!(p.tau_car > 0.f)) return VSD_ERR_INVALID_ARG;  // +inf allowed: zeta = 1/K
+    if (!(p.w_base > 0.0) || !isfinite(p.w_base)) return VSD_ERR_INVALID_ARG;
+    if (!(p.tau_car > 0.0)) return VSD_ERR_INVALID_ARG;  // +inf allowed: zeta = 1/K
     if (p.zeta_mode != 0 && p.zeta_mode != 1) return VSD_ERR_INVALID_ARG;
     if (p.grad_dtype != VSD_F32 && p.grad_dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
     return VSD_OK;
@@ -138,8 +138,8 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.ts.T = T_;
     P.ts.Td = (double)T_;
     P.parent = L.parent;
-    P.w_base = 1.05f;
-    P.tau_car = 0.2f;
+    P.w_base = 1.05;
+    P.tau_car = 0.2;
     P.timeout_ns = kDefaultTimeoutNs;
     const WsLayout w = ws_layout(L);
     P.status = at<int>(ws, w.status);

@@ -79,7 +79,7 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int* status, uint64_t
         if (ld_acquire(flag)) return true;
         if (*(volatile int*)status & VSD_STATUS_TIMEOUT) return false;
         if (global_timer_ns() - t0 > timeout_ns) return false;
-        __nanosleep(256);
+        __nanosleep(1000);
     }
 }
 

@@ -102,7 +102,7 @@ struct Problem {
     const float* ref_logkappa;    // [B][D] or null
     const int32_t* given_tokens;  // [R] or null (draft sampling)
     const int32_t* parent;        // tree [B][N]
-    float w_base, tau_car;
+    double w_base, tau_car;
     int zeta_mode;
     int grad_bf16;
     int inject_wait_fault;
@@ -748,7 +748,7 @@ __device__ void weights_pass(const Problem<T>& P, const EStepView& E, int b, flo
     double Jp = 0.0, Np = 0.0, lqt = 0.0, lqc = 0.0;
     for (int d = 0; d < D; ++d) {
         const int l = d + 1;
-        const double w = pow((double)P.w_base, (double)l);  // w(l), App. F
+        const double w = pow(P.w_base, (double)l);  // w(l), App. F
         double ot = 0.0, op = 0.0;
         if (act) {
             const int r = rbase + d;
@@ -760,7 +760,7 @@ __device__ void weights_pass(const Problem<T>& P, const EStepView& E, int b, flo
             op = ot > 0.0 ? w : ((lkc >= lkr) ? w : 0.0);
             sh.ot[s] = ot;
             sh.op[s] = op;
-            sh.cq[s] = (P.zeta_mode == 0 ? exp(lqt) : lqt) / (double)P.tau_car;
+            sh.cq[s] = (P.zeta_mode == 0 ? exp(lqt) : lqt) / P.tau_car;
         }
         __syncthreads();
         if (act) {
@@ -845,7 +845,7 @@ __device__ __forceinline__ void grad_store(G* g, int64_t v0, const float (&o)[PV
 template <typename T, bool VEC, typename G>
 __device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* grad) {
     constexpr int PV = Traits<T>::kPerVec;
-    constexpr int U = 4;  // vectors in flight per thread
+    constexpr int U = 8;  // vectors in flight per thread
     const int64_t V = P.V;
     const T* x = P.draft + (int64_t)r * V;
     G* g = grad + (int64_t)r * V;

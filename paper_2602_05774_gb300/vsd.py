@@ -38,7 +38,7 @@ class Layout(C.Structure):
 
 
 class Params(C.Structure):
-    _fields_ = [("w_base", C.c_float), ("tau_car", C.c_float), ("zeta_mode", C.c_int32),
+    _fields_ = [("w_base", C.c_double), ("tau_car", C.c_double), ("zeta_mode", C.c_int32),
                 ("grad_dtype", C.c_int32), ("wait_timeout_ns", C.c_uint64),
                 ("test_never_publish", C.c_int32)]
 
