@@ -41,17 +41,19 @@ def up_to_date():
 
 
 def build_library(force=False, verbose=False):
-    """Compile libvsd.so if missing or stale; return its path."""
+    """Compile libvsd.so if missing or stale; return its path.  Extra nvcc
+    flags (tuning experiments) may be given in the VSD_NVCC_FLAGS variable."""
     if not force and up_to_date():
         return LIB
     os.makedirs(OUT_DIR, exist_ok=True)
     cc = nvcc()
+    extra = os.environ.get("VSD_NVCC_FLAGS", "").split()
     procs = []
     objs = []
     for src in SOURCES:
         obj = os.path.join(OUT_DIR, src.replace(".cu", ".o"))
         objs.append(obj)
-        cmd = [cc] + ARCH + FLAGS + ["-c", os.path.join(CSRC, src), "-o", obj]
+        cmd = [cc] + ARCH + FLAGS + extra + ["-c", os.path.join(CSRC, src), "-o", obj]
         if verbose:
             print(" ".join(cmd), file=sys.stderr)
         procs.append((cmd, subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT)))

@@ -6,13 +6,29 @@
 
 namespace vsd {
 
+// Dynamic shared memory: [Ring (vector rows)] [chunk table].
+template <bool VEC>
+__device__ __forceinline__ void smem_views(unsigned char* dsm, Ring*& rg, float4*& tab) {
+    if (VEC) {
+        rg = reinterpret_cast<Ring*>(dsm);
+        tab = reinterpret_cast<float4*>(dsm + sizeof(Ring));
+        ring_init(rg);
+    } else {
+        rg = nullptr;
+        tab = reinterpret_cast<float4*>(dsm);
+    }
+}
+
 // ------------------------------------------------------------ separate kernels
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads) k_sample(Problem<T> P) {
-    extern __shared__ float4 tab[];
+    extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ RowShared sh;
+    Ring* rg;
+    float4* tab;
+    smem_views<VEC>(dsm, rg, tab);
     const int r = blockIdx.x;
-    row_pass<T, VEC, false, kSampleToken, false>(P, r, tab, sh);
+    row_pass<T, VEC, false, kSampleToken, false>(P, r, rg, tab, sh);
     if (threadIdx.x == 0) {
         const RowRec rec = P.rows[r];
         P.out.tokens[r] = rec.tok;
@@ -25,26 +41,35 @@ __global__ void __launch_bounds__(kThreads) k_sample(Problem<T> P) {
 
 template <typename T, bool VEC, bool TREE>
 __global__ void __launch_bounds__(kThreads) k_rows_verify(Problem<T> P) {
-    extern __shared__ float4 tab[];
+    extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ RowShared sh;
+    Ring* rg;
+    float4* tab;
+    smem_views<VEC>(dsm, rg, tab);
     if (TREE)
-        row_pass<T, VEC, true, kNoToken, false>(P, blockIdx.x, tab, sh);
+        row_pass<T, VEC, true, kNoToken, false>(P, blockIdx.x, rg, tab, sh);
     else
-        row_pass<T, VEC, true, kGivenToken, true>(P, blockIdx.x, tab, sh);
+        row_pass<T, VEC, true, kGivenToken, true>(P, blockIdx.x, rg, tab, sh);
 }
 
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads) k_paths(Problem<T> P) {
-    extern __shared__ float4 tab[];
+    extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ PathShared sh;
-    path_pass<T, VEC>(P, blockIdx.x, tab, sh);
+    Ring* rg;
+    float4* tab;
+    smem_views<VEC>(dsm, rg, tab);
+    path_pass<T, VEC>(P, blockIdx.x, rg, tab, sh);
 }
 
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads) k_tree(Problem<T> P) {
-    extern __shared__ float4 tab[];
+    extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ TreeShared sh;
-    tree_pass<T, VEC>(P, blockIdx.x, tab, sh);
+    Ring* rg;
+    float4* tab;
+    smem_views<VEC>(dsm, rg, tab);
+    tree_pass<T, VEC>(P, blockIdx.x, rg, tab, sh);
 }
 
 template <typename T>
@@ -93,14 +118,20 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int* status, uint64_t
 // blocks that never wait, so progress does not depend on residency.  Gradient
 // rows follow their prefix closely, so the draft rows they re-read are still
 // in L2.
+#ifndef VSD_FUSED_MIN_BLOCKS
+#define VSD_FUSED_MIN_BLOCKS 3
+#endif
 template <typename T, bool VEC, typename G>
-__global__ void __launch_bounds__(kThreads, 2) k_fused(Problem<T> P, G* grad) {
-    extern __shared__ float4 tab[];
+__global__ void __launch_bounds__(kThreads, VSD_FUSED_MIN_BLOCKS) k_fused(Problem<T> P, G* grad) {
+    extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ union {
         RowShared row;
         PathShared path;
         WeightsShared w;
     } sh;
+    Ring* rg;
+    float4* tab;
+    smem_views<VEC>(dsm, rg, tab);
     __shared__ int s_kind, s_idx, s_flag;
     const int Pp = P.K * P.D;
     const int B = P.B;
@@ -111,6 +142,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_fused(Problem<T> P, G* grad) {
             int kind = 0, idx = 0;  // 0: finished, 1: logit row, 2: gradient row
             int g = *(volatile int*)P.grad_head;
             for (;;) {
+                if (*(volatile int*)P.status & VSD_STATUS_TIMEOUT) break;  // stop after a failed wait
                 while (g < B && ld_acquire(P.ready + g)) {
                     const int t = atomicAdd(P.grad_cnt + g, 1);
                     if (t < Pp) { kind = 2; idx = g * Pp + t; break; }
@@ -135,7 +167,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_fused(Problem<T> P, G* grad) {
         if (kind == 0) break;
         if (kind == 1) {
             const int prefix = r / Pp;
-            row_pass<T, VEC, true, kSampleToken, true>(P, r, tab, sh.row);
+            row_pass<T, VEC, true, kSampleToken, true>(P, r, rg, tab, sh.row);
             const int path = r / P.D;
             if (threadIdx.x == 0) {
                 __threadfence();
@@ -144,7 +176,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_fused(Problem<T> P, G* grad) {
             }
             __syncthreads();
             if (s_flag) {
-                path_pass<T, VEC>(P, path, tab, sh.path);
+                path_pass<T, VEC>(P, path, rg, tab, sh.path);
                 __syncthreads();
                 if (threadIdx.x == 0) {
                     __threadfence();
@@ -183,7 +215,7 @@ static cudaError_t prep(K kernel, size_t smem) {
 
 template <>
 cudaError_t Launch<VSD_T>::sample(const Problem<VSD_T>& P, bool vec, cudaStream_t s) {
-    const size_t smem = table_smem_bytes(P.nch);
+    const size_t smem = stream_smem_bytes(P.nch, vec);
     if (vec) {
         cudaError_t e = prep(k_sample<VSD_T, true>, smem);
         if (e) return e;
@@ -199,7 +231,7 @@ cudaError_t Launch<VSD_T>::sample(const Problem<VSD_T>& P, bool vec, cudaStream_
 template <>
 cudaError_t Launch<VSD_T>::rows_verify(const Problem<VSD_T>& P, bool vec, bool tree,
                                        cudaStream_t s) {
-    const size_t smem = table_smem_bytes(P.nch);
+    const size_t smem = stream_smem_bytes(P.nch, vec);
 #define VSD_ROWS(V_, T_)                                              \
     do {                                                              \
         cudaError_t e = prep(k_rows_verify<VSD_T, V_, T_>, smem);     \
@@ -216,7 +248,7 @@ cudaError_t Launch<VSD_T>::rows_verify(const Problem<VSD_T>& P, bool vec, bool t
 
 template <>
 cudaError_t Launch<VSD_T>::paths(const Problem<VSD_T>& P, bool vec, cudaStream_t s) {
-    const size_t smem = table_smem_bytes(P.nch);
+    const size_t smem = stream_smem_bytes(P.nch, vec);
     const int npaths = P.B * P.K;
     if (vec) {
         cudaError_t e = prep(k_paths<VSD_T, true>, smem);
@@ -232,7 +264,7 @@ cudaError_t Launch<VSD_T>::paths(const Problem<VSD_T>& P, bool vec, cudaStream_t
 
 template <>
 cudaError_t Launch<VSD_T>::tree(const Problem<VSD_T>& P, bool vec, cudaStream_t s) {
-    const size_t smem = table_smem_bytes(P.nch);
+    const size_t smem = stream_smem_bytes(P.nch, vec);
     if (vec) {
         cudaError_t e = prep(k_tree<VSD_T, true>, smem);
         if (e) return e;
@@ -268,7 +300,7 @@ cudaError_t Launch<VSD_T>::grad(const Problem<VSD_T>& P, bool vec, const float4*
 template <>
 cudaError_t Launch<VSD_T>::fused(const Problem<VSD_T>& P, bool vec, void* grad, bool grad_bf16,
                                  int ctas, cudaStream_t s) {
-    const size_t smem = table_smem_bytes(P.nch);
+    const size_t smem = stream_smem_bytes(P.nch, vec);
 #define VSD_FUSED(V_, G_)                                                              \
     do {                                                                               \
         cudaError_t e = prep(k_fused<VSD_T, V_, G_>, smem);                            \
@@ -285,7 +317,12 @@ cudaError_t Launch<VSD_T>::fused(const Problem<VSD_T>& P, bool vec, void* grad, 
 
 template <>
 int Launch<VSD_T>::fused_blocks_per_sm(const Problem<VSD_T>& P, bool vec, bool grad_bf16) {
-    const size_t smem = table_smem_bytes(P.nch);
+    const size_t smem = stream_smem_bytes(P.nch, vec);
+    // the attribute must allow this much before the occupancy query counts it
+    if (vec && grad_bf16) prep(k_fused<VSD_T, true, __nv_bfloat16>, smem);
+    else if (vec) prep(k_fused<VSD_T, true, float>, smem);
+    else if (grad_bf16) prep(k_fused<VSD_T, false, __nv_bfloat16>, smem);
+    else prep(k_fused<VSD_T, false, float>, smem);
     int n = 0;
     cudaError_t e;
     if (vec && grad_bf16)

@@ -31,5 +31,10 @@ template <typename T> struct Launch {
 };
 
 inline size_t table_smem_bytes(int nch) { return (size_t)nch * sizeof(float4); }
+// Dynamic shared memory of a streaming kernel: the TMA ring (vector rows
+// only) followed by the chunk table.
+inline size_t stream_smem_bytes(int nch, bool vec) {
+    return (vec ? sizeof(Ring) : 0) + table_smem_bytes(nch);
+}
 
 }  // namespace vsd

@@ -139,7 +139,9 @@ __device__ __forceinline__ float2 chunk_stats(const uint4 (&buf)[kLoads], float 
     float mk[kLoads];
 #pragma unroll
     for (int k = 0; k < kLoads; ++k) mk[k] = vec_max<T>(buf[k]);
-    float m = fmaxf(fmaxf(mk[0], mk[1]), fmaxf(mk[2], mk[3]));
+    float m = mk[0];
+#pragma unroll
+    for (int k = 1; k < kLoads; ++k) m = fmaxf(m, mk[k]);
     m = warp_max(m);
     const float mm = frame_of(m);
     float s[kLoads];
@@ -152,19 +154,126 @@ __device__ __forceinline__ float2 chunk_stats(const uint4 (&buf)[kLoads], float 
         for (int e = 0; e < PV; ++e) a += mass_rel(f[e], mm, c);
         s[k] = a;
     }
-    float t = (s[0] + s[1]) + (s[2] + s[3]);
+    float t = s[0];
+#pragma unroll
+    for (int k = 1; k < kLoads; ++k) t += s[k];
     t = warp_sum(t);
     return make_float2(m, t);
+}
+
+// --------------------------------------------------------------- TMA ring
+// Every warp owns kStages slots, each holding one chunk of the draft row and
+// one of the target row.  The warp's lane 0 issues 1-D bulk copies (TMA) up
+// to kStages chunks ahead; all lanes wait on the slot's mbarrier, read their
+// own vectors, and the slot is refilled once the warp has read it.  Each warp
+// produces and consumes its own slots, so no block-wide synchronisation is
+// involved.  pos[w] counts the chunks warp w has consumed (slot = pos %
+// kStages, barrier phase = (pos / kStages) & 1) and persists across rows.
+struct Ring {
+    uint4 data[kWarps][kStages][2][kLoads * 32];
+    uint64_t bar[kWarps][kStages];
+    int pos[kWarps];
+    int broken[kWarps];  // a wait ran out: no further waits or copies in this block
+};
+
+__device__ __forceinline__ void ring_init(Ring* rg) {
+    if ((threadIdx.x & 31) == 0) {
+        const int w = threadIdx.x >> 5;
+        for (int st = 0; st < kStages; ++st) mbar_init(&rg->bar[w][st], 1);
+        rg->pos[w] = 0;
+        rg->broken[w] = 0;
+        mbar_init_fence();
+    }
+    __syncthreads();
+}
+
+// Bounded wait on a slot; false (and the timeout status bit) if it ran out.
+__device__ __forceinline__ bool ring_wait(uint64_t* bar, uint32_t parity, int* status) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (global_timer_ns() - t0 > 2000000000ull) {
+            atomicOr(status, VSD_STATUS_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+// Warp-level stream of this warp's chunks (warp, warp + kWarps, ...) of row x
+// (and y) through the ring; consume(ch, bx, by) gets each chunk in registers
+// (positions at or beyond V read as -inf).  Rows must be 16-byte aligned with
+// V * sizeof(T) a multiple of 16.
+template <typename T, bool HAS_Y, class Consume>
+__device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, int64_t V, int nch,
+                                            uint64_t polx, uint64_t poly, int* status,
+                                            Consume&& consume) {
+    constexpr int PV = Traits<T>::kPerVec;
+    constexpr int CE = chunk_elems<T>();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nj = nch > warp ? (nch - warp + kWarps - 1) / kWarps : 0;
+    const int pos = rg->pos[warp];
+    bool broken = rg->broken[warp] != 0;
+    auto issue = [&](int j) {
+        const int ch = warp + j * kWarps;
+        const int slot = (pos + j) % kStages;
+        const int64_t e0 = (int64_t)ch * CE;
+        const int64_t ne = V - e0 < CE ? V - e0 : CE;
+        const uint32_t bytes = (uint32_t)(ne * (int64_t)sizeof(T));
+        uint64_t* bar = &rg->bar[warp][slot];
+        fence_proxy_async();
+        mbar_expect_tx(bar, HAS_Y ? 2 * bytes : bytes);
+        bulk_g2s(rg->data[warp][slot][0], x + e0, bytes, bar, polx);
+        if (HAS_Y) bulk_g2s(rg->data[warp][slot][1], y + e0, bytes, bar, poly);
+    };
+    if (lane == 0)
+        for (int j = 0; j < nj && j < kStages; ++j) issue(j);
+    for (int j = 0; j < nj; ++j) {
+        const int slot = (pos + j) % kStages;
+        const uint32_t parity = (uint32_t)((pos + j) / kStages) & 1u;
+        bool ok = broken ? false : ring_wait(&rg->bar[warp][slot], parity, status);
+        broken = __any_sync(0xffffffffu, !ok);
+        const int ch = warp + j * kWarps;
+        const int64_t e0 = (int64_t)ch * CE;
+        uint4 bx[kLoads], by[kLoads];
+#pragma unroll
+        for (int k = 0; k < kLoads; ++k) {
+            const bool in = e0 + (int64_t)k * 32 * PV + lane * PV < V;
+            const uint4 ninf = make_uint4(Traits<T>::kNegInf, Traits<T>::kNegInf,
+                                          Traits<T>::kNegInf, Traits<T>::kNegInf);
+            bx[k] = in ? rg->data[warp][slot][0][k * 32 + lane] : ninf;
+            if (HAS_Y) by[k] = in ? rg->data[warp][slot][1][k * 32 + lane] : ninf;
+        }
+        __syncwarp();
+        if (lane == 0 && !broken && j + kStages < nj) issue(j + kStages);
+        consume(ch, bx, by);
+    }
+    __syncwarp();
+    if (lane == 0) {
+        rg->pos[warp] = pos + nj;
+        rg->broken[warp] = broken ? 1 : 0;
+    }
+    __syncwarp();
 }
 
 // Stream a row (and optionally its target row) once, filling tab[c] =
 // (max_x, sum_x, max_y, sum_y) for every chunk c.  Warps take chunks
 // round-robin and keep the next chunk's loads in flight.
 template <typename T, bool VEC, bool HAS_Y>
-__device__ __forceinline__ void stream_tables(const T* x, const T* y, int64_t V, int nch,
+__device__ __forceinline__ void stream_tables(Ring* rg, const T* x, const T* y, int64_t V, int nch,
                                               float4* tab, float c, uint64_t polx,
-                                              uint64_t poly) {
+                                              uint64_t poly, int* status) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if constexpr (VEC) {
+        ring_stream<T, HAS_Y>(rg, x, y, V, nch, polx, poly, status,
+                              [&](int ch, const uint4 (&bx)[kLoads], const uint4 (&by)[kLoads]) {
+                                  const float2 sx = chunk_stats<T>(bx, c);
+                                  float2 sy = make_float2(0.f, 0.f);
+                                  if (HAS_Y) sy = chunk_stats<T>(by, c);
+                                  if (lane == 0) tab[ch] = make_float4(sx.x, sx.y, sy.x, sy.y);
+                              });
+        return;
+    }
     int ch = warp;
     uint4 bx[kLoads], by[kLoads];
     if (ch < nch) {
@@ -406,15 +515,15 @@ enum XMode { kNoToken = 0, kSampleToken = 1, kGivenToken = 2 };
 // u_draft, read from given_tokens, or absent (trees).  ARGMAX: locate the
 // greedy reference token.
 template <typename T, bool VEC, bool HAS_Y, int XMODE, bool ARGMAX>
-__device__ void row_pass(const Problem<T>& P, int r, float4* tab, RowShared& sh) {
+__device__ void row_pass(const Problem<T>& P, int r, Ring* rg, float4* tab, RowShared& sh) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t V = P.V;
     const T* x = P.draft + (int64_t)r * V;
     const T* y = HAS_Y ? P.target + (int64_t)r * V : nullptr;
     const float c = P.ts.c;
     // The draft row is read again by the gradient pass: ask L2 to keep it.
-    stream_tables<T, VEC, HAS_Y>(x, y, V, P.nch, tab, c, policy_evict_last(),
-                                 policy_evict_first());
+    stream_tables<T, VEC, HAS_Y>(rg, x, y, V, P.nch, tab, c, policy_evict_last(),
+                                 policy_evict_first(), P.status);
     __syncthreads();
     const uint64_t pol = policy_evict_normal();
     if (warp == 0) {
@@ -503,12 +612,40 @@ __device__ void row_pass(const Problem<T>& P, int r, float4* tab, RowShared& sh)
 // --------------------------------------------------------------- residual
 // Stream rows x, y once more and fill tab[c].y with the chunk sums of the
 // residual mass max(0, p - q).
-template <typename T, bool VEC>
-__device__ void stream_residual(const T* x, const T* y, int64_t V, int nch, float4* tab,
-                                const MassRes& mr) {
+template <typename T>
+__device__ __forceinline__ float residual_chunk(const uint4 (&bx)[kLoads], const uint4 (&by)[kLoads],
+                                               const MassRes& mr) {
     constexpr int PV = Traits<T>::kPerVec;
+    float s4[kLoads];
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k) {
+        float fx[PV], fy[PV];
+        unpack<T>(bx[k], fx);
+        unpack<T>(by[k], fy);
+        float a = 0.f;
+#pragma unroll
+        for (int e = 0; e < PV; ++e) a += mr(fx[e], fy[e]);
+        s4[k] = a;
+    }
+    float t = s4[0];
+#pragma unroll
+    for (int k = 1; k < kLoads; ++k) t += s4[k];
+    return warp_sum(t);
+}
+
+template <typename T, bool VEC>
+__device__ void stream_residual(Ring* rg, const T* x, const T* y, int64_t V, int nch, float4* tab,
+                                const MassRes& mr, int* status) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint64_t pol = policy_evict_normal();
+    if constexpr (VEC) {
+        ring_stream<T, true>(rg, x, y, V, nch, pol, pol, status,
+                             [&](int ch, const uint4 (&bx)[kLoads], const uint4 (&by)[kLoads]) {
+                                 const float t = residual_chunk<T>(bx, by, mr);
+                                 if (lane == 0) tab[ch] = make_float4(0.f, t, 0.f, 0.f);
+                             });
+        return;
+    }
     int ch = warp;
     uint4 bx[kLoads], by[kLoads];
     if (ch < nch) {
@@ -522,18 +659,7 @@ __device__ void stream_residual(const T* x, const T* y, int64_t V, int nch, floa
             load_chunk<T, VEC>(x, V, cn, lane, pol, nx);
             load_chunk<T, VEC>(y, V, cn, lane, pol, ny);
         }
-        float s4[kLoads];
-#pragma unroll
-        for (int k = 0; k < kLoads; ++k) {
-            float fx[PV], fy[PV];
-            unpack<T>(bx[k], fx);
-            unpack<T>(by[k], fy);
-            float a = 0.f;
-#pragma unroll
-            for (int e = 0; e < PV; ++e) a += mr(fx[e], fy[e]);
-            s4[k] = a;
-        }
-        const float t = warp_sum((s4[0] + s4[1]) + (s4[2] + s4[3]));
+        const float t = residual_chunk<T>(bx, by, mr);
         if (lane == 0) tab[ch] = make_float4(0.f, t, 0.f, 0.f);
 #pragma unroll
         for (int k = 0; k < kLoads; ++k) {
@@ -547,15 +673,15 @@ __device__ void stream_residual(const T* x, const T* y, int64_t V, int nch, floa
 // Residual draw norm(max(0, p - q)) at row r with uniform u (block).  Returns
 // -1 when the residual has no mass.
 template <typename T, bool VEC>
-__device__ int residual_draw(const Problem<T>& P, int r, const RowRec& rec, float u, float4* tab,
-                             int* out) {
+__device__ int residual_draw(const Problem<T>& P, int r, const RowRec& rec, float u, Ring* rg,
+                             float4* tab, int* out) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t V = P.V;
     const T* x = P.draft + (int64_t)r * V;
     const T* y = P.target + (int64_t)r * V;
     const float c = P.ts.c;
     const MassRes mr{rec.mx, rec.my, (float)exp(-rec.lzx), (float)exp(-rec.lzy), c};
-    stream_residual<T, VEC>(x, y, V, P.nch, tab, mr);
+    stream_residual<T, VEC>(rg, x, y, V, P.nch, tab, mr, P.status);
     __syncthreads();
     if (warp == 0) {
         const double Rt = table_total(tab, P.nch, 0, 0.f, c, lane);
@@ -577,13 +703,13 @@ __device__ int residual_draw(const Problem<T>& P, int r, const RowRec& rec, floa
 
 // Inverse-CDF draw from p at row r with uniform u (block; streams the target row).
 template <typename T, bool VEC>
-__device__ int p_draw(const Problem<T>& P, int r, float u, float4* tab, int* out) {
+__device__ int p_draw(const Problem<T>& P, int r, float u, Ring* rg, float4* tab, int* out) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t V = P.V;
     const T* y = P.target + (int64_t)r * V;
     const float c = P.ts.c;
     const uint64_t pol = policy_evict_normal();
-    stream_tables<T, VEC, false>(y, nullptr, V, P.nch, tab, c, pol, pol);
+    stream_tables<T, VEC, false>(rg, y, nullptr, V, P.nch, tab, c, pol, pol, P.status);
     __syncthreads();
     if (warp == 0) {
         const float M = table_max(tab, P.nch, 0, lane);
@@ -610,7 +736,7 @@ struct PathShared {
 // handles the rows lane-parallel (two rounds when D > 32) with warp scans for
 // the prefix sums over l; the whole block streams the residual row.
 template <typename T, bool VEC>
-__device__ void path_pass(const Problem<T>& P, int path, float4* tab, PathShared& sh) {
+__device__ void path_pass(const Problem<T>& P, int path, Ring* rg, float4* tab, PathShared& sh) {
     const int D = P.D;
     const int r0 = path * D;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -636,7 +762,7 @@ __device__ void path_pass(const Problem<T>& P, int path, float4* tab, PathShared
     const int A = sh.A;
     int resid = -1;
     if (A < D && !sh.rec.flags)
-        resid = residual_draw<T, VEC>(P, r0 + A, sh.rec, __ldg(P.u_correct + r0 + A), tab,
+        resid = residual_draw<T, VEC>(P, r0 + A, sh.rec, __ldg(P.u_correct + r0 + A), rg, tab,
                                       &sh.resid);
     if (warp == 0) {
         const int b = path / P.K;
@@ -718,7 +844,7 @@ __device__ void path_pass(const Problem<T>& P, int path, float4* tab, PathShared
 
 // --------------------------------------------------------------- weights
 struct WeightsShared {
-    double ot[256], op[256], cq[256];
+    double ot[256], op[256], cq[256], lqt[256], lqc[256];
     double red[kThreads];
 };
 
@@ -734,36 +860,31 @@ __device__ __forceinline__ double block_sum(double v, double* red) {
     return r;
 }
 
-// M-step of prefix b (block; thread s owns proposal s, K <= kThreads).
+// M-step of prefix b (block; proposals s strided over the threads, K <= 256).
 // Writes coef[] for the prefix's rows, the optional weights table and
 // loss_out[b].  Arithmetic in double.
 template <typename T>
 __device__ void weights_pass(const Problem<T>& P, const EStepView& E, int b, float* weights_out,
                              float* loss_out, WeightsShared& sh) {
     const int K = P.K, D = P.D;
-    const int s = threadIdx.x;
-    const bool act = s < K;
-    const int rbase = (b * K + s) * D;  // rows of proposal s
-    // per-l terms o'(o~ - beta zeta) and o'(1 - o~) of row (s, l-1): P.wscr
-    double Jp = 0.0, Np = 0.0, lqt = 0.0, lqc = 0.0;
+    double Jp = 0.0, Np = 0.0;
+    for (int s = threadIdx.x; s < K; s += kThreads) sh.lqt[s] = sh.lqc[s] = 0.0;
     for (int d = 0; d < D; ++d) {
         const int l = d + 1;
         const double w = pow(P.w_base, (double)l);  // w(l), App. F
-        double ot = 0.0, op = 0.0;
-        if (act) {
-            const int r = rbase + d;
+        for (int s = threadIdx.x; s < K; s += kThreads) {
+            const int r = (b * K + s) * D + d;
             const double lk = ld_cg(E.lk + r), lkc = ld_cg(E.lkc + r), lkr = ld_cg(E.lkr + r);
-            lqt += (double)ld_cg(E.lq_tok + r);
-            lqc += (double)ld_cg(E.lq_corr + r);
+            sh.lqt[s] += (double)ld_cg(E.lq_tok + r);
+            sh.lqc[s] += (double)ld_cg(E.lq_corr + r);
             // Algorithm 2 scores z~; Algorithm 1 keeps z~ if it passes, else z'.
-            ot = (lk >= lkr) ? 1.0 : 0.0;
-            op = ot > 0.0 ? w : ((lkc >= lkr) ? w : 0.0);
+            const double ot = (lk >= lkr) ? 1.0 : 0.0;
             sh.ot[s] = ot;
-            sh.op[s] = op;
-            sh.cq[s] = (P.zeta_mode == 0 ? exp(lqt) : lqt) / P.tau_car;
+            sh.op[s] = ot > 0.0 ? w : ((lkc >= lkr) ? w : 0.0);
+            sh.cq[s] = (P.zeta_mode == 0 ? exp(sh.lqt[s]) : sh.lqt[s]) / P.tau_car;
         }
         __syncthreads();
-        if (act) {
+        for (int s = threadIdx.x; s < K; s += kThreads) {
             double num = 0.0, den = 0.0, M = -INFINITY;
             for (int j = 0; j < K; ++j) {
                 if (j != s) { num += sh.op[j] * sh.ot[j]; den += sh.op[j]; }
@@ -773,10 +894,12 @@ __device__ void weights_pass(const Problem<T>& P, const EStepView& E, int b, flo
             double Zs = 0.0;
             for (int j = 0; j < K; ++j) Zs += exp(sh.cq[j] - M);
             const double zeta = exp(sh.cq[s] - M) / Zs;        // Eq. zeta
-            const double lqz = ot > 0.0 ? lqt : lqc;
-            if (op != 0.0) Jp += op * (lqz - beta * zeta * lqt);  // Eq. advance
+            const double ot = sh.ot[s], op = sh.op[s];
+            const double lqz = ot > 0.0 ? sh.lqt[s] : sh.lqc[s];
+            if (op != 0.0) Jp += op * (lqz - beta * zeta * sh.lqt[s]);  // Eq. advance
             Np += op;
-            P.wscr[rbase + d] = make_double2(op * (ot - beta * zeta), op * (1.0 - ot));
+            // per-l terms o'(o~ - beta zeta) and o'(1 - o~) of row (s, l-1)
+            P.wscr[(b * K + s) * D + d] = make_double2(op * (ot - beta * zeta), op * (1.0 - ot));
             if (weights_out) {
                 float4* wo = reinterpret_cast<float4*>(weights_out) + ((int64_t)b * D + d) * K + s;
                 *wo = make_float4((float)ot, (float)op, (float)beta, (float)zeta);
@@ -786,8 +909,9 @@ __device__ void weights_pass(const Problem<T>& P, const EStepView& E, int b, flo
     }
     const double N = block_sum(Np, sh.red);
     const double J = block_sum(Jp, sh.red);
-    if (act) {
-        const double scale = N > 0.0 ? 1.0 / ((double)P.B * N * P.ts.Td) : 0.0;
+    const double scale = N > 0.0 ? 1.0 / ((double)P.B * N * P.ts.Td) : 0.0;
+    for (int s = threadIdx.x; s < K; s += kThreads) {
+        const int rbase = (b * K + s) * D;
         double c0 = 0.0, c1 = 0.0;
         for (int d = D - 1; d >= 0; --d) {
             const int r = rbase + d;
@@ -908,7 +1032,7 @@ struct TreeShared {
 // One draft tree per block; rows of tree b are b*N .. b*N + N - 1, row n is
 // the distribution node n's children were drafted from (App. E tree).
 template <typename T, bool VEC>
-__device__ void tree_pass(const Problem<T>& P, int b, float4* tab, TreeShared& sh) {
+__device__ void tree_pass(const Problem<T>& P, int b, Ring* rg, float4* tab, TreeShared& sh) {
     const int N = P.N;
     const int64_t V = P.V;
     const int n0 = b * N;
@@ -993,7 +1117,7 @@ __device__ void tree_pass(const Problem<T>& P, int b, float4* tab, TreeShared& s
         const float c = P.ts.c;
         const MassRes mr{sh.rec.mx, sh.rec.my, (float)exp(-sh.rec.lzx), (float)exp(-sh.rec.lzy),
                          c};
-        stream_residual<T, VEC>(x, y, V, P.nch, tab, mr);
+        stream_residual<T, VEC>(rg, x, y, V, P.nch, tab, mr, P.status);
         __syncthreads();
         if (warp == 0) {
             const double Rt = table_total(tab, P.nch, 0, 0.f, c, lane);
@@ -1017,7 +1141,7 @@ __device__ void tree_pass(const Problem<T>& P, int b, float4* tab, TreeShared& s
             // no residual mass: each rejected child draws from p (reading R10)
             for (int n = first; n < N; ++n) {
                 if (__ldg(par + n) != u || sh.pacc[n]) continue;
-                const int tok = p_draw<T, VEC>(P, r, __ldg(P.u_correct + n0 + n), tab, &sh.resid);
+                const int tok = p_draw<T, VEC>(P, r, __ldg(P.u_correct + n0 + n), rg, tab, &sh.resid);
                 if (threadIdx.x == 0) o.corr_tokens[n0 + n] = tok;
             }
         }
