@@ -15,7 +15,7 @@ constexpr int kThreads = 128;            // threads of every block-level pass
 constexpr int kWarps = kThreads / 32;
 constexpr int kLoads = 4;                // 16-byte vectors per lane per chunk per tensor
 #ifndef VSD_STAGES
-#define VSD_STAGES 4
+#define VSD_STAGES 2
 #endif
 constexpr int kStages = VSD_STAGES;      // TMA ring depth per warp (chunks in flight)
 constexpr double kLog2e = 1.4426950408889634073599246810019;

@@ -119,7 +119,7 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int* status, uint64_t
 // rows follow their prefix closely, so the draft rows they re-read are still
 // in L2.
 #ifndef VSD_FUSED_MIN_BLOCKS
-#define VSD_FUSED_MIN_BLOCKS 3
+#define VSD_FUSED_MIN_BLOCKS 4
 #endif
 template <typename T, bool VEC, typename G>
 __global__ void __launch_bounds__(kThreads, VSD_FUSED_MIN_BLOCKS) k_fused(Problem<T> P, G* grad) {
