@@ -55,7 +55,9 @@ typedef enum {
     VSD_ERR_CUDA = 3,        /* a CUDA runtime call failed                        */
     VSD_ERR_TIMEOUT = 4,     /* a device-side wait gave up (vsd_device_status)    */
     VSD_ERR_WORKSPACE = 5,   /* workspace missing or smaller than required        */
-    VSD_ERR_DEVICE_DATA = 6  /* a device-side data check failed (status bits)     */
+    VSD_ERR_DEVICE_DATA = 6, /* a device-side data check failed (status bits)     */
+    VSD_ERR_TOO_LARGE = 7    /* the problem needs more scratch than the library's
+                                built-in array (vsd_estep_mstep_noalloc)           */
 } vsd_status;
 
 typedef enum { VSD_F32 = 0, VSD_BF16 = 1 } vsd_dtype;
@@ -176,6 +178,34 @@ vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtyp
                            const float* u_accept, const float* u_correct,
                            const float* ref_logkappa, const vsd_params* params,
                            vsd_linear_outputs* out, void* ws, size_t ws_bytes, void* stream);
+
+/* Allocation-free variant of vsd_estep_mstep; the paper has no counterpart.
+ * For callers that cannot allocate device memory where they call the library
+ * (a plugin given only its input and output pointers, a process whose device
+ * memory belongs entirely to another allocator, a latency-critical loop where
+ * cudaMalloc/cudaFree would synchronise the device).  Instead of a caller
+ * workspace it uses a fixed array of VSD_NOALLOC_SCRATCH_BYTES in device memory
+ * that the library owns; every GPU that loads the library holds that array until
+ * the process exits.  Arguments, required outputs and results are those of
+ * vsd_estep_mstep.
+ *   - Limit: the layout's vsd_workspace_bytes() must not exceed
+ *     VSD_NOALLOC_SCRATCH_BYTES (1 MiB: every linear layout of up to 4096 rows);
+ *     larger problems return VSD_ERR_TOO_LARGE before anything is enqueued.
+ *   - The first call on a device looks up the array's device address with that
+ *     device current (cudaGetSymbolAddress); make that first call before any
+ *     stream capture.  The call allocates nothing.
+ *   - All calls on a device share the one array, which keeps the last call's
+ *     contents (each call clears the part that must start at zero).  Calls that
+ *     overlap on the GPU -- on different streams, or from different host
+ *     threads -- race on it; order them on one stream.
+ *   - The device status word of these calls lives in that array and is not
+ *     exposed; argument and launch errors are returned as usual. */
+#define VSD_NOALLOC_SCRATCH_BYTES (1u << 20)
+vsd_status vsd_estep_mstep_noalloc(const void* draft, const void* target, vsd_dtype dtype,
+                                   vsd_layout layout, float T, const float* u_draft,
+                                   const float* u_accept, const float* u_correct,
+                                   const float* ref_logkappa, const vsd_params* params,
+                                   vsd_linear_outputs* out, void* stream);
 
 /* Waits for `stream`, then reads and clears the device status word of `ws`
  * into *status_bits (host).  Returns VSD_ERR_TIMEOUT if the timeout bit is set,

@@ -395,6 +395,8 @@ const char* vsd_status_string(vsd_status status) {
         case VSD_ERR_TIMEOUT: return "a device-side wait timed out";
         case VSD_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
         case VSD_ERR_DEVICE_DATA: return "device-side data check failed";
+        case VSD_ERR_TOO_LARGE:
+            return "problem needs more scratch than the built-in array of vsd_estep_mstep_noalloc";
     }
     return "unknown status";
 }

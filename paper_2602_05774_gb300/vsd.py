@@ -18,11 +18,12 @@ VSD_F32, VSD_BF16 = 0, 1
 STATUS_BAD_ROW, STATUS_TIMEOUT, STATUS_BAD_TREE, STATUS_BAD_TOKEN = 1, 2, 4, 8
 _STATUS_NAMES = {0: "VSD_OK", 1: "VSD_ERR_INVALID_ARG", 2: "VSD_ERR_UNSUPPORTED",
                  3: "VSD_ERR_CUDA", 4: "VSD_ERR_TIMEOUT", 5: "VSD_ERR_WORKSPACE",
-                 6: "VSD_ERR_DEVICE_DATA"}
+                 6: "VSD_ERR_DEVICE_DATA", 7: "VSD_ERR_TOO_LARGE"}
 
 SYMBOLS = ("vsd_workspace_bytes", "vsd_sample_paths", "vsd_verify_paths",
            "vsd_weighted_loss_fwd_bwd", "vsd_estep_mstep", "vsd_device_status",
-           "vsd_status_string", "vsd_version")
+           "vsd_status_string", "vsd_version", "vsd_estep_mstep_noalloc")
+NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
 class VsdError(RuntimeError):
@@ -86,12 +87,15 @@ def _lib():
         lib.vsd_estep_mstep.argtypes = [vp, vp, C.c_int, Layout, C.c_float, vp, vp, vp, vp,
                                         C.POINTER(Params), C.POINTER(LinearOutputs), vp,
                                         C.c_size_t, vp]
+        lib.vsd_estep_mstep_noalloc.argtypes = [vp, vp, C.c_int, Layout, C.c_float, vp, vp, vp,
+                                                vp, C.POINTER(Params), C.POINTER(LinearOutputs),
+                                                vp]
         lib.vsd_device_status.argtypes = [vp, vp, C.POINTER(C.c_int32)]
         lib.vsd_status_string.argtypes = [C.c_int]
         lib.vsd_status_string.restype = C.c_char_p
         lib.vsd_version.restype = C.c_char_p
         for name in ("vsd_sample_paths", "vsd_verify_paths", "vsd_weighted_loss_fwd_bwd",
-                     "vsd_estep_mstep", "vsd_device_status"):
+                     "vsd_estep_mstep", "vsd_device_status", "vsd_estep_mstep_noalloc"):
             getattr(lib, name).restype = C.c_int
         _LIB = lib
     return _LIB
@@ -312,6 +316,31 @@ def estep_mstep(draft, target, u_draft, u_accept, u_correct, K, D, T, ref_logkap
                                   _ptr(u_draft), _ptr(u_accept), _ptr(u_correct),
                                   _ptr(ref_logkappa), C.byref(prm), C.byref(st), _ptr(ws),
                                   ws.numel(), _stream(dev)), "vsd_estep_mstep")
+    return out
+
+
+def estep_mstep_noalloc(draft, target, u_draft, u_accept, u_correct, K, D, T,
+                        ref_logkappa=None, prm=None, out=None, full=True):
+    """The fused E-step + M-step without a workspace argument, for callers that
+    cannot allocate device scratch: the library uses its own fixed array in
+    device memory (limit: layouts whose workspace fits NOALLOC_SCRATCH_BYTES).
+    Calls on one device share that array, so they must not overlap on the GPU.
+    Outputs are allocated here when `out` is None, as in estep_mstep()."""
+    _need_cuda(draft, target, u_draft, u_accept, u_correct, ref_logkappa)
+    V = draft.shape[-1]
+    R = _rows(draft, V)
+    B = R // (K * D)
+    lay = layout(B, K, D, V)
+    dev = draft.device
+    prm = prm or params(like=draft)
+    if out is None:
+        gdt = torch.bfloat16 if prm.grad_dtype == VSD_BF16 else torch.float32
+        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full)
+    st = _linear_struct(out)
+    _check(_lib().vsd_estep_mstep_noalloc(_ptr(draft), _ptr(target), _dtype_code(draft), lay,
+                                          float(T), _ptr(u_draft), _ptr(u_accept),
+                                          _ptr(u_correct), _ptr(ref_logkappa), C.byref(prm),
+                                          C.byref(st), _stream(dev)), "vsd_estep_mstep_noalloc")
     return out
 
 
