@@ -189,7 +189,8 @@ vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtyp
  * the process exits.  Arguments, required outputs and results are those of
  * vsd_estep_mstep.
  *   - Limit: the layout's vsd_workspace_bytes() must not exceed
- *     VSD_NOALLOC_SCRATCH_BYTES (1 MiB: every linear layout of up to 4096 rows);
+ *     VSD_NOALLOC_SCRATCH_BYTES (32 MiB: every linear layout of up to 4096 rows
+ *     with V <= 200000; the B=32, K=16, D=8, V=128256 workload needs 17 MB);
  *     larger problems return VSD_ERR_TOO_LARGE before anything is enqueued.
  *   - The first call on a device looks up the array's device address with that
  *     device current (cudaGetSymbolAddress); make that first call before any
@@ -200,7 +201,7 @@ vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtyp
  *     threads -- race on it; order them on one stream.
  *   - The device status word of these calls lives in that array and is not
  *     exposed; argument and launch errors are returned as usual. */
-#define VSD_NOALLOC_SCRATCH_BYTES (1u << 20)
+#define VSD_NOALLOC_SCRATCH_BYTES (32u << 20)
 vsd_status vsd_estep_mstep_noalloc(const void* draft, const void* target, vsd_dtype dtype,
                                    vsd_layout layout, float T, const float* u_draft,
                                    const float* u_accept, const float* u_correct,

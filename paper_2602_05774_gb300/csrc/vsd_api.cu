@@ -23,10 +23,22 @@ constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct WsLayout {
-    size_t status, ticket, prefix_done, grad_head, path_cnt, prefix_cnt, ready, grad_cnt, zero_end;
+    size_t status, ticket, prefix_done, grad_head, resq_head, resq_tail;
+    size_t path_cnt, prefix_cnt, ready, grad_cnt, row_seg_cnt, res_seg_cnt, resq_flag, zero_end;
     size_t rows, rstats, es_tok, es_corr, es_lq_tok, es_lq_corr, es_lk, es_lkc, es_lkr;
-    size_t coef, wscr, total;
+    size_t coef, wscr, path_A, resq, gtab, total;
+    int nch_ws, nseg_ws;
 };
+
+// Chunks per segment of the fused kernel's work items.
+#ifndef VSD_SEG_CHUNKS
+#define VSD_SEG_CHUNKS 64
+#endif
+constexpr int kSegChunks = VSD_SEG_CHUNKS;
+
+// Upper bounds of the chunk count and segment count of a row over both logit
+// dtypes (the smaller float32 chunk gives the larger count).
+int chunks_upper(int V) { return (V + chunk_elems<float>() - 1) / chunk_elems<float>(); }
 
 bool layout_ok(const vsd_layout& L) {
     if (L.B < 1 || L.V < 1 || L.V > kMaxV) return false;
@@ -47,15 +59,24 @@ WsLayout ws_layout(const vsd_layout& L) {
     const size_t R = (size_t)rows_of(L);
     const size_t npath = L.parent ? (size_t)L.B : (size_t)L.B * L.K;
     size_t o = 0;
+    w.nch_ws = chunks_upper(L.V);
+    w.nseg_ws = (w.nch_ws + kSegChunks - 1) / kSegChunks;
+    const size_t nseg = (size_t)w.nseg_ws;
+    // hot counters on separate 256-byte lines (distinct L2 lines and slices)
     w.status = 0;
-    w.ticket = 4;
-    w.prefix_done = 8;
-    w.grad_head = 12;
-    o = 256;
+    w.ticket = 256;
+    w.prefix_done = 512;
+    w.grad_head = 768;
+    w.resq_head = 1024;
+    w.resq_tail = 1280;
+    o = 1536;
     w.path_cnt = o; o = align256(o + 4 * npath);
     w.prefix_cnt = o; o = align256(o + 4 * (size_t)L.B);
     w.ready = o; o = align256(o + 4 * (size_t)L.B);
     w.grad_cnt = o; o = align256(o + 4 * (size_t)L.B);
+    w.row_seg_cnt = o; o = align256(o + 4 * R);
+    w.res_seg_cnt = o; o = align256(o + 4 * npath);
+    w.resq_flag = o; o = align256(o + 4 * npath * nseg);
     w.zero_end = o;
     w.rows = o; o = align256(o + sizeof(RowRec) * R);
     w.rstats = o; o = align256(o + sizeof(float4) * R);
@@ -68,6 +89,9 @@ WsLayout ws_layout(const vsd_layout& L) {
     w.es_lkr = o; o = align256(o + 4 * R);
     w.coef = o; o = align256(o + sizeof(Coef) * R);
     w.wscr = o; o = align256(o + sizeof(double2) * R);
+    w.path_A = o; o = align256(o + 4 * npath);
+    w.resq = o; o = align256(o + 4 * npath * nseg);
+    w.gtab = o; o = align256(o + sizeof(float4) * R * (size_t)w.nch_ws);
     w.total = o;
     return w;
 }
@@ -137,6 +161,7 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.ts.c = (float)(kLog2e / (double)T_);
     P.ts.T = T_;
     P.ts.Td = (double)T_;
+    P.ts.invTd = 1.0 / (double)T_;
     P.parent = L.parent;
     P.w_base = 1.05;
     P.tau_car = 0.2;
@@ -161,6 +186,17 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.es.lkr = at<float>(ws, w.es_lkr);
     P.coef = at<Coef>(ws, w.coef);
     P.wscr = at<double2>(ws, w.wscr);
+    P.segc = kSegChunks;
+    P.nseg = (P.nch + kSegChunks - 1) / kSegChunks;
+    P.nch_ws = w.nch_ws;
+    P.gtab = at<float4>(ws, w.gtab);
+    P.row_seg_cnt = at<int>(ws, w.row_seg_cnt);
+    P.res_seg_cnt = at<int>(ws, w.res_seg_cnt);
+    P.path_A = at<int>(ws, w.path_A);
+    P.resq = at<int>(ws, w.resq);
+    P.resq_flag = at<int>(ws, w.resq_flag);
+    P.resq_head = at<int>(ws, w.resq_head);
+    P.resq_tail = at<int>(ws, w.resq_tail);
     return P;
 }
 
@@ -258,7 +294,7 @@ vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float
     const size_t gelem = P.grad_bf16 ? 2 : 4;
     const bool vec = vec_ok(draft, target, out->grad, L.V, sizeof(T), gelem);
     const int per_sm = Launch<T>::fused_blocks_per_sm(P, vec, P.grad_bf16);
-    const int64_t tickets = 2 * (int64_t)P.R;
+    const int64_t tickets = 2 * (int64_t)P.R * P.nseg;
     int ctas = per_sm * num_sms();
     if ((int64_t)ctas > tickets) ctas = (int)tickets;
     const char* env_ctas = getenv("VSD_FUSED_CTAS");

@@ -41,6 +41,7 @@ struct TempScale {
     float c;        // log2(e)/T rounded to float
     float T;
     double Td;
+    double invTd;   // 1/T
 };
 
 __device__ __forceinline__ float ex2(float x) {
@@ -214,6 +215,73 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
     return ok != 0;
+}
+
+// ---------------------------------------------------------------- packed f32x2
+// Blackwell executes two float32 add/sub/mul in one instruction on a 64-bit
+// register pair; each lane of the pair is an ordinary IEEE round-to-nearest op.
+__device__ __forceinline__ uint64_t f2(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1,%2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void f2split(uint64_t v, float& lo, float& hi) {
+    asm("mov.b64 {%0,%1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2sub(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ uint64_t f2mul(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ uint64_t f2add(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+// The logits of one 16-byte vector as packed pairs (element 2i in the low half).
+template <typename T> __device__ __forceinline__ void vec_pairs(const uint4& v, uint64_t* p);
+template <> __device__ __forceinline__ void vec_pairs<float>(const uint4& v, uint64_t* p) {
+    p[0] = f2(__uint_as_float(v.x), __uint_as_float(v.y));
+    p[1] = f2(__uint_as_float(v.z), __uint_as_float(v.w));
+}
+__device__ __forceinline__ uint64_t bf16x2_pair(uint32_t u) {
+    return f2(__uint_as_float(u << 16), __uint_as_float(u & 0xFFFF0000u));
+}
+template <> __device__ __forceinline__ void vec_pairs<__nv_bfloat16>(const uint4& v, uint64_t* p) {
+    p[0] = bf16x2_pair(v.x);
+    p[1] = bf16x2_pair(v.y);
+    p[2] = bf16x2_pair(v.z);
+    p[3] = bf16x2_pair(v.w);
+}
+// 2^{(v - m) c} of a packed pair: the same per-element arithmetic as the
+// scalar ex2((v - m) * c).
+__device__ __forceinline__ uint64_t f2_mass(uint64_t v2, uint64_t m2, uint64_t c2) {
+    float lo, hi;
+    f2split(f2mul(f2sub(v2, m2), c2), lo, hi);
+    return f2(ex2(lo), ex2(hi));
+}
+// Max over a lane's chunk vectors (NaN elements are ignored here; they surface
+// through the exponential sums).
+template <typename T> __device__ __forceinline__ float lane_max(const uint4 (&buf)[kLoads]);
+template <> __device__ __forceinline__ float lane_max<float>(const uint4 (&buf)[kLoads]) {
+    float m = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k)
+        m = fmaxf(fmaxf(m, fmaxf(__uint_as_float(buf[k].x), __uint_as_float(buf[k].y))),
+                  fmaxf(__uint_as_float(buf[k].z), __uint_as_float(buf[k].w)));
+    return m;
+}
+template <> __device__ __forceinline__ float lane_max<__nv_bfloat16>(const uint4 (&buf)[kLoads]) {
+    const __nv_bfloat162* w = reinterpret_cast<const __nv_bfloat162*>(&buf[0]);
+    __nv_bfloat162 m = w[0];
+#pragma unroll
+    for (int i = 1; i < 4 * kLoads; ++i) m = __hmax2(m, w[i]);
+    return fmaxf(__low2float(m), __high2float(m));
 }
 
 // ---------------------------------------------------------------- warps

@@ -121,6 +121,17 @@ struct Problem {
     EStepStore es;                // [R] each
     Coef* coef;                   // [R]
     double2* wscr;                // [R] M-step scratch
+    // fused kernel: rows, residual rows and gradient rows are split into
+    // segments of segc chunks (nseg per row)
+    int segc, nseg, nch_ws;       // nch_ws: row stride of gtab (>= nch)
+    float4* gtab;                 // [R][nch_ws] per-chunk tables of each row
+    int* row_seg_cnt;             // [R] segments of a row completed
+    int* res_seg_cnt;             // [B*K] residual segments of a path completed
+    int* path_A;                  // [B*K] accepted length of a path
+    int* resq;                    // [B*K*nseg] residual segment items (path*nseg + seg)
+    int* resq_flag;               // [B*K*nseg] item written
+    int* resq_head;               // next item to take
+    int* resq_tail;               // next free slot
     // outputs (device, caller-owned; null = not written)
     vsd_linear_outputs out;
     vsd_tree_outputs tout;
@@ -135,30 +146,25 @@ __device__ __forceinline__ float mass_rel(float f, float mm, float c) { return e
 // Chunk statistics of one tensor: (max, sum_v 2^{(v - max) c}) over the warp's chunk.
 template <typename T>
 __device__ __forceinline__ float2 chunk_stats(const uint4 (&buf)[kLoads], float c) {
-    constexpr int PV = Traits<T>::kPerVec;
-    float mk[kLoads];
-#pragma unroll
-    for (int k = 0; k < kLoads; ++k) mk[k] = vec_max<T>(buf[k]);
-    float m = mk[0];
-#pragma unroll
-    for (int k = 1; k < kLoads; ++k) m = fmaxf(m, mk[k]);
-    m = warp_max(m);
+    constexpr int NP = Traits<T>::kPerVec / 2;
+    const float m = warp_max(lane_max<T>(buf));
     const float mm = frame_of(m);
-    float s[kLoads];
+    const uint64_t mm2 = f2(mm, mm), c2 = f2(c, c);
+    uint64_t acc0 = f2(0.f, 0.f), acc1 = acc0;
 #pragma unroll
     for (int k = 0; k < kLoads; ++k) {
-        float f[PV];
-        unpack<T>(buf[k], f);
-        float a = 0.f;
+        uint64_t pr[NP];
+        vec_pairs<T>(buf[k], pr);
 #pragma unroll
-        for (int e = 0; e < PV; ++e) a += mass_rel(f[e], mm, c);
-        s[k] = a;
+        for (int i = 0; i < NP; ++i) {
+            const uint64_t e2 = f2_mass(pr[i], mm2, c2);
+            if (i & 1) acc1 = f2add(acc1, e2);
+            else acc0 = f2add(acc0, e2);
+        }
     }
-    float t = s[0];
-#pragma unroll
-    for (int k = 1; k < kLoads; ++k) t += s[k];
-    t = warp_sum(t);
-    return make_float2(m, t);
+    float lo, hi;
+    f2split(f2add(acc0, acc1), lo, hi);
+    return make_float2(m, warp_sum(lo + hi));
 }
 
 // --------------------------------------------------------------- TMA ring
@@ -200,22 +206,23 @@ __device__ __forceinline__ bool ring_wait(uint64_t* bar, uint32_t parity, int* s
     }
 }
 
-// Warp-level stream of this warp's chunks (warp, warp + kWarps, ...) of row x
-// (and y) through the ring; consume(ch, bx, by) gets each chunk in registers
-// (positions at or beyond V read as -inf).  Rows must be 16-byte aligned with
-// V * sizeof(T) a multiple of 16.
+// Warp-level stream of this warp's chunks (ch0 + warp, ch0 + warp + kWarps,
+// ... < ch1) of row x (and y) through the ring; consume(ch, bx, by) gets each
+// chunk in registers (positions at or beyond V read as -inf).  Rows must be
+// 16-byte aligned with V * sizeof(T) a multiple of 16.
 template <typename T, bool HAS_Y, class Consume>
-__device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, int64_t V, int nch,
-                                            uint64_t polx, uint64_t poly, int* status,
+__device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, int64_t V, int ch0,
+                                            int ch1, uint64_t polx, uint64_t poly, int* status,
                                             Consume&& consume) {
     constexpr int PV = Traits<T>::kPerVec;
     constexpr int CE = chunk_elems<T>();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nj = nch > warp ? (nch - warp + kWarps - 1) / kWarps : 0;
+    const int nrange = ch1 - ch0;
+    const int nj = nrange > warp ? (nrange - warp + kWarps - 1) / kWarps : 0;
     const int pos = rg->pos[warp];
     bool broken = rg->broken[warp] != 0;
     auto issue = [&](int j) {
-        const int ch = warp + j * kWarps;
+        const int ch = ch0 + warp + j * kWarps;
         const int slot = (pos + j) % kStages;
         const int64_t e0 = (int64_t)ch * CE;
         const int64_t ne = V - e0 < CE ? V - e0 : CE;
@@ -233,16 +240,24 @@ __device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, in
         const uint32_t parity = (uint32_t)((pos + j) / kStages) & 1u;
         bool ok = broken ? false : ring_wait(&rg->bar[warp][slot], parity, status);
         broken = __any_sync(0xffffffffu, !ok);
-        const int ch = warp + j * kWarps;
+        const int ch = ch0 + warp + j * kWarps;
         const int64_t e0 = (int64_t)ch * CE;
         uint4 bx[kLoads], by[kLoads];
+        if (e0 + CE <= V) {  // full chunk (all but possibly the row's last)
 #pragma unroll
-        for (int k = 0; k < kLoads; ++k) {
-            const bool in = e0 + (int64_t)k * 32 * PV + lane * PV < V;
-            const uint4 ninf = make_uint4(Traits<T>::kNegInf, Traits<T>::kNegInf,
-                                          Traits<T>::kNegInf, Traits<T>::kNegInf);
-            bx[k] = in ? rg->data[warp][slot][0][k * 32 + lane] : ninf;
-            if (HAS_Y) by[k] = in ? rg->data[warp][slot][1][k * 32 + lane] : ninf;
+            for (int k = 0; k < kLoads; ++k) {
+                bx[k] = rg->data[warp][slot][0][k * 32 + lane];
+                if (HAS_Y) by[k] = rg->data[warp][slot][1][k * 32 + lane];
+            }
+        } else {
+#pragma unroll
+            for (int k = 0; k < kLoads; ++k) {
+                const bool in = e0 + (int64_t)k * 32 * PV + lane * PV < V;
+                const uint4 ninf = make_uint4(Traits<T>::kNegInf, Traits<T>::kNegInf,
+                                              Traits<T>::kNegInf, Traits<T>::kNegInf);
+                bx[k] = in ? rg->data[warp][slot][0][k * 32 + lane] : ninf;
+                if (HAS_Y) by[k] = in ? rg->data[warp][slot][1][k * 32 + lane] : ninf;
+            }
         }
         __syncwarp();
         if (lane == 0 && !broken && j + kStages < nj) issue(j + kStages);
@@ -256,16 +271,17 @@ __device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, in
     __syncwarp();
 }
 
-// Stream a row (and optionally its target row) once, filling tab[c] =
-// (max_x, sum_x, max_y, sum_y) for every chunk c.  Warps take chunks
-// round-robin and keep the next chunk's loads in flight.
+// Stream chunks [ch0, ch1) of a row (and optionally its target row) once,
+// filling tab[c] = (max_x, sum_x, max_y, sum_y) for each chunk c (tab is a
+// shared-memory table or a row's table in global memory).  Warps take chunks
+// round-robin and keep the next chunks' loads in flight.
 template <typename T, bool VEC, bool HAS_Y>
-__device__ __forceinline__ void stream_tables(Ring* rg, const T* x, const T* y, int64_t V, int nch,
-                                              float4* tab, float c, uint64_t polx,
+__device__ __forceinline__ void stream_tables(Ring* rg, const T* x, const T* y, int64_t V, int ch0,
+                                              int ch1, float4* tab, float c, uint64_t polx,
                                               uint64_t poly, int* status) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if constexpr (VEC) {
-        ring_stream<T, HAS_Y>(rg, x, y, V, nch, polx, poly, status,
+        ring_stream<T, HAS_Y>(rg, x, y, V, ch0, ch1, polx, poly, status,
                               [&](int ch, const uint4 (&bx)[kLoads], const uint4 (&by)[kLoads]) {
                                   const float2 sx = chunk_stats<T>(bx, c);
                                   float2 sy = make_float2(0.f, 0.f);
@@ -274,16 +290,16 @@ __device__ __forceinline__ void stream_tables(Ring* rg, const T* x, const T* y, 
                               });
         return;
     }
-    int ch = warp;
+    int ch = ch0 + warp;
     uint4 bx[kLoads], by[kLoads];
-    if (ch < nch) {
+    if (ch < ch1) {
         load_chunk<T, VEC>(x, V, ch, lane, polx, bx);
         if (HAS_Y) load_chunk<T, VEC>(y, V, ch, lane, poly, by);
     }
-    while (ch < nch) {
+    while (ch < ch1) {
         const int cn = ch + kWarps;
         uint4 nx[kLoads], ny[kLoads];
-        if (cn < nch) {
+        if (cn < ch1) {
             load_chunk<T, VEC>(x, V, cn, lane, polx, nx);
             if (HAS_Y) load_chunk<T, VEC>(y, V, cn, lane, poly, ny);
         }
@@ -492,9 +508,9 @@ __device__ __forceinline__ bool row_ok(float M, double Z) {
 // log q and log alpha = min(0, log p - log q) of token v (Eq. 1), in double.
 template <typename T>
 __device__ __forceinline__ void token_logs(const T* x, const T* y, int v, const RowRec& rec,
-                                           double Td, float* lq, float* la) {
-    const double lqd = ((double)elem_value(x, v) - (double)rec.mx) / Td - rec.lzx;
-    const double lpd = ((double)elem_value(y, v) - (double)rec.my) / Td - rec.lzy;
+                                           double invT, float* lq, float* la) {
+    const double lqd = ((double)elem_value(x, v) - (double)rec.mx) * invT - rec.lzx;
+    const double lpd = ((double)elem_value(y, v) - (double)rec.my) * invT - rec.lzy;
     const double d = lpd - lqd;
     *lq = (float)lqd;
     *la = (float)(d >= 0.0 ? 0.0 : d);
@@ -503,28 +519,23 @@ __device__ __forceinline__ void token_logs(const T* x, const T* y, int v, const 
 // --------------------------------------------------------------- row pass
 struct RowShared {
     float Mx, My;
-    double Zx, Zy;
+    double Zx, Zy, lzx, lzy;
     int tok, ps, ref;
     float lq[3], la[3];
 };
 
 enum XMode { kNoToken = 0, kSampleToken = 1, kGivenToken = 2 };
 
-// Streams row r of the draft (and, with HAS_Y, of the target) once and
-// writes rows[r] and rstats[r].  XMODE: whether z~ is drawn from q with
-// u_draft, read from given_tokens, or absent (trees).  ARGMAX: locate the
-// greedy reference token.
+// The per-row work once the row's chunk table tab[0..nch) is complete in
+// shared memory (block): row statistics, the draws, the argmax, the token
+// log-probabilities; writes rows[r] and rstats[r].
 template <typename T, bool VEC, bool HAS_Y, int XMODE, bool ARGMAX>
-__device__ void row_pass(const Problem<T>& P, int r, Ring* rg, float4* tab, RowShared& sh) {
+__device__ void row_tail(const Problem<T>& P, int r, const float4* tab, RowShared& sh) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t V = P.V;
     const T* x = P.draft + (int64_t)r * V;
     const T* y = HAS_Y ? P.target + (int64_t)r * V : nullptr;
     const float c = P.ts.c;
-    // The draft row is read again by the gradient pass: ask L2 to keep it.
-    stream_tables<T, VEC, HAS_Y>(rg, x, y, V, P.nch, tab, c, policy_evict_last(),
-                                 policy_evict_first(), P.status);
-    __syncthreads();
     const uint64_t pol = policy_evict_normal();
     if (warp == 0) {
         const float M = table_max(tab, P.nch, 0, lane);
@@ -538,7 +549,12 @@ __device__ void row_pass(const Problem<T>& P, int r, Ring* rg, float4* tab, RowS
             tok = __ldg(P.given_tokens + r);
         }
         if (XMODE == kSampleToken && (tok < 0 || tok >= V)) tok = -1;
-        if (lane == 0) { sh.Mx = M; sh.Zx = Z; sh.tok = tok; }
+        if (lane == 0) {
+            sh.Mx = M;
+            sh.Zx = Z;
+            sh.lzx = row_ok(M, Z) ? log(Z) : 0.0;
+            sh.tok = tok;
+        }
     } else if (HAS_Y && warp == 1) {
         const float M = table_max(tab, P.nch, 1, lane);
         const double Z = table_total(tab, P.nch, 1, frame_of(M), c, lane);
@@ -547,7 +563,12 @@ __device__ void row_pass(const Problem<T>& P, int r, Ring* rg, float4* tab, RowS
             ps = warp_sample<T, VEC>(x, y, V, tab, P.nch, 1, M, Z, __ldg(P.u_correct + r), c,
                                      lane, pol);
         if (ps >= V) ps = -1;
-        if (lane == 0) { sh.My = M; sh.Zy = Z; sh.ps = ps; }
+        if (lane == 0) {
+            sh.My = M;
+            sh.Zy = Z;
+            sh.lzy = row_ok(M, Z) ? log(Z) : 0.0;
+            sh.ps = ps;
+        }
     } else if (HAS_Y && ARGMAX && warp == 2) {
         const float M = table_max(tab, P.nch, 1, lane);
         const int ref =
@@ -556,7 +577,7 @@ __device__ void row_pass(const Problem<T>& P, int r, Ring* rg, float4* tab, RowS
     }
     __syncthreads();
     // log q and log alpha of z~, of the p-draw and of the argmax: one lane each.
-    const double Td = P.ts.Td;
+    const double invT = P.ts.invTd;
     const bool okx = row_ok(sh.Mx, sh.Zx);
     const bool oky = HAS_Y ? row_ok(sh.My, sh.Zy) : true;
     const bool ok = okx && oky;
@@ -570,13 +591,13 @@ __device__ void row_pass(const Problem<T>& P, int r, Ring* rg, float4* tab, RowS
         if (want && ok && v >= 0 && v < V) {
             RowRec tmp;
             tmp.mx = sh.Mx;
-            tmp.lzx = log(sh.Zx);
+            tmp.lzx = sh.lzx;
             tmp.my = HAS_Y ? sh.My : 0.f;
-            tmp.lzy = HAS_Y ? log(sh.Zy) : 0.0;
+            tmp.lzy = HAS_Y ? sh.lzy : 0.0;
             if (HAS_Y)
-                token_logs(x, y, v, tmp, Td, &lq, &la);
+                token_logs(x, y, v, tmp, invT, &lq, &la);
             else
-                lq = (float)(((double)elem_value(x, v) - (double)tmp.mx) / Td - tmp.lzx);
+                lq = (float)(((double)elem_value(x, v) - (double)tmp.mx) * invT - tmp.lzx);
         }
         sh.lq[which] = lq;
         sh.la[which] = la;
@@ -585,9 +606,9 @@ __device__ void row_pass(const Problem<T>& P, int r, Ring* rg, float4* tab, RowS
     if (threadIdx.x == 0) {
         RowRec rec;
         rec.mx = sh.Mx;
-        rec.lzx = okx ? log(sh.Zx) : 0.0;
+        rec.lzx = okx ? sh.lzx : 0.0;
         rec.my = HAS_Y ? sh.My : 0.f;
-        rec.lzy = (HAS_Y && oky) ? log(sh.Zy) : 0.0;
+        rec.lzy = (HAS_Y && oky) ? sh.lzy : 0.0;
         rec.flags = ok ? 0 : 1;
         if (!ok) atomicOr(P.status, VSD_STATUS_BAD_ROW);
         int t = tok;
@@ -609,53 +630,71 @@ __device__ void row_pass(const Problem<T>& P, int r, Ring* rg, float4* tab, RowS
     }
 }
 
+// Streams row r of the draft (and, with HAS_Y, of the target) once, then runs
+// row_tail.  XMODE: whether z~ is drawn from q with u_draft, read from
+// given_tokens, or absent (trees).  ARGMAX: locate the greedy reference token.
+template <typename T, bool VEC, bool HAS_Y, int XMODE, bool ARGMAX>
+__device__ void row_pass(const Problem<T>& P, int r, Ring* rg, float4* tab, RowShared& sh) {
+    const int64_t V = P.V;
+    const T* x = P.draft + (int64_t)r * V;
+    const T* y = HAS_Y ? P.target + (int64_t)r * V : nullptr;
+    // The draft row is read again by the gradient pass: ask L2 to keep it.
+    stream_tables<T, VEC, HAS_Y>(rg, x, y, V, 0, P.nch, tab, P.ts.c, policy_evict_last(),
+                                 policy_evict_first(), P.status);
+    __syncthreads();
+    row_tail<T, VEC, HAS_Y, XMODE, ARGMAX>(P, r, tab, sh);
+}
+
 // --------------------------------------------------------------- residual
 // Stream rows x, y once more and fill tab[c].y with the chunk sums of the
 // residual mass max(0, p - q).
 template <typename T>
 __device__ __forceinline__ float residual_chunk(const uint4 (&bx)[kLoads], const uint4 (&by)[kLoads],
                                                const MassRes& mr) {
-    constexpr int PV = Traits<T>::kPerVec;
-    float s4[kLoads];
+    constexpr int NP = Traits<T>::kPerVec / 2;
+    const uint64_t mx2 = f2(mr.mx, mr.mx), my2 = f2(mr.my, mr.my), c2 = f2(mr.c, mr.c);
+    const uint64_t izx2 = f2(mr.izx, mr.izx), izy2 = f2(mr.izy, mr.izy);
+    float acc = 0.f;
 #pragma unroll
     for (int k = 0; k < kLoads; ++k) {
-        float fx[PV], fy[PV];
-        unpack<T>(bx[k], fx);
-        unpack<T>(by[k], fy);
-        float a = 0.f;
+        uint64_t px[NP], py[NP];
+        vec_pairs<T>(bx[k], px);
+        vec_pairs<T>(by[k], py);
 #pragma unroll
-        for (int e = 0; e < PV; ++e) a += mr(fx[e], fy[e]);
-        s4[k] = a;
+        for (int i = 0; i < NP; ++i) {
+            const uint64_t q2 = f2mul(f2_mass(px[i], mx2, c2), izx2);
+            const uint64_t p2 = f2mul(f2_mass(py[i], my2, c2), izy2);
+            float lo, hi;
+            f2split(f2sub(p2, q2), lo, hi);
+            acc += fmaxf(lo, 0.f) + fmaxf(hi, 0.f);
+        }
     }
-    float t = s4[0];
-#pragma unroll
-    for (int k = 1; k < kLoads; ++k) t += s4[k];
-    return warp_sum(t);
+    return warp_sum(acc);
 }
 
 template <typename T, bool VEC>
-__device__ void stream_residual(Ring* rg, const T* x, const T* y, int64_t V, int nch, float4* tab,
-                                const MassRes& mr, int* status) {
+__device__ void stream_residual(Ring* rg, const T* x, const T* y, int64_t V, int ch0, int ch1,
+                                float4* tab, const MassRes& mr, int* status) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint64_t pol = policy_evict_normal();
     if constexpr (VEC) {
-        ring_stream<T, true>(rg, x, y, V, nch, pol, pol, status,
+        ring_stream<T, true>(rg, x, y, V, ch0, ch1, pol, pol, status,
                              [&](int ch, const uint4 (&bx)[kLoads], const uint4 (&by)[kLoads]) {
                                  const float t = residual_chunk<T>(bx, by, mr);
                                  if (lane == 0) tab[ch] = make_float4(0.f, t, 0.f, 0.f);
                              });
         return;
     }
-    int ch = warp;
+    int ch = ch0 + warp;
     uint4 bx[kLoads], by[kLoads];
-    if (ch < nch) {
+    if (ch < ch1) {
         load_chunk<T, VEC>(x, V, ch, lane, pol, bx);
         load_chunk<T, VEC>(y, V, ch, lane, pol, by);
     }
-    while (ch < nch) {
+    while (ch < ch1) {
         const int cn = ch + kWarps;
         uint4 nx[kLoads], ny[kLoads];
-        if (cn < nch) {
+        if (cn < ch1) {
             load_chunk<T, VEC>(x, V, cn, lane, pol, nx);
             load_chunk<T, VEC>(y, V, cn, lane, pol, ny);
         }
@@ -681,7 +720,7 @@ __device__ int residual_draw(const Problem<T>& P, int r, const RowRec& rec, floa
     const T* y = P.target + (int64_t)r * V;
     const float c = P.ts.c;
     const MassRes mr{rec.mx, rec.my, (float)exp(-rec.lzx), (float)exp(-rec.lzy), c};
-    stream_residual<T, VEC>(rg, x, y, V, P.nch, tab, mr, P.status);
+    stream_residual<T, VEC>(rg, x, y, V, 0, P.nch, tab, mr, P.status);
     __syncthreads();
     if (warp == 0) {
         const double Rt = table_total(tab, P.nch, 0, 0.f, c, lane);
@@ -709,7 +748,7 @@ __device__ int p_draw(const Problem<T>& P, int r, float u, Ring* rg, float4* tab
     const T* y = P.target + (int64_t)r * V;
     const float c = P.ts.c;
     const uint64_t pol = policy_evict_normal();
-    stream_tables<T, VEC, false>(rg, y, nullptr, V, P.nch, tab, c, pol, pol, P.status);
+    stream_tables<T, VEC, false>(rg, y, nullptr, V, 0, P.nch, tab, c, pol, pol, P.status);
     __syncthreads();
     if (warp == 0) {
         const float M = table_max(tab, P.nch, 0, lane);
@@ -732,11 +771,11 @@ struct PathShared {
     RowRec rec;
 };
 
-// Linear proposal path (b, s) = path: rows path*D .. path*D + D - 1.  Warp 0
-// handles the rows lane-parallel (two rounds when D > 32) with warp scans for
-// the prefix sums over l; the whole block streams the residual row.
-template <typename T, bool VEC>
-__device__ void path_pass(const Problem<T>& P, int path, Ring* rg, float4* tab, PathShared& sh) {
+// Linear proposal path (b, s) = path: rows path*D .. path*D + D - 1.
+// path_head (warp 0): the accepted length A (first rejection by ballot) and,
+// if A < D, the record of row A.  Written to sh.A, sh.rec.
+template <typename T>
+__device__ void path_head(const Problem<T>& P, int path, PathShared& sh) {
     const int D = P.D;
     const int r0 = path * D;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -758,12 +797,17 @@ __device__ void path_pass(const Problem<T>& P, int path, Ring* rg, float4* tab, 
             if (A < D) sh.rec = ld_cg(P.rows + r0 + A);
         }
     }
-    __syncthreads();
-    const int A = sh.A;
-    int resid = -1;
-    if (A < D && !sh.rec.flags)
-        resid = residual_draw<T, VEC>(P, r0 + A, sh.rec, __ldg(P.u_correct + r0 + A), rg, tab,
-                                      &sh.resid);
+}
+
+// path_epilogue (warp 0): given A and the residual token at row A (-1: none
+// or no residual mass), the corrected path, alpha', the log-kappa prefix sums
+// of z~, z' and the reference (Eq. 2, warp scans), E[A] (Eq. 11); writes the
+// E-step view and the requested outputs.
+template <typename T>
+__device__ void path_epilogue(const Problem<T>& P, int path, int A, int resid) {
+    const int D = P.D;
+    const int r0 = path * D;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (warp == 0) {
         const int b = path / P.K;
         const double NEG = -INFINITY;
@@ -791,7 +835,7 @@ __device__ void path_pass(const Problem<T>& P, int path, Ring* rg, float4* tab, 
                         lqc = rec.lq_ps; lac = rec.la_ps;
                     } else {
                         token_logs(P.draft + (int64_t)r * V, P.target + (int64_t)r * V, zc, rec,
-                                   P.ts.Td, &lqc, &lac);
+                                   P.ts.invTd, &lqc, &lac);
                     }
                 } else {
                     zc = rec.ps; lqc = rec.lq_ps; lac = rec.la_ps;
@@ -842,10 +886,29 @@ __device__ void path_pass(const Problem<T>& P, int path, Ring* rg, float4* tab, 
     }
 }
 
+
+// The whole path (block): head, the residual draw at the first rejection (one
+// more streaming read of that row), epilogue.
+template <typename T, bool VEC>
+__device__ void path_pass(const Problem<T>& P, int path, Ring* rg, float4* tab, PathShared& sh) {
+    const int D = P.D;
+    const int r0 = path * D;
+    path_head<T>(P, path, sh);
+    __syncthreads();
+    const int A = sh.A;
+    int resid = -1;
+    if (A < D && !sh.rec.flags)
+        resid = residual_draw<T, VEC>(P, r0 + A, sh.rec, __ldg(P.u_correct + r0 + A), rg, tab,
+                                      &sh.resid);
+    path_epilogue<T>(P, path, A, resid);
+}
+
 // --------------------------------------------------------------- weights
 struct WeightsShared {
-    double ot[256], op[256], cq[256], lqt[256], lqc[256];
+    double ot[256], op[256], lqt[256], lqc[256], cq[256];
+    float ez[256];
     double red[kThreads];
+    double w, cmax;
 };
 
 __device__ __forceinline__ double block_sum(double v, double* red) {
@@ -870,8 +933,9 @@ __device__ void weights_pass(const Problem<T>& P, const EStepView& E, int b, flo
     double Jp = 0.0, Np = 0.0;
     for (int s = threadIdx.x; s < K; s += kThreads) sh.lqt[s] = sh.lqc[s] = 0.0;
     for (int d = 0; d < D; ++d) {
-        const int l = d + 1;
-        const double w = pow(P.w_base, (double)l);  // w(l), App. F
+        if (threadIdx.x == 0) sh.w = pow(P.w_base, (double)(d + 1));  // w(l), App. F
+        __syncthreads();
+        const double w = sh.w;
         for (int s = threadIdx.x; s < K; s += kThreads) {
             const int r = (b * K + s) * D + d;
             const double lk = ld_cg(E.lk + r), lkc = ld_cg(E.lkc + r), lkr = ld_cg(E.lkr + r);
@@ -884,16 +948,24 @@ __device__ void weights_pass(const Problem<T>& P, const EStepView& E, int b, flo
             sh.cq[s] = (P.zeta_mode == 0 ? exp(sh.lqt[s]) : sh.lqt[s]) / P.tau_car;
         }
         __syncthreads();
+        if (threadIdx.x < 32) {  // max of the CAR logits over the K proposals
+            double m = -INFINITY;
+            for (int j = threadIdx.x; j < K; j += 32) m = fmax(m, sh.cq[j]);
+#pragma unroll
+            for (int o = 16; o; o >>= 1) m = fmax(m, __shfl_xor_sync(0xffffffffu, m, o));
+            if (threadIdx.x == 0) sh.cmax = m;
+        }
+        __syncthreads();
+        for (int s = threadIdx.x; s < K; s += kThreads) sh.ez[s] = expf((float)(sh.cq[s] - sh.cmax));
+        __syncthreads();
         for (int s = threadIdx.x; s < K; s += kThreads) {
-            double num = 0.0, den = 0.0, M = -INFINITY;
+            double num = 0.0, den = 0.0, Zs = 0.0;
             for (int j = 0; j < K; ++j) {
                 if (j != s) { num += sh.op[j] * sh.ot[j]; den += sh.op[j]; }
-                M = fmax(M, sh.cq[j]);
+                Zs += (double)sh.ez[j];
             }
             const double beta = den > 0.0 ? num / den : 0.0;  // Eq. beta (leave-one-out)
-            double Zs = 0.0;
-            for (int j = 0; j < K; ++j) Zs += exp(sh.cq[j] - M);
-            const double zeta = exp(sh.cq[s] - M) / Zs;        // Eq. zeta
+            const double zeta = (double)sh.ez[s] / Zs;         // Eq. zeta
             const double ot = sh.ot[s], op = sh.op[s];
             const double lqz = ot > 0.0 ? sh.lqt[s] : sh.lqc[s];
             if (op != 0.0) Jp += op * (lqz - beta * zeta * sh.lqt[s]);  // Eq. advance
@@ -966,10 +1038,13 @@ __device__ __forceinline__ void grad_store(G* g, int64_t v0, const float (&o)[PV
     }
 }
 
+// Gradient of elements [e0, e1) of row r (block).  On the vector path e0 and
+// e1 are multiples of the vector width.
 template <typename T, bool VEC, typename G>
-__device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* grad) {
+__device__ void grad_pass_range(const Problem<T>& P, int r, int64_t e0, int64_t e1,
+                                const float4* rstats, G* grad) {
     constexpr int PV = Traits<T>::kPerVec;
-    constexpr int U = 8;  // vectors in flight per thread
+    constexpr int U = 8;  // vectors per batch per thread (two batches in flight)
     const int64_t V = P.V;
     const T* x = P.draft + (int64_t)r * V;
     G* g = grad + (int64_t)r * V;
@@ -980,34 +1055,53 @@ __device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* g
     const float gq = (float)((double)cf.g * exp(-(double)st.y));
     const uint64_t pol = policy_evict_first();
     if constexpr (VEC) {
-        const int64_t nvec = V / PV;
-        for (int64_t i0 = threadIdx.x; i0 < nvec; i0 += (int64_t)kThreads * U) {
-            uint4 raw[U];
+        constexpr int NP = PV / 2;
+        const uint64_t mx2 = f2(mx, mx), c2 = f2(c, c), gq2 = f2(gq, gq);
+        const int nvec = (int)(e1 / PV);
+        const int ib = (int)(e0 / PV) + threadIdx.x;
+        uint4 cur[U], nxt[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int i = ib + u * kThreads;
+            if (i < nvec) cur[u] = ld_stream(x + (int64_t)i * PV, pol);
+        }
+        for (int i0 = ib; i0 < nvec; i0 += kThreads * U) {
+            // the next batch is in flight while this one is computed and stored
+            const int in = i0 + kThreads * U;
 #pragma unroll
             for (int u = 0; u < U; ++u) {
-                const int64_t i = i0 + (int64_t)u * kThreads;
-                if (i < nvec) raw[u] = ld_stream(x + i * PV, pol);
+                const int i = in + u * kThreads;
+                if (i < nvec) nxt[u] = ld_stream(x + (int64_t)i * PV, pol);
             }
 #pragma unroll
             for (int u = 0; u < U; ++u) {
-                const int64_t i = i0 + (int64_t)u * kThreads;
+                const int i = i0 + u * kThreads;
                 if (i >= nvec) break;
-                const int64_t v0 = i * PV;
-                float f[PV], o[PV];
-                unpack<T>(raw[u], f);
+                const int v0 = i * PV;
+                uint64_t pr[NP];
+                vec_pairs<T>(cur[u], pr);
+                float o[PV];
 #pragma unroll
-                for (int e = 0; e < PV; ++e) {
-                    float val = gq * ex2((f[e] - mx) * c);
-                    const int64_t v = v0 + e;
-                    if (v == cf.t0) val -= cf.c0;
-                    if (v == cf.t1) val -= cf.c1;
-                    o[e] = val;
+                for (int k = 0; k < NP; ++k)
+                    f2split(f2mul(f2_mass(pr[k], mx2, c2), gq2), o[2 * k], o[2 * k + 1]);
+                // the sparse terms touch at most two positions of the row
+                if ((unsigned)(cf.t0 - v0) < (unsigned)PV) {
+#pragma unroll
+                    for (int e = 0; e < PV; ++e)
+                        if (v0 + e == cf.t0) o[e] -= cf.c0;
+                }
+                if ((unsigned)(cf.t1 - v0) < (unsigned)PV) {
+#pragma unroll
+                    for (int e = 0; e < PV; ++e)
+                        if (v0 + e == cf.t1) o[e] -= cf.c1;
                 }
                 grad_store<T, G, PV>(g, v0, o, pol);
             }
+#pragma unroll
+            for (int u = 0; u < U; ++u) cur[u] = nxt[u];
         }
     } else {
-        for (int64_t v = threadIdx.x; v < V; v += kThreads) {
+        for (int64_t v = e0 + threadIdx.x; v < e1; v += kThreads) {
             float val = gq * ex2((elem_value(x, v) - mx) * c);
             if (v == cf.t0) val -= cf.c0;
             if (v == cf.t1) val -= cf.c1;
@@ -1017,6 +1111,11 @@ __device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* g
                 g[v] = val;
         }
     }
+}
+
+template <typename T, bool VEC, typename G>
+__device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* grad) {
+    grad_pass_range<T, VEC, G>(P, r, 0, P.V, rstats, grad);
 }
 
 // --------------------------------------------------------------- tree pass
@@ -1081,7 +1180,7 @@ __device__ void tree_pass(const Problem<T>& P, int b, Ring* rg, float4* tab, Tre
             } else if (!rec.flags) {
                 float lq, laf;
                 token_logs(P.draft + (int64_t)(n0 + pn) * V, P.target + (int64_t)(n0 + pn) * V,
-                           tok, rec, P.ts.Td, &lq, &laf);
+                           tok, rec, P.ts.invTd, &lq, &laf);
                 la = (double)laf;
             }
             const double a = exp(la);
@@ -1117,7 +1216,7 @@ __device__ void tree_pass(const Problem<T>& P, int b, Ring* rg, float4* tab, Tre
         const float c = P.ts.c;
         const MassRes mr{sh.rec.mx, sh.rec.my, (float)exp(-sh.rec.lzx), (float)exp(-sh.rec.lzy),
                          c};
-        stream_residual<T, VEC>(rg, x, y, V, P.nch, tab, mr, P.status);
+        stream_residual<T, VEC>(rg, x, y, V, 0, P.nch, tab, mr, P.status);
         __syncthreads();
         if (warp == 0) {
             const double Rt = table_total(tab, P.nch, 0, 0.f, c, lane);

@@ -23,7 +23,7 @@ _STATUS_NAMES = {0: "VSD_OK", 1: "VSD_ERR_INVALID_ARG", 2: "VSD_ERR_UNSUPPORTED"
 SYMBOLS = ("vsd_workspace_bytes", "vsd_sample_paths", "vsd_verify_paths",
            "vsd_weighted_loss_fwd_bwd", "vsd_estep_mstep", "vsd_device_status",
            "vsd_status_string", "vsd_version", "vsd_estep_mstep_noalloc")
-NOALLOC_SCRATCH_BYTES = 1 << 20
+NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
 class VsdError(RuntimeError):

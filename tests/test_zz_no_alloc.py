@@ -27,7 +27,7 @@ def vsd():
 def test_rejects_layouts_beyond_the_scratch(vsd):
     """Host-side check, before any CUDA call: too large -> VSD_ERR_TOO_LARGE."""
     lib = vsd.load()
-    lay = vsd.layout(64, 64, 64, 1024)  # needs ~40 MB of scratch
+    lay = vsd.layout(64, 64, 64, 1024)  # needs ~49 MB of scratch
     assert vsd.workspace_bytes(lay) > vsd.NOALLOC_SCRATCH_BYTES
     fake = C.c_void_p(0x1000)  # never dereferenced: the size check fails first
     outs = vsd.LinearOutputs(*([0x1000] * len(vsd.LINEAR_FIELDS)))
