@@ -144,6 +144,13 @@ vsd_status check_params(const vsd_params& p) {
 }
 
 // Fill the shape, temperature, workspace views of a problem.
+// w(l) = w_base^l for l = 1 .. D, with the host's pow, and 1 / tau_car.
+template <typename T>
+void fill_wl(Problem<T>& P) {
+    for (int d = 0; d < 64; ++d) P.wl[d] = d < P.D ? pow(P.w_base, (double)(d + 1)) : 0.0;
+    P.inv_tau = 1.0 / P.tau_car;
+}
+
 template <typename T>
 Problem<T> make_problem(const void* draft, const void* target, const vsd_layout& L, float T_,
                         void* ws) {
@@ -165,6 +172,7 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.parent = L.parent;
     P.w_base = 1.05;
     P.tau_car = 0.2;
+    fill_wl(P);
     P.timeout_ns = kDefaultTimeoutNs;
     const WsLayout w = ws_layout(L);
     P.status = at<int>(ws, w.status);
@@ -208,6 +216,7 @@ void set_params(Problem<T>& P, const vsd_params& p) {
     P.grad_bf16 = p.grad_dtype == VSD_BF16;
     P.timeout_ns = p.wait_timeout_ns ? p.wait_timeout_ns : kDefaultTimeoutNs;
     P.inject_wait_fault = p.test_never_publish;
+    fill_wl(P);
 }
 
 cudaError_t clear_counters(void* ws, const vsd_layout& L, cudaStream_t s) {

@@ -217,6 +217,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
+// 16-byte asynchronous copy global -> shared that bypasses registers; with
+// valid = false nothing is read and the 16 bytes are zero-filled.
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;"
+                 :: "r"(smem_u32(dst)), "l"(src), "r"(valid ? 16u : 0u) : "memory");
+}
+// Wait for all of this thread's cp.async copies.
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- packed f32x2
 // Blackwell executes two float32 add/sub/mul in one instruction on a 64-bit
 // register pair; each lane of the pair is an ordinary IEEE round-to-nearest op.

@@ -108,47 +108,241 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int* status, uint64_t
     }
 }
 
-// End of a path (block): epilogue, then the prefix counter; the block that
-// completes the prefix's last path runs its M-step and publishes it.
+// The fused kernel's block: kWarps streaming warps (threads 0 .. kThreads-1)
+// that only move logits, and one control warp (the last) that claims work,
+// keeps the counters and runs every per-row, per-path and per-prefix step.
+constexpr int kFusedThreads = kThreads + 32;
+constexpr int kSlots = 3;  // jobs handed to the streaming warps ahead of time
+// Named barriers (0 is __syncthreads): slot s is FULL (1 + s) when the control
+// warp has written a job into it, DONE (1 + kSlots + s) when the streaming
+// warps have finished that job.
+__device__ __forceinline__ int bar_full(int s) { return 1 + s; }
+__device__ __forceinline__ int bar_done(int s) { return 1 + kSlots + s; }
+__device__ __forceinline__ void named_sync(int id) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(kFusedThreads) : "memory");
+}
+__device__ __forceinline__ void named_arrive(int id) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(kFusedThreads) : "memory");
+}
+
+enum JobKind { kJobEnd = 0, kJobRow = 1, kJobGrad = 2, kJobResidual = 3 };
+struct Job {
+    int kind;
+    int r;       // the row streamed (residual: row A of the path)
+    int item;    // row segment or residual item index
+    int c0, c1;  // chunk range of the segment
+    int path, A;
+    MassRes mr;  // residual segment: the row's normalisers
+};
+
+// Claim the next job (lane 0 of the control warp), in this order of priority:
+//   1. a residual segment from the queue (residual draws gate a prefix's M-step),
+//   2. a gradient segment of the oldest prefix whose M-step is published,
+//   3. the next logit-row segment (rows in prefix order).
+// With wait = false returns false at once when nothing is available; with
+// wait = true polls (bounded by the wait timeout) until a job or the end.
+// The caller may only wait when it has no job in flight whose follow-up steps
+// it still owes, so that no block waits on work that it holds itself.
 template <typename T>
-__device__ void finish_path(const Problem<T>& P, const EStepView& E, int path, int A, int resid,
-                            WeightsShared& wsh, int* s_flag) {
-    path_epilogue<T>(P, path, A, resid);
-    __syncthreads();
-    const int prefix = path / P.K;
-    if (threadIdx.x == 0) {
-        __threadfence();
-        *s_flag = atomicAdd(P.prefix_cnt + prefix, 1) == P.K - 1;
-        if (*s_flag) __threadfence();
-    }
-    __syncthreads();
-    if (*s_flag) {
-        weights_pass<T>(P, E, prefix, P.out.weights, P.out.loss, wsh);
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            __threadfence();
-            if (!P.inject_wait_fault) st_release(P.ready + prefix, 1);
-            if (atomicAdd(P.prefix_done, 1) == P.B - 1) {
-                __threadfence();
-                loss_mean(P.out.loss, P.B);
+__device__ bool claim_job(const Problem<T>& P, bool wait, int& g, Job& j) {
+    const int B = P.B, nseg = P.nseg, segc = P.segc;
+    const int row_items = P.R * nseg;
+    const int grad_items = P.K * P.D * nseg;  // per prefix
+    uint64_t idle_since = 0;
+    j.kind = kJobEnd;
+    for (;;) {
+        // independent reads first (one round trip), then at most one attempt
+        // per kind of work
+        const int h = *(volatile int*)P.resq_head;
+        const int tl = *(volatile int*)P.resq_tail;
+        const int tk = *(volatile int*)P.ticket;
+        const int rdy = g < B ? ld_acquire(P.ready + g) : 0;
+        if (h < tl && atomicCAS(P.resq_head, h, h + 1) == h) {
+            if (!wait_flag(P.resq_flag + h, P.status, P.timeout_ns)) {
+                atomicOr(P.status, VSD_STATUS_TIMEOUT);
+                return true;  // end
             }
+            const int it = ld_cg(P.resq + h);
+            const int path = it / nseg, seg = it - path * nseg;
+            const int A = ld_cg(P.path_A + path);
+            const int rA = path * P.D + A;
+            const RowRec rec = ld_cg(P.rows + rA);
+            j.kind = kJobResidual;
+            j.item = it;
+            j.path = path;
+            j.A = A;
+            j.r = rA;
+            j.c0 = seg * segc;
+            j.c1 = min(P.nch, j.c0 + segc);
+            j.mr = MassRes{rec.mx, rec.my, rec.izx, rec.izy, P.ts.c};
+            return true;
+        }
+        if (rdy) {
+            const int t = atomicAdd(P.grad_cnt + g, 1);
+            if (t < grad_items) {
+                const int seg = t % nseg;
+                j.kind = kJobGrad;
+                j.r = g * P.K * P.D + t / nseg;
+                j.c0 = seg * segc;
+                j.c1 = min(P.nch, j.c0 + segc);
+                return true;
+            }
+            atomicMax(P.grad_head, g + 1);
+            ++g;
+            continue;
+        }
+        if (tk < row_items) {
+            const int t = atomicAdd(P.ticket, 1);
+            if (t < row_items) {
+                const int seg = t % nseg;
+                j.kind = kJobRow;
+                j.item = t;
+                j.r = t / nseg;
+                j.c0 = seg * segc;
+                j.c1 = min(P.nch, j.c0 + segc);
+                return true;
+            }
+        }
+        if (g >= B) return true;  // every gradient segment has been claimed: end
+        if (*(volatile int*)P.status & VSD_STATUS_TIMEOUT) return true;
+        if (!wait) return false;
+        if (h < tl) continue;  // residual work is pending: try again at once
+        const uint64_t now = global_timer_ns();
+        if (idle_since == 0) {
+            idle_since = now;
+        } else if (now - idle_since > P.timeout_ns) {
+            atomicOr(P.status, VSD_STATUS_TIMEOUT);
+            return true;
+        }
+        __nanosleep(1000);
+    }
+}
+
+// Last-finisher counter (control warp): lane 0 adds one to *cnt after a fence
+// and every lane learns whether it completed the count n.
+__device__ __forceinline__ bool warp_count_last(int* cnt, int n, int lane) {
+    int last = 0;
+    if (lane == 0) {
+        __threadfence();
+        last = atomicAdd(cnt, 1) == n - 1;
+        if (last) __threadfence();
+    }
+    return __shfl_sync(0xffffffffu, last, 0) != 0;
+}
+
+// Shared memory of the control warp.
+union CtlShared {
+    WeightsShared w;
+    RescanBuf rb;
+};
+
+// End of a path (control warp): epilogue, then the prefix counter; the warp
+// that completes the prefix's last path runs its M-step and publishes it.
+template <typename T>
+__device__ void finish_path_warp(const Problem<T>& P, const EStepView& E, int path, int A,
+                                 int resid, bool have_rl, float rlq, float rla, CtlShared& cs,
+                                 int lane) {
+    path_epilogue_warp<T>(P, path, A, resid, lane, have_rl, rlq, rla);
+    __syncwarp();
+    const int prefix = path / P.K;
+    if (!warp_count_last(P.prefix_cnt + prefix, P.K, lane)) return;
+    weights_warp<T>(P, E, prefix, P.out.weights, P.out.loss, cs.w, lane);
+    __syncwarp();
+    if (lane == 0) {
+        __threadfence();
+        if (!P.inject_wait_fault) st_release(P.ready + prefix, 1);
+        if (atomicAdd(P.prefix_done, 1) == P.B - 1) {
+            __threadfence();
+            loss_mean(P.out.loss, P.B);
         }
     }
 }
 
-// Persistent E-step + M-step over row segments (segc chunks of a row).  Each
-// block repeatedly takes, in this order of priority:
-//   1. a residual segment from the queue (residual draws gate a prefix's M-step),
-//   2. a gradient segment of the oldest prefix whose M-step is published,
-//   3. the next logit-row segment (rows in prefix order).
-// A row segment streams its chunks of the draft and target rows into the
-// row's table in global memory; the block completing a row's last segment
-// runs the row tail; the block completing a path's last row finds its
-// accepted length and queues the residual row's segments (or, if every token
-// was accepted, ends the path); the block completing a path's last residual
-// segment draws the residual token and ends the path; the block ending a
-// prefix's last path runs the M-step and publishes it.  Claimed work never
-// waits; a block with nothing to claim polls (bounded by the wait timeout),
+// What the control warp does after the streaming warps finished job j.
+template <typename T, bool VEC>
+__device__ void post_job(const Problem<T>& P, const EStepView& E, const Job& j, float4* tab,
+                         CtlShared& cs, int lane) {
+    const int D = P.D, nseg = P.nseg, nch = P.nch;
+    if (j.kind == kJobRow) {
+        const int r = j.r;
+        if (!warp_count_last(P.row_seg_cnt + r, nseg, lane)) return;
+        row_tail_warp<T, VEC>(P, r, tab, cs.rb, lane);
+        __syncwarp();
+        const int path = r / D;
+        if (!warp_count_last(P.path_cnt + path, D, lane)) return;
+        const int A = path_accept_len<T>(P, path, lane);
+        const int flags = A < D ? ld_cg(P.rows + path * D + A).flags : 0;
+        if (A < D && !flags) {
+            if (lane == 0) {  // queue the residual row's segments
+                P.path_A[path] = A;
+                const int base = atomicAdd(P.resq_tail, nseg);
+                for (int sg = 0; sg < nseg; ++sg) P.resq[base + sg] = path * nseg + sg;
+                __threadfence();
+                for (int sg = 0; sg < nseg; ++sg) st_release(P.resq_flag + base + sg, 1);
+            }
+        } else {
+            finish_path_warp<T>(P, E, path, A, -1, false, 0.f, 0.f, cs, lane);
+        }
+    } else if (j.kind == kJobResidual) {
+        if (!warp_count_last(P.res_seg_cnt + j.path, nseg, lane)) return;
+        const int rA = j.r;
+        const int64_t V = P.V;
+        const T* x = P.draft + (int64_t)rA * V;
+        const T* y = P.target + (int64_t)rA * V;
+        const float c = P.ts.c;
+        // one round trip: row A's residual table, record and uniform
+        const float u = __ldg(P.u_correct + rA);
+        const RowRec rec = ld_cg(P.rows + rA);
+        const float4* rtab = P.gtab + (int64_t)rA * P.nch_ws;
+        for (int ch = lane; ch < nch; ch += 32) tab[ch] = ld_cg(rtab + ch);
+        __syncwarp();
+        const TableSum Rt = table_sum(tab, nch, 0, 0.f, c, lane);
+        int tok = -1;
+        Located loc{-1, 0.f};
+        if (Rt.Z > 0.0) loc = table_locate(tab, nch, 0, 0.f, c, Rt, u, lane);
+        uint4 bx[kLoads], by[kLoads];
+        if (loc.ch >= 0) {
+            if (VEC) {  // one round trip for both rows' chunks
+                chunk_async<T>(cs.rb.c[0], x, V, loc.ch, lane);
+                chunk_async<T>(cs.rb.c[1], y, V, loc.ch, lane);
+                cp_async_wait_all();
+                __syncwarp();
+                chunk_from_smem<T>(cs.rb.c[0], V, loc.ch, lane, bx);
+                chunk_from_smem<T>(cs.rb.c[1], V, loc.ch, lane, by);
+            } else {
+                load_chunk<T, VEC>(x, V, loc.ch, lane, policy_evict_normal(), bx);
+                load_chunk<T, VEC>(y, V, loc.ch, lane, policy_evict_normal(), by);
+            }
+            tok = rescan_regs<T, true, true>(bx, by, loc.ch, loc.tc, j.mr, lane);
+        }
+        if (tok >= V) tok = -1;
+        float rlq = 0.f, rla = 0.f;
+        if (tok >= 0) {
+            const float xv = VEC ? smem_elem(cs.rb.c[0], loc.ch, tok, x) : elem_value(x, tok);
+            const float yv = VEC ? smem_elem(cs.rb.c[1], loc.ch, tok, y) : elem_value(y, tok);
+            token_logs_vals(xv, yv, rec, P.ts.invTd, &rlq, &rla);
+        }
+        __syncwarp();
+        finish_path_warp<T>(P, E, j.path, j.A, tok, tok >= 0, rlq, rla, cs, lane);
+    }
+}
+
+// Persistent E-step + M-step over row segments (segc chunks of a row).  The
+// streaming warps run the jobs that the control warp hands them through
+// kSlots shared-memory slots:
+//   row segment: its chunks of the draft and target rows into the row's
+//     table in global memory;
+//   residual segment: its chunks of row A's residual mass into row A's table;
+//   gradient segment: its chunks of the draft row into the gradient row.
+// The control warp claims jobs ahead, and after each job does its counter:
+// the block completing a row's last segment runs the row tail; the block
+// completing a path's last row finds its accepted length and queues the
+// residual row's segments (or, if every token was accepted, ends the path);
+// the block completing a path's last residual segment draws the residual
+// token and ends the path; the block ending a prefix's last path runs the
+// M-step and publishes it.  So the streaming warps never wait for a claim or
+// a tail unless there is no work.  Claimed work never waits for other
+// blocks; a block with nothing to claim polls (bounded by the wait timeout),
 // so progress does not depend on residency.  Splitting rows lets a prefix be
 // published soon after its rows are read, so its gradient segments re-read
 // draft rows that are still in L2.
@@ -156,179 +350,78 @@ __device__ void finish_path(const Problem<T>& P, const EStepView& E, int path, i
 #define VSD_FUSED_MIN_BLOCKS 4
 #endif
 template <typename T, bool VEC, typename G>
-__global__ void __launch_bounds__(kThreads, VSD_FUSED_MIN_BLOCKS) k_fused(Problem<T> P, G* grad) {
+__global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
+    k_fused(Problem<T> P, G* grad) {
     extern __shared__ __align__(128) unsigned char dsm[];
-    __shared__ union {
-        RowShared row;
-        PathShared path;
-        WeightsShared w;
-    } sh;
-    __shared__ int s_kind, s_idx, s_flag;
+    __shared__ CtlShared cs;
+    __shared__ Job slots[kSlots];
     Ring* rg;
     float4* tab;
     smem_views<VEC>(dsm, rg, tab);
-    constexpr int CE = chunk_elems<T>();
-    const int Pp = P.K * P.D;
-    const int B = P.B, D = P.D, nseg = P.nseg, segc = P.segc, nch = P.nch;
-    const int row_items = P.R * nseg;
-    const int grad_items = Pp * nseg;  // per prefix
-    const int64_t V = P.V;
-    const float c = P.ts.c;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (warp < kWarps) {  // ------------------------------- streaming warps
+        for (int i = 0;; ++i) {
+            const int s = i % kSlots;
+            named_sync(bar_full(s));
+            const Job j = slots[s];
+            if (j.kind == kJobEnd) break;
+            const int64_t V = P.V;
+            const T* x = P.draft + (int64_t)j.r * V;
+            if (j.kind == kJobRow) {
+                // The draft row is read again for the gradient: ask L2 to keep it.
+                stream_tables<T, VEC, true>(rg, x, P.target + (int64_t)j.r * V, V, j.c0, j.c1,
+                                            P.gtab + (int64_t)j.r * P.nch_ws, P.ts.c,
+                                            policy_evict_last(), policy_evict_first(), P.status);
+            } else if (j.kind == kJobResidual) {
+                // row A's table was consumed by its row tail: reuse it
+                stream_residual<T, VEC>(rg, x, P.target + (int64_t)j.r * V, V, j.c0, j.c1,
+                                        P.gtab + (int64_t)j.r * P.nch_ws, j.mr, P.status);
+            } else {
+                stream_grad<T, VEC, G>(rg, P, j.r, j.c0, j.c1, grad);
+            }
+            __syncwarp();
+            named_arrive(bar_done(s));
+        }
+        return;
+    }
+    // ------------------------------------------------------------ control warp
     const EStepView E{P.es.tok, P.es.corr, P.es.lq_tok, P.es.lq_corr,
                       P.es.lk, P.es.lkc, P.es.lkr};
+    int g = *(volatile int*)P.grad_head;
+    int head = 0, tail = 0, inflight = 0;
+    bool ended = false;
     for (;;) {
-        if (threadIdx.x == 0) {
-            int kind = 0, idx = 0;  // 0 finished, 1 row, 2 gradient, 3 residual segment
-            uint64_t idle_since = 0;
-            int g = *(volatile int*)P.grad_head;
-            for (;;) {
-                // independent reads first (one round trip), then at most one
-                // attempt per kind of work
-                const int h = *(volatile int*)P.resq_head;
-                const int tl = *(volatile int*)P.resq_tail;
-                const int tk = *(volatile int*)P.ticket;
-                const int rdy = g < B ? ld_acquire(P.ready + g) : 0;
-                if (h < tl && atomicCAS(P.resq_head, h, h + 1) == h) {
-                    if (!wait_flag(P.resq_flag + h, P.status, P.timeout_ns)) {
-                        atomicOr(P.status, VSD_STATUS_TIMEOUT);
-                        break;
-                    }
-                    kind = 3;
-                    idx = ld_cg(P.resq + h);
-                    break;
-                }
-                if (rdy) {
-                    const int t = atomicAdd(P.grad_cnt + g, 1);
-                    if (t < grad_items) { kind = 2; idx = g * grad_items + t; break; }
-                    atomicMax(P.grad_head, g + 1);
-                    ++g;
-                    continue;
-                }
-                if (tk < row_items) {
-                    const int t = atomicAdd(P.ticket, 1);
-                    if (t < row_items) { kind = 1; idx = t; break; }
-                }
-                if (g >= B) break;  // every gradient segment has been claimed
-                if (*(volatile int*)P.status & VSD_STATUS_TIMEOUT) break;
-                if (h < tl) continue;  // residual work is pending: try again at once
-                const uint64_t now = global_timer_ns();
-                if (idle_since == 0) {
-                    idle_since = now;
-                } else if (now - idle_since > P.timeout_ns) {
-                    atomicOr(P.status, VSD_STATUS_TIMEOUT);
-                    break;
-                }
-                __nanosleep(1000);
+        while (!ended && inflight < kSlots) {
+            int got = 0;
+            if (lane == 0) got = claim_job<T>(P, inflight == 0, g, slots[tail % kSlots]) ? 1 : 0;
+            got = __shfl_sync(0xffffffffu, got, 0);
+            if (!got) break;
+            __syncwarp();
+            const int kind = slots[tail % kSlots].kind;
+            named_arrive(bar_full(tail % kSlots));
+            ++tail;
+            if (kind == kJobEnd) {
+                ended = true;
+                break;
             }
-            s_kind = kind;
-            s_idx = idx;
+            ++inflight;
         }
-        __syncthreads();
-        const int kind = s_kind, it = s_idx;
-        __syncthreads();
-        if (kind == 0) break;
-        if (kind == 1) {  // ------------------------------------- row segment
-            const int r = it / nseg, seg = it - r * nseg;
-            const int c0 = seg * segc, c1 = min(nch, c0 + segc);
-            const T* x = P.draft + (int64_t)r * V;
-            const T* y = P.target + (int64_t)r * V;
-            float4* rtab = P.gtab + (int64_t)r * P.nch_ws;
-            // The draft row is read again for the gradient: ask L2 to keep it.
-            stream_tables<T, VEC, true>(rg, x, y, V, c0, c1, rtab, c, policy_evict_last(),
-                                        policy_evict_first(), P.status);
-            __syncthreads();
-            if (threadIdx.x == 0) {
-                __threadfence();
-                s_flag = atomicAdd(P.row_seg_cnt + r, 1) == nseg - 1;
-                if (s_flag) __threadfence();
-            }
-            __syncthreads();
-            if (!s_flag) continue;
-            for (int ch = threadIdx.x; ch < nch; ch += kThreads) tab[ch] = ld_cg(rtab + ch);
-            __syncthreads();
-            row_tail<T, VEC, true, kSampleToken, true>(P, r, tab, sh.row);
-            __syncthreads();
-            const int path = r / D;
-            if (threadIdx.x == 0) {
-                __threadfence();
-                s_flag = atomicAdd(P.path_cnt + path, 1) == D - 1;
-                if (s_flag) __threadfence();
-            }
-            __syncthreads();
-            if (!s_flag) continue;
-            path_head<T>(P, path, sh.path);
-            __syncthreads();
-            const int A = sh.path.A;
-            if (A < D && !sh.path.rec.flags) {
-                if (threadIdx.x == 0) {  // queue the residual row's segments
-                    P.path_A[path] = A;
-                    const int base = atomicAdd(P.resq_tail, nseg);
-                    for (int sg = 0; sg < nseg; ++sg) P.resq[base + sg] = path * nseg + sg;
-                    __threadfence();
-                    for (int sg = 0; sg < nseg; ++sg) st_release(P.resq_flag + base + sg, 1);
-                }
-            } else {
-                finish_path<T>(P, E, path, A, -1, sh.w, &s_flag);
-            }
-        } else if (kind == 3) {  // ------------------------- residual segment
-            const int path = it / nseg, seg = it - path * nseg;
-            const int c0 = seg * segc, c1 = min(nch, c0 + segc);
-            if (threadIdx.x == 0) {
-                sh.path.A = ld_cg(P.path_A + path);
-                sh.path.rec = ld_cg(P.rows + path * D + sh.path.A);
-            }
-            __syncthreads();
-            const int A = sh.path.A;
-            const int rA = path * D + A;
-            const RowRec rec = sh.path.rec;
-            const T* x = P.draft + (int64_t)rA * V;
-            const T* y = P.target + (int64_t)rA * V;
-            float4* rtab = P.gtab + (int64_t)rA * P.nch_ws;  // row A's table is free again
-            const MassRes mr{rec.mx, rec.my, (float)exp(-rec.lzx), (float)exp(-rec.lzy), c};
-            stream_residual<T, VEC>(rg, x, y, V, c0, c1, rtab, mr, P.status);
-            __syncthreads();
-            if (threadIdx.x == 0) {
-                __threadfence();
-                s_flag = atomicAdd(P.res_seg_cnt + path, 1) == nseg - 1;
-                if (s_flag) __threadfence();
-            }
-            __syncthreads();
-            if (!s_flag) continue;
-            for (int ch = threadIdx.x; ch < nch; ch += kThreads) tab[ch] = ld_cg(rtab + ch);
-            __syncthreads();
-            const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-            if (warp == 0) {
-                const double Rt = table_total(tab, nch, 0, 0.f, c, lane);
-                int tok = -1;
-                if (Rt > 0.0) {
-                    const float u = __ldg(P.u_correct + rA);
-                    const Located loc = table_locate(tab, nch, 0, 0.f, c, (double)u * Rt, lane);
-                    if (loc.ch >= 0)
-                        tok = warp_rescan<T, VEC, true, true>(x, y, V, loc.ch, loc.tc, mr, lane,
-                                                              policy_evict_normal());
-                }
-                if (lane == 0) sh.path.resid = tok < V ? tok : -1;
-            }
-            __syncthreads();
-            finish_path<T>(P, E, path, A, sh.path.resid, sh.w, &s_flag);
-        } else {  // ------------------------------------------ gradient segment
-            const int b = it / grad_items, t = it - b * grad_items;
-            const int r = b * Pp + t / nseg, seg = t % nseg;
-            const int64_t e0 = (int64_t)seg * segc * CE;
-            const int64_t e1 = min(V, e0 + (int64_t)segc * CE);
-            grad_pass_range<T, VEC, G>(P, r, e0, e1, P.rstats, grad);
-        }
-        __syncthreads();
+        if (inflight == 0) break;
+        const int s = head % kSlots;
+        named_sync(bar_done(s));
+        if (slots[s].kind != kJobGrad) post_job<T, VEC>(P, E, slots[s], tab, cs, lane);
+        __syncwarp();
+        ++head;
+        --inflight;
     }
 }
 
 // ------------------------------------------------------------ launchers
+// Static plus dynamic shared memory above 48 KB needs the kernel's opt-in.
 template <typename K>
 static cudaError_t prep(K kernel, size_t smem) {
-    if (smem > 48 * 1024)
-        return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)smem);
-    return cudaSuccess;
+    if (smem == 0) return cudaSuccess;
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }
 
 template <>
@@ -423,7 +516,7 @@ cudaError_t Launch<VSD_T>::fused(const Problem<VSD_T>& P, bool vec, void* grad, 
     do {                                                                               \
         cudaError_t e = prep(k_fused<VSD_T, V_, G_>, smem);                            \
         if (e) return e;                                                               \
-        k_fused<VSD_T, V_, G_><<<ctas, kThreads, smem, s>>>(P, reinterpret_cast<G_*>(grad)); \
+        k_fused<VSD_T, V_, G_><<<ctas, kFusedThreads, smem, s>>>(P, reinterpret_cast<G_*>(grad)); \
     } while (0)
     if (vec && grad_bf16) VSD_FUSED(true, __nv_bfloat16);
     else if (vec) VSD_FUSED(true, float);
@@ -444,13 +537,13 @@ int Launch<VSD_T>::fused_blocks_per_sm(const Problem<VSD_T>& P, bool vec, bool g
     int n = 0;
     cudaError_t e;
     if (vec && grad_bf16)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, true, __nv_bfloat16>, kThreads, smem);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, true, __nv_bfloat16>, kFusedThreads, smem);
     else if (vec)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, true, float>, kThreads, smem);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, true, float>, kFusedThreads, smem);
     else if (grad_bf16)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, false, __nv_bfloat16>, kThreads, smem);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, false, __nv_bfloat16>, kFusedThreads, smem);
     else
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, false, float>, kThreads, smem);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, false, float>, kFusedThreads, smem);
     if (e != cudaSuccess || n < 1) return 1;
     return n;
 }

@@ -32,6 +32,7 @@ namespace vsd {
 struct __align__(16) RowRec {  // one logit row after row_pass (workspace)
     double lzx, lzy;         // ln sum_v exp((v - max)/T) of the q and p rows
     float mx, my;            // row maxima (exact input values)
+    float izx, izy;          // 1 / sum_v exp((v - max)/T) in float (0 if the row is invalid)
     int tok;                 // z~ (drawn from q, or given); -1 if none
     float lq_tok, la_tok;    // log q(z~), log alpha(z~) = min(0, log p - log q)
     int ps;                  // draw from p with u_correct
@@ -39,8 +40,9 @@ struct __align__(16) RowRec {  // one logit row after row_pass (workspace)
     int ref;                 // argmax of the target row
     float la_ref;
     int flags;               // 1: invalid row, 2: invalid given token
+    int pad[3];
 };
-static_assert(sizeof(RowRec) == 64, "RowRec layout");
+static_assert(sizeof(RowRec) == 80, "RowRec layout");
 
 struct __align__(16) Coef {     // grad[v] = g q(v) - c0 [v == t0] - c1 [v == t1]
     float g;
@@ -103,6 +105,8 @@ struct Problem {
     const int32_t* given_tokens;  // [R] or null (draft sampling)
     const int32_t* parent;        // tree [B][N]
     double w_base, tau_car;
+    double wl[64];  // w(l) = w_base^l for l = 1 .. D (App. F), computed on the host
+    double inv_tau;  // 1 / tau_car
     int zeta_mode;
     int grad_bf16;
     int inject_wait_fault;
@@ -173,20 +177,30 @@ __device__ __forceinline__ float2 chunk_stats(const uint4 (&buf)[kLoads], float 
 // to kStages chunks ahead; all lanes wait on the slot's mbarrier, read their
 // own vectors, and the slot is refilled once the warp has read it.  Each warp
 // produces and consumes its own slots, so no block-wide synchronisation is
-// involved.  pos[w] counts the chunks warp w has consumed (slot = pos %
-// kStages, barrier phase = (pos / kStages) & 1) and persists across rows.
+// involved.  A stream of one row only (no target) uses the same memory as
+// 2 kStages single-chunk slots, so it keeps as many bytes in flight.  Each
+// layout has its own barriers and its own count of consumed chunks (pos2 for
+// two rows, pos1 for one; slot = pos % stages, phase = (pos / stages) & 1),
+// which persist across calls; a call consumes every chunk it issues, so the
+// two layouts never hold a buffer at the same time.
 struct Ring {
     uint4 data[kWarps][kStages][2][kLoads * 32];
-    uint64_t bar[kWarps][kStages];
-    int pos[kWarps];
+    uint64_t bar2[kWarps][kStages];
+    uint64_t bar1[kWarps][2 * kStages];
+    int pos2[kWarps];
+    int pos1[kWarps];
     int broken[kWarps];  // a wait ran out: no further waits or copies in this block
 };
 
+// Every thread of the block calls it; warps beyond the streaming warps (the
+// fused kernel's control warp) own no ring slots.
 __device__ __forceinline__ void ring_init(Ring* rg) {
-    if ((threadIdx.x & 31) == 0) {
+    if ((threadIdx.x & 31) == 0 && (threadIdx.x >> 5) < kWarps) {
         const int w = threadIdx.x >> 5;
-        for (int st = 0; st < kStages; ++st) mbar_init(&rg->bar[w][st], 1);
-        rg->pos[w] = 0;
+        for (int st = 0; st < kStages; ++st) mbar_init(&rg->bar2[w][st], 1);
+        for (int st = 0; st < 2 * kStages; ++st) mbar_init(&rg->bar1[w][st], 1);
+        rg->pos2[w] = 0;
+        rg->pos1[w] = 0;
         rg->broken[w] = 0;
         mbar_init_fence();
     }
@@ -216,37 +230,46 @@ __device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, in
                                             Consume&& consume) {
     constexpr int PV = Traits<T>::kPerVec;
     constexpr int CE = chunk_elems<T>();
+    constexpr int NS = HAS_Y ? kStages : 2 * kStages;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint64_t* bars = HAS_Y ? rg->bar2[warp] : rg->bar1[warp];
+    int* posp = HAS_Y ? &rg->pos2[warp] : &rg->pos1[warp];
+    // slot q: the x and y halves of stage q (two rows), or half q & 1 of
+    // stage q >> 1 (one row)
+    auto xbuf = [&](int q) -> uint4* {
+        return HAS_Y ? rg->data[warp][q][0] : rg->data[warp][q >> 1][q & 1];
+    };
     const int nrange = ch1 - ch0;
     const int nj = nrange > warp ? (nrange - warp + kWarps - 1) / kWarps : 0;
-    const int pos = rg->pos[warp];
+    const int pos = *posp;
     bool broken = rg->broken[warp] != 0;
     auto issue = [&](int j) {
         const int ch = ch0 + warp + j * kWarps;
-        const int slot = (pos + j) % kStages;
+        const int slot = (pos + j) % NS;
         const int64_t e0 = (int64_t)ch * CE;
         const int64_t ne = V - e0 < CE ? V - e0 : CE;
         const uint32_t bytes = (uint32_t)(ne * (int64_t)sizeof(T));
-        uint64_t* bar = &rg->bar[warp][slot];
+        uint64_t* bar = &bars[slot];
         fence_proxy_async();
         mbar_expect_tx(bar, HAS_Y ? 2 * bytes : bytes);
-        bulk_g2s(rg->data[warp][slot][0], x + e0, bytes, bar, polx);
+        bulk_g2s(xbuf(slot), x + e0, bytes, bar, polx);
         if (HAS_Y) bulk_g2s(rg->data[warp][slot][1], y + e0, bytes, bar, poly);
     };
     if (lane == 0)
-        for (int j = 0; j < nj && j < kStages; ++j) issue(j);
+        for (int j = 0; j < nj && j < NS; ++j) issue(j);
     for (int j = 0; j < nj; ++j) {
-        const int slot = (pos + j) % kStages;
-        const uint32_t parity = (uint32_t)((pos + j) / kStages) & 1u;
-        bool ok = broken ? false : ring_wait(&rg->bar[warp][slot], parity, status);
+        const int slot = (pos + j) % NS;
+        const uint32_t parity = (uint32_t)((pos + j) / NS) & 1u;
+        bool ok = broken ? false : ring_wait(&bars[slot], parity, status);
         broken = __any_sync(0xffffffffu, !ok);
         const int ch = ch0 + warp + j * kWarps;
         const int64_t e0 = (int64_t)ch * CE;
+        const uint4* sx = xbuf(slot);
         uint4 bx[kLoads], by[kLoads];
         if (e0 + CE <= V) {  // full chunk (all but possibly the row's last)
 #pragma unroll
             for (int k = 0; k < kLoads; ++k) {
-                bx[k] = rg->data[warp][slot][0][k * 32 + lane];
+                bx[k] = sx[k * 32 + lane];
                 if (HAS_Y) by[k] = rg->data[warp][slot][1][k * 32 + lane];
             }
         } else {
@@ -255,17 +278,17 @@ __device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, in
                 const bool in = e0 + (int64_t)k * 32 * PV + lane * PV < V;
                 const uint4 ninf = make_uint4(Traits<T>::kNegInf, Traits<T>::kNegInf,
                                               Traits<T>::kNegInf, Traits<T>::kNegInf);
-                bx[k] = in ? rg->data[warp][slot][0][k * 32 + lane] : ninf;
+                bx[k] = in ? sx[k * 32 + lane] : ninf;
                 if (HAS_Y) by[k] = in ? rg->data[warp][slot][1][k * 32 + lane] : ninf;
             }
         }
         __syncwarp();
-        if (lane == 0 && !broken && j + kStages < nj) issue(j + kStages);
+        if (lane == 0 && !broken && j + NS < nj) issue(j + NS);
         consume(ch, bx, by);
     }
     __syncwarp();
     if (lane == 0) {
-        rg->pos[warp] = pos + nj;
+        *posp = pos + nj;
         rg->broken[warp] = broken ? 1 : 0;
     }
     __syncwarp();
@@ -327,50 +350,134 @@ __device__ __forceinline__ float table_max(const float4* tab, int nch, int comp,
     return warp_max(M);
 }
 
-// Weight of chunk ch in the row frame Mm: s_c 2^{(m_c - Mm) c}.
-__device__ __forceinline__ double chunk_weight(const float4* tab, int ch, int comp, float Mm,
-                                               float c, float* scale_out) {
-    const float2 ms = tab_ms(tab[ch], comp);
-    const float sc = ex2((frame_of(ms.x) - Mm) * c);
-    if (scale_out) *scale_out = sc;
-    return (double)ms.y * (double)sc;
+// --------------------------------------------------------------- table sums
+// The weight of chunk c in the row frame Mm is w_c = s_c 2^{(m_c - Mm) c}.
+// Tables are summed in exact 64-bit fixed point, w_c 2^E rounded down, with E
+// set from the largest weight so that it keeps at least 50 significant bits
+// and no sum of up to 2048 weights overflows.  Integer sums are exact and do
+// not depend on their order, so a total and the prefix sums that search it
+// agree, and none of it runs on the slow FP64 pipe.
+
+__device__ __forceinline__ float chunk_scale(const float4* tab, int ch, int comp, float Mm,
+                                             float c) {
+    return ex2((frame_of(tab_ms(tab[ch], comp).x) - Mm) * c);
 }
 
-// Sum of the chunk weights in a fixed order (groups of 32 chunks, warp scan).
-__device__ __forceinline__ double table_total(const float4* tab, int nch, int comp, float Mm,
-                                              float c, int lane) {
-    double base = 0.0;
-    for (int g = 0; g < nch; g += 32) {
-        const int ch = g + lane;
-        const double w = ch < nch ? chunk_weight(tab, ch, comp, Mm, c, nullptr) : 0.0;
-        const double inc = warp_incl_scan(w, lane);
-        base += __shfl_sync(0xffffffffu, inc, 31);
+// floor(s sc 2^E) for finite s, sc >= 0, by integer arithmetic on the two
+// 24-bit significands.
+__device__ __forceinline__ long long fixed_prod(float s, float sc, int E) {
+    if (!(s > 0.f) || !(sc > 0.f)) return 0;
+    const unsigned bs = __float_as_uint(s), bc = __float_as_uint(sc);
+    const int xs = (bs >> 23) & 0xFF, xc = (bc >> 23) & 0xFF;
+    const unsigned long long ms = xs ? ((bs & 0x7FFFFFu) | 0x800000u) : (bs & 0x7FFFFFu);
+    const unsigned long long mc = xc ? ((bc & 0x7FFFFFu) | 0x800000u) : (bc & 0x7FFFFFu);
+    const int sh = (xs ? xs : 1) + (xc ? xc : 1) - 300 + E;  // s sc 2^E = ms mc 2^sh
+    const unsigned long long pm = ms * mc;                   // < 2^48
+    if (sh >= 0) return (long long)(pm << min(sh, 15));
+    return sh > -64 ? (long long)(pm >> -sh) : 0;
+}
+
+// floor(u Zi) for Zi >= 0 (exact, 128-bit product); u >= 1 or NaN gives Zi
+// (no chunk is crossed), u <= 0 gives 0.
+__device__ __forceinline__ long long fixed_scale(long long Zi, float u) {
+    if (!(u < 1.f)) return Zi;
+    if (!(u > 0.f)) return 0;
+    const unsigned bu = __float_as_uint(u);
+    const int xu = (bu >> 23) & 0xFF;
+    const unsigned long long mu = xu ? ((bu & 0x7FFFFFu) | 0x800000u) : (bu & 0x7FFFFFu);
+    const int k = 150 - (xu ? xu : 1);  // u = mu 2^-k, k >= 24
+    const unsigned long long Z = (unsigned long long)Zi;
+    const unsigned long long lo = Z * mu, hi = __umul64hi(Z, mu);
+    if (k >= 128) return 0;
+    if (k >= 64) return (long long)(hi >> (k - 64));
+    return (long long)((hi << (64 - k)) | (lo >> k));
+}
+
+// 2^-E as a double (|E| <= 1000).
+__device__ __forceinline__ double pow2_neg(int E) {
+    return __longlong_as_double((long long)(1023 - E) << 52);
+}
+
+__device__ __forceinline__ long long warp_sum_ll(long long v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ long long warp_incl_scan_ll(long long v, int lane) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const long long n = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += n;
     }
-    return base;
+    return v;
 }
 
-// Find the chunk where the running weight first exceeds t (same order and
-// arithmetic as table_total).  Returns the chunk and the threshold in that
-// chunk's own frame; if no chunk crosses (rounding), the last chunk with
-// weight and an infinite threshold (the rescan then takes its last token
-// with mass).
-struct Located { int ch; double tc; };
+// A table total: Z = Zi 2^-E (NaN if a weight is not finite).
+struct TableSum {
+    long long Zi;
+    int E;
+    double Z;
+};
+
+// Sum of the chunk weights of one table component (warp).
+__device__ __forceinline__ TableSum table_sum(const float4* tab, int nch, int comp, float Mm,
+                                              float c, int lane) {
+    float wm = 0.f;
+    bool bad = false;
+    for (int ch = lane; ch < nch; ch += 32) {
+        const float w = tab_ms(tab[ch], comp).y * chunk_scale(tab, ch, comp, Mm, c);
+        bad |= !(w < INFINITY) && !(w == 0.f);
+        wm = fmaxf(wm, w);
+    }
+    bad = __any_sync(0xffffffffu, bad);
+    wm = warp_max(wm);
+    TableSum r{0, 0, 0.0};
+    if (bad) {
+        r.Z = __longlong_as_double(0x7FF8000000000000ll);  // NaN
+        return r;
+    }
+    if (!(wm > 0.f)) return r;
+    r.E = 50 - ilogbf(wm);
+    long long acc = 0;
+    for (int ch = lane; ch < nch; ch += 32)
+        acc += fixed_prod(tab_ms(tab[ch], comp).y, chunk_scale(tab, ch, comp, Mm, c), r.E);
+    r.Zi = warp_sum_ll(acc);
+    r.Z = (double)r.Zi * pow2_neg(r.E);
+    return r;
+}
+
+// Find the chunk where the running weight first exceeds ti = floor(u Zi).
+// Returns the chunk and the threshold in that chunk's own frame, rounded down
+// to a float (a float running mass exceeds the exact threshold if and only if
+// it exceeds this float); if no chunk crosses, the last chunk with weight and
+// an infinite threshold (the rescan then takes its last token with mass).
+struct Located {
+    int ch;
+    float tc;
+};
 __device__ __forceinline__ Located table_locate(const float4* tab, int nch, int comp, float Mm,
-                                                float c, double t, int lane) {
-    double base = 0.0;
+                                                float c, const TableSum& S, float u, int lane) {
+    const long long ti = fixed_scale(S.Zi, u);
+    long long base = 0;
     int last = -1;
     for (int g = 0; g < nch; g += 32) {
         const int ch = g + lane;
         float sc = 1.f;
-        const double w = ch < nch ? chunk_weight(tab, ch, comp, Mm, c, &sc) : 0.0;
-        const double inc = warp_incl_scan(w, lane);
-        const unsigned hit = __ballot_sync(0xffffffffu, ch < nch && base + inc > t);
-        const unsigned pos = __ballot_sync(0xffffffffu, ch < nch && w > 0.0);
+        long long w = 0;
+        if (ch < nch) {
+            sc = chunk_scale(tab, ch, comp, Mm, c);
+            w = fixed_prod(tab_ms(tab[ch], comp).y, sc, S.E);
+        }
+        const long long inc = warp_incl_scan_ll(w, lane);
+        const unsigned hit = __ballot_sync(0xffffffffu, ch < nch && base + inc > ti);
+        const unsigned pos = __ballot_sync(0xffffffffu, ch < nch && w > 0);
         if (hit) {
             const int L = __ffs(hit) - 1;
-            const double before = __shfl_sync(0xffffffffu, base + inc - w, L);
+            const long long before = __shfl_sync(0xffffffffu, base + inc - w, L);
             const float scL = __shfl_sync(0xffffffffu, sc, L);
-            return Located{g + L, (t - before) / (double)scL};
+            // ti - before < w_L < 2^52: exact in double, as is the scaling
+            const double rem = (double)(ti - before) * pow2_neg(S.E);
+            return Located{g + L, __double2float_rd(__ddiv_rd(rem, (double)scL))};
         }
         if (pos) last = g + 31 - __clz(pos);
         base += __shfl_sync(0xffffffffu, inc, 31);
@@ -378,18 +485,16 @@ __device__ __forceinline__ Located table_locate(const float4* tab, int nch, int 
     return Located{last, INFINITY};
 }
 
-// Scan chunk ch in token order and return the first token of positive mass
-// whose running mass exceeds tc (the chunk-frame threshold); if none does,
-// the last token with mass; -1 if the chunk has no mass.  Only tokens of
-// positive mass can be returned, so masked positions (at or beyond V) never
-// are.  mass(fx, fy) gives a token's mass.
-template <typename T, bool VEC, bool NEED_X, bool NEED_Y, class Mass>
-__device__ __forceinline__ int warp_rescan(const T* x, const T* y, int64_t V, int ch, double tc,
-                                           const Mass& mass, int lane, uint64_t pol) {
+// Scan chunk ch (in registers: bx, by as load_chunk gives them) in token order
+// and return the first token of positive mass whose running mass exceeds tc
+// (the chunk-frame threshold); if none does, the last token with mass; -1 if
+// the chunk has no mass.  Only tokens of positive mass can be returned, so
+// masked positions (at or beyond V) never are.  mass(fx, fy) gives a token's
+// mass.
+template <typename T, bool NEED_X, bool NEED_Y, class Mass>
+__device__ __forceinline__ int rescan_regs(const uint4 (&bx)[kLoads], const uint4 (&by)[kLoads],
+                                           int ch, float tc, const Mass& mass, int lane) {
     constexpr int PV = Traits<T>::kPerVec;
-    uint4 bx[kLoads], by[kLoads];
-    if (NEED_X) load_chunk<T, VEC>(x, V, ch, lane, pol, bx);
-    if (NEED_Y) load_chunk<T, VEC>(y, V, ch, lane, pol, by);
     float carry = 0.f;
     int last = -1;
     const int64_t base = (int64_t)ch * chunk_elems<T>();
@@ -415,7 +520,7 @@ __device__ __forceinline__ int warp_rescan(const T* x, const T* y, int64_t V, in
 #pragma unroll
         for (int e = 0; e < PV; ++e) {
             acc += m[e];
-            if (epos < 0 && m[e] > 0.f && (double)acc > tc) epos = e;
+            if (epos < 0 && m[e] > 0.f && acc > tc) epos = e;
         }
         const unsigned hit = __ballot_sync(0xffffffffu, epos >= 0);
         if (hit) {
@@ -432,6 +537,16 @@ __device__ __forceinline__ int warp_rescan(const T* x, const T* y, int64_t V, in
         carry += tot;
     }
     return last;
+}
+
+// rescan_regs on chunk ch loaded from global memory.
+template <typename T, bool VEC, bool NEED_X, bool NEED_Y, class Mass>
+__device__ __forceinline__ int warp_rescan(const T* x, const T* y, int64_t V, int ch, float tc,
+                                           const Mass& mass, int lane, uint64_t pol) {
+    uint4 bx[kLoads], by[kLoads];
+    if (NEED_X) load_chunk<T, VEC>(x, V, ch, lane, pol, bx);
+    if (NEED_Y) load_chunk<T, VEC>(y, V, ch, lane, pol, by);
+    return rescan_regs<T, NEED_X, NEED_Y>(bx, by, ch, tc, mass, lane);
 }
 
 struct MassX {
@@ -453,14 +568,12 @@ struct MassRes {
 };
 
 // Inverse-CDF draw from the distribution of one table component (warp).
-// Z is the table total; returns the token (or -1 if the row has no mass).
+// S is the table total; returns the token (or -1 if the row has no mass).
 template <typename T, bool VEC>
 __device__ __forceinline__ int warp_sample(const T* x, const T* y, int64_t V, const float4* tab,
-                                           int nch, int comp, float M, double Z, float u,
+                                           int nch, int comp, float M, const TableSum& S, float u,
                                            float c, int lane, uint64_t pol) {
-    const float Mm = frame_of(M);
-    const double t = (double)u * Z;
-    const Located loc = table_locate(tab, nch, comp, Mm, c, t, lane);
+    const Located loc = table_locate(tab, nch, comp, frame_of(M), c, S, u, lane);
     if (loc.ch < 0) return -1;
     const float mm = frame_of(tab_ms(tab[loc.ch], comp).x);
     if (comp == 0)
@@ -468,20 +581,22 @@ __device__ __forceinline__ int warp_sample(const T* x, const T* y, int64_t V, co
     return warp_rescan<T, VEC, false, true>(x, y, V, loc.ch, loc.tc, MassY{mm, c}, lane, pol);
 }
 
-// Lowest index whose target logit equals the row max M (warp).
-template <typename T, bool VEC>
-__device__ __forceinline__ int warp_first_max(const T* y, int64_t V, const float4* tab, int nch,
-                                              float M, int lane, uint64_t pol) {
-    int ch = -1;
-    for (int g = 0; g < nch && ch < 0; g += 32) {
-        const int cc = g + lane;
+// First chunk whose target maximum equals the row max M (warp; -1 if none).
+__device__ __forceinline__ int table_first_max(const float4* tab, int nch, float M) {
+    for (int g = 0; g < nch; g += 32) {
+        const int cc = g + (threadIdx.x & 31);
         const unsigned hit = __ballot_sync(0xffffffffu, cc < nch && tab[cc].z == M);
-        if (hit) ch = g + __ffs(hit) - 1;
+        if (hit) return g + __ffs(hit) - 1;
     }
-    if (ch < 0) return -1;
+    return -1;
+}
+
+// Lowest index of chunk ch (target chunk in registers) whose logit equals M
+// (warp; -1 if none).
+template <typename T>
+__device__ __forceinline__ int first_max_regs(const uint4 (&by)[kLoads], int ch, float M) {
     constexpr int PV = Traits<T>::kPerVec;
-    uint4 by[kLoads];
-    load_chunk<T, VEC>(y, V, ch, lane, pol, by);
+    const int lane = threadIdx.x & 31;
     const int64_t base = (int64_t)ch * chunk_elems<T>();
 #pragma unroll
     for (int k = 0; k < kLoads; ++k) {
@@ -501,114 +616,134 @@ __device__ __forceinline__ int warp_first_max(const T* y, int64_t V, const float
     return -1;
 }
 
+// Lowest index whose target logit equals the row max M (warp).
+template <typename T, bool VEC>
+__device__ __forceinline__ int warp_first_max(const T* y, int64_t V, const float4* tab, int nch,
+                                              float M, int lane, uint64_t pol) {
+    const int ch = table_first_max(tab, nch, M);
+    if (ch < 0) return -1;
+    uint4 by[kLoads];
+    load_chunk<T, VEC>(y, V, ch, lane, pol, by);
+    return first_max_regs<T>(by, ch, M);
+}
+
 __device__ __forceinline__ bool row_ok(float M, double Z) {
     return M > -INFINITY && M < INFINITY && Z > 0.0 && Z < INFINITY;
 }
 
 // log q and log alpha = min(0, log p - log q) of token v (Eq. 1), in double.
-template <typename T>
-__device__ __forceinline__ void token_logs(const T* x, const T* y, int v, const RowRec& rec,
-                                           double invT, float* lq, float* la) {
-    const double lqd = ((double)elem_value(x, v) - (double)rec.mx) * invT - rec.lzx;
-    const double lpd = ((double)elem_value(y, v) - (double)rec.my) * invT - rec.lzy;
+// The same from the token's draft and target logits xv, yv.
+__device__ __forceinline__ void token_logs_vals(float xv, float yv, const RowRec& rec, double invT,
+                                                float* lq, float* la) {
+    const double lqd = ((double)xv - (double)rec.mx) * invT - rec.lzx;
+    const double lpd = ((double)yv - (double)rec.my) * invT - rec.lzy;
     const double d = lpd - lqd;
     *lq = (float)lqd;
     *la = (float)(d >= 0.0 ? 0.0 : d);
 }
+template <typename T>
+__device__ __forceinline__ void token_logs(const T* x, const T* y, int v, const RowRec& rec,
+                                           double invT, float* lq, float* la) {
+    token_logs_vals(elem_value(x, v), elem_value(y, v), rec, invT, lq, la);
+}
 
 // --------------------------------------------------------------- row pass
-struct RowShared {
-    float Mx, My;
-    double Zx, Zy, lzx, lzy;
-    int tok, ps, ref;
-    float lq[3], la[3];
-};
-
 enum XMode { kNoToken = 0, kSampleToken = 1, kGivenToken = 2 };
 
-// The per-row work once the row's chunk table tab[0..nch) is complete in
-// shared memory (block): row statistics, the draws, the argmax, the token
-// log-probabilities; writes rows[r] and rstats[r].
-template <typename T, bool VEC, bool HAS_Y, int XMODE, bool ARGMAX>
-__device__ void row_tail(const Problem<T>& P, int r, const float4* tab, RowShared& sh) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+// One of the row's three table-driven results (warp; every lane returns the
+// same values): which = 0 the draft statistics and z~ (drawn from q with
+// u_draft, or read from given_tokens), 1 the target statistics and the draw
+// from p with u_correct, 2 the lowest-index argmax of the target.
+struct RowTask {
+    float M;
+    TableSum S;
+    int tok;
+};
+template <typename T, bool VEC, int XMODE>
+__device__ __forceinline__ RowTask row_task(const Problem<T>& P, int r, const float4* tab,
+                                            int which, int lane) {
     const int64_t V = P.V;
     const T* x = P.draft + (int64_t)r * V;
-    const T* y = HAS_Y ? P.target + (int64_t)r * V : nullptr;
+    const T* y = P.target + (int64_t)r * V;
     const float c = P.ts.c;
     const uint64_t pol = policy_evict_normal();
-    if (warp == 0) {
-        const float M = table_max(tab, P.nch, 0, lane);
-        const double Z = table_total(tab, P.nch, 0, frame_of(M), c, lane);
-        int tok = -1;
-        if (XMODE == kSampleToken) {
-            if (row_ok(M, Z))
-                tok = warp_sample<T, VEC>(x, y, V, tab, P.nch, 0, M, Z, __ldg(P.u_draft + r), c,
-                                          lane, pol);
-        } else if (XMODE == kGivenToken) {
-            tok = __ldg(P.given_tokens + r);
-        }
-        if (XMODE == kSampleToken && (tok < 0 || tok >= V)) tok = -1;
-        if (lane == 0) {
-            sh.Mx = M;
-            sh.Zx = Z;
-            sh.lzx = row_ok(M, Z) ? log(Z) : 0.0;
-            sh.tok = tok;
-        }
-    } else if (HAS_Y && warp == 1) {
-        const float M = table_max(tab, P.nch, 1, lane);
-        const double Z = table_total(tab, P.nch, 1, frame_of(M), c, lane);
-        int ps = -1;
-        if (row_ok(M, Z))
-            ps = warp_sample<T, VEC>(x, y, V, tab, P.nch, 1, M, Z, __ldg(P.u_correct + r), c,
-                                     lane, pol);
-        if (ps >= V) ps = -1;
-        if (lane == 0) {
-            sh.My = M;
-            sh.Zy = Z;
-            sh.lzy = row_ok(M, Z) ? log(Z) : 0.0;
-            sh.ps = ps;
-        }
-    } else if (HAS_Y && ARGMAX && warp == 2) {
-        const float M = table_max(tab, P.nch, 1, lane);
-        const int ref =
-            (M > -INFINITY) ? warp_first_max<T, VEC>(y, V, tab, P.nch, M, lane, pol) : -1;
-        if (lane == 0) sh.ref = ref < V ? ref : -1;
+    RowTask t;
+    t.M = table_max(tab, P.nch, which == 0 ? 0 : 1, lane);
+    t.S = TableSum{0, 0, 0.0};
+    t.tok = -1;
+    if (which == 2) {
+        if (t.M > -INFINITY) t.tok = warp_first_max<T, VEC>(y, V, tab, P.nch, t.M, lane, pol);
+        if (t.tok >= V) t.tok = -1;
+        return t;
     }
-    __syncthreads();
-    // log q and log alpha of z~, of the p-draw and of the argmax: one lane each.
+    t.S = table_sum(tab, P.nch, which, frame_of(t.M), c, lane);
+    if (which == 0) {
+        if (XMODE == kSampleToken) {
+            if (row_ok(t.M, t.S.Z))
+                t.tok = warp_sample<T, VEC>(x, y, V, tab, P.nch, 0, t.M, t.S,
+                                            __ldg(P.u_draft + r), c, lane, pol);
+            if (t.tok >= V) t.tok = -1;
+        } else if (XMODE == kGivenToken) {
+            t.tok = __ldg(P.given_tokens + r);
+        }
+    } else {
+        if (row_ok(t.M, t.S.Z))
+            t.tok = warp_sample<T, VEC>(x, y, V, tab, P.nch, 1, t.M, t.S, __ldg(P.u_correct + r),
+                                        c, lane, pol);
+        if (t.tok >= V) t.tok = -1;
+    }
+    return t;
+}
+
+// The row record from the three tasks (warp): lanes 0..2 take the log q and
+// log alpha of z~, of the p-draw and of the argmax; lane 0 writes rows[r] and
+// rstats[r].
+// vals(which, v, xv, yv) gives the draft and target logits of token v (the
+// draw `which`).
+template <typename T, bool HAS_Y, int XMODE, bool ARGMAX, class Vals>
+__device__ __forceinline__ void row_finish(const Problem<T>& P, int r, const RowTask& tx,
+                                           const RowTask& ty, int ref, int lane, const Vals& vals) {
+    const int64_t V = P.V;
     const double invT = P.ts.invTd;
-    const bool okx = row_ok(sh.Mx, sh.Zx);
-    const bool oky = HAS_Y ? row_ok(sh.My, sh.Zy) : true;
+    const bool okx = row_ok(tx.M, tx.S.Z);
+    const bool oky = HAS_Y ? row_ok(ty.M, ty.S.Z) : true;
     const bool ok = okx && oky;
-    const int tok = XMODE == kNoToken ? -1 : sh.tok;
+    // the two logarithms at once, on lanes 0 and 1
+    const double lz = log(lane == 0 ? tx.S.Z : ty.S.Z);
+    const double lzx0 = __shfl_sync(0xffffffffu, lz, 0), lzy0 = __shfl_sync(0xffffffffu, lz, 1);
+    const double lzx = okx ? lzx0 : 0.0;
+    const double lzy = (HAS_Y && oky) ? lzy0 : 0.0;
+    const int tok = XMODE == kNoToken ? -1 : tx.tok;
     const bool tok_ok = tok >= 0 && tok < V;
-    if (threadIdx.x < 3) {
-        const int which = threadIdx.x;
-        const int v = which == 0 ? tok : (which == 1 ? sh.ps : sh.ref);
-        float lq = -INFINITY, la = -INFINITY;
-        const bool want = which == 0 || (HAS_Y && (which == 1 || ARGMAX));
+    float lq = -INFINITY, la = -INFINITY;
+    if (lane < 3) {
+        const int v = lane == 0 ? tok : (lane == 1 ? ty.tok : ref);
+        const bool want = lane == 0 || (HAS_Y && (lane == 1 || ARGMAX));
         if (want && ok && v >= 0 && v < V) {
             RowRec tmp;
-            tmp.mx = sh.Mx;
-            tmp.lzx = sh.lzx;
-            tmp.my = HAS_Y ? sh.My : 0.f;
-            tmp.lzy = HAS_Y ? sh.lzy : 0.0;
+            tmp.mx = tx.M;
+            tmp.lzx = lzx;
+            tmp.my = HAS_Y ? ty.M : 0.f;
+            tmp.lzy = lzy;
+            float xv, yv;
+            vals(lane, v, xv, yv);
             if (HAS_Y)
-                token_logs(x, y, v, tmp, invT, &lq, &la);
+                token_logs_vals(xv, yv, tmp, invT, &lq, &la);
             else
-                lq = (float)(((double)elem_value(x, v) - (double)tmp.mx) * invT - tmp.lzx);
+                lq = (float)(((double)xv - (double)tmp.mx) * invT - tmp.lzx);
         }
-        sh.lq[which] = lq;
-        sh.la[which] = la;
     }
-    __syncthreads();
-    if (threadIdx.x == 0) {
+    const float lq1 = __shfl_sync(0xffffffffu, lq, 1), la1 = __shfl_sync(0xffffffffu, la, 1);
+    const float la2 = __shfl_sync(0xffffffffu, la, 2);
+    if (lane == 0) {
         RowRec rec;
-        rec.mx = sh.Mx;
-        rec.lzx = okx ? sh.lzx : 0.0;
-        rec.my = HAS_Y ? sh.My : 0.f;
-        rec.lzy = (HAS_Y && oky) ? sh.lzy : 0.0;
+        rec.mx = tx.M;
+        rec.lzx = lzx;
+        rec.my = HAS_Y ? ty.M : 0.f;
+        rec.lzy = lzy;
+        rec.izx = okx ? 1.f / (float)tx.S.Z : 0.f;
+        rec.izy = (HAS_Y && oky) ? 1.f / (float)ty.S.Z : 0.f;
+        rec.pad[0] = rec.pad[1] = rec.pad[2] = 0;
         rec.flags = ok ? 0 : 1;
         if (!ok) atomicOr(P.status, VSD_STATUS_BAD_ROW);
         int t = tok;
@@ -618,16 +753,159 @@ __device__ void row_tail(const Problem<T>& P, int r, const float4* tab, RowShare
             rec.flags |= 2;
         }
         rec.tok = t;
-        rec.lq_tok = (ok && t >= 0) ? sh.lq[0] : -INFINITY;
-        rec.la_tok = (ok && t >= 0) ? sh.la[0] : -INFINITY;
-        rec.ps = (HAS_Y && ok) ? sh.ps : -1;
-        rec.lq_ps = (HAS_Y && ok) ? sh.lq[1] : -INFINITY;
-        rec.la_ps = (HAS_Y && ok) ? sh.la[1] : -INFINITY;
-        rec.ref = (HAS_Y && ARGMAX && ok) ? sh.ref : -1;
-        rec.la_ref = (HAS_Y && ARGMAX && ok) ? sh.la[2] : -INFINITY;
+        rec.lq_tok = (ok && t >= 0) ? lq : -INFINITY;
+        rec.la_tok = (ok && t >= 0) ? la : -INFINITY;
+        rec.ps = (HAS_Y && ok) ? ty.tok : -1;
+        rec.lq_ps = (HAS_Y && ok) ? lq1 : -INFINITY;
+        rec.la_ps = (HAS_Y && ok) ? la1 : -INFINITY;
+        rec.ref = (HAS_Y && ARGMAX && ok) ? ref : -1;
+        rec.la_ref = (HAS_Y && ARGMAX && ok) ? la2 : -INFINITY;
         P.rows[r] = rec;
         P.rstats[r] = make_float4(rec.mx, (float)rec.lzx, rec.my, (float)rec.lzy);
     }
+}
+
+struct RowShared {
+    RowTask t[3];
+};
+
+// The per-row work once the row's chunk table tab[0..nch) is complete in
+// shared memory (block): warps 0, 1 and 2 take the three tasks at once, warp
+// 0 then writes the record.
+template <typename T, bool VEC, bool HAS_Y, int XMODE, bool ARGMAX>
+__device__ void row_tail(const Problem<T>& P, int r, const float4* tab, RowShared& sh) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (warp == 0 || (HAS_Y && (warp == 1 || (ARGMAX && warp == 2)))) {
+        const RowTask t = row_task<T, VEC, XMODE>(P, r, tab, warp, lane);
+        if (lane == 0) sh.t[warp] = t;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        RowTask ty = sh.t[1];
+        if (!HAS_Y) ty = RowTask{0.f, TableSum{0, 0, 0.0}, -1};
+        const int ref = (HAS_Y && ARGMAX) ? sh.t[2].tok : -1;
+        const T* x = P.draft + (int64_t)r * P.V;
+        const T* y = HAS_Y ? P.target + (int64_t)r * P.V : nullptr;
+        row_finish<T, HAS_Y, XMODE, ARGMAX>(P, r, sh.t[0], ty, ref, lane,
+                                            [&](int, int v, float& xv, float& yv) {
+                                                xv = elem_value(x, v);
+                                                yv = HAS_Y ? elem_value(y, v) : 0.f;
+                                            });
+    }
+}
+
+// Chunk ch of a row into a shared-memory buffer with cp.async (warp; rows
+// 16-byte aligned).  Vectors at or beyond V are not read.
+template <typename T>
+__device__ __forceinline__ void chunk_async(uint4* buf, const T* row, int64_t V, int ch,
+                                            int lane) {
+    constexpr int PV = Traits<T>::kPerVec;
+    const int64_t base = (int64_t)ch * chunk_elems<T>() + lane * PV;
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k) {
+        const int64_t v0 = base + (int64_t)k * 32 * PV;
+        cp_async16(buf + k * 32 + lane, row + (v0 < V ? v0 : 0), v0 < V);
+    }
+}
+// The chunk in registers as load_chunk gives it (positions at or beyond V
+// read as -inf).
+template <typename T>
+__device__ __forceinline__ void chunk_from_smem(const uint4* buf, int64_t V, int ch, int lane,
+                                                uint4 (&b)[kLoads]) {
+    constexpr int PV = Traits<T>::kPerVec;
+    const int64_t base = (int64_t)ch * chunk_elems<T>() + lane * PV;
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k)
+        b[k] = base + (int64_t)k * 32 * PV < V
+                   ? buf[k * 32 + lane]
+                   : make_uint4(Traits<T>::kNegInf, Traits<T>::kNegInf, Traits<T>::kNegInf,
+                                Traits<T>::kNegInf);
+}
+// Logit v of a buffer holding chunk ch.
+__device__ __forceinline__ float smem_elem(const uint4* buf, int ch, int v, const float*) {
+    return reinterpret_cast<const float*>(buf)[v - ch * chunk_elems<float>()];
+}
+__device__ __forceinline__ float smem_elem(const uint4* buf, int ch, int v, const __nv_bfloat16*) {
+    return __bfloat162float(
+        reinterpret_cast<const __nv_bfloat16*>(buf)[v - ch * chunk_elems<__nv_bfloat16>()]);
+}
+
+// Shared memory of the fused kernel's control warp: the six chunks a row tail
+// rescans, or the M-step's scratch (never both at once).
+struct RescanBuf {
+    uint4 c[6][kLoads * 32];
+};
+
+// The row tail of row r by one warp (the fused kernel's control warp) with
+// its memory accesses batched, because each dependent round trip to memory
+// is slow while the streaming warps keep DRAM busy: one round trip for the
+// row's table (from global memory into tab) and its uniforms, then the three
+// draws' table work, then one round trip (cp.async) for the draft and target
+// chunks at the three chunks the draws rescan, which also hold the logits of
+// the tokens they return.  Same tokens and record as row_tail.
+template <typename T, bool VEC>
+__device__ void row_tail_warp(const Problem<T>& P, int r, float4* tab, RescanBuf& rb, int lane) {
+    const int64_t V = P.V;
+    const int nch = P.nch;
+    const T* x = P.draft + (int64_t)r * V;
+    const T* y = P.target + (int64_t)r * V;
+    const float c = P.ts.c;
+    const float ud = __ldg(P.u_draft + r), uc = __ldg(P.u_correct + r);
+    const float4* rtab = P.gtab + (int64_t)r * P.nch_ws;
+    for (int ch = lane; ch < nch; ch += 32) tab[ch] = ld_cg(rtab + ch);
+    __syncwarp();
+    RowTask tx{table_max(tab, nch, 0, lane), TableSum{0, 0, 0.0}, -1};
+    tx.S = table_sum(tab, nch, 0, frame_of(tx.M), c, lane);
+    RowTask ty{table_max(tab, nch, 1, lane), TableSum{0, 0, 0.0}, -1};
+    ty.S = table_sum(tab, nch, 1, frame_of(ty.M), c, lane);
+    Located lx{-1, 0.f}, ly{-1, 0.f};
+    if (row_ok(tx.M, tx.S.Z)) lx = table_locate(tab, nch, 0, frame_of(tx.M), c, tx.S, ud, lane);
+    if (row_ok(ty.M, ty.S.Z)) ly = table_locate(tab, nch, 1, frame_of(ty.M), c, ty.S, uc, lane);
+    const int ca = ty.M > -INFINITY ? table_first_max(tab, nch, ty.M) : -1;
+    const int chs[3] = {lx.ch, ly.ch, ca};
+    if (VEC) {
+#pragma unroll
+        for (int w = 0; w < 3; ++w)
+            if (chs[w] >= 0) {
+                chunk_async<T>(rb.c[2 * w], x, V, chs[w], lane);
+                chunk_async<T>(rb.c[2 * w + 1], y, V, chs[w], lane);
+            }
+        cp_async_wait_all();
+        __syncwarp();
+    }
+    const uint64_t pol = policy_evict_normal();
+    uint4 b[kLoads];
+    if (lx.ch >= 0) {
+        if (VEC) chunk_from_smem<T>(rb.c[0], V, lx.ch, lane, b);
+        else load_chunk<T, VEC>(x, V, lx.ch, lane, pol, b);
+        const float mm = frame_of(tab_ms(tab[lx.ch], 0).x);
+        tx.tok = rescan_regs<T, true, false>(b, b, lx.ch, lx.tc, MassX{mm, c}, lane);
+        if (tx.tok >= V) tx.tok = -1;
+    }
+    if (ly.ch >= 0) {
+        if (VEC) chunk_from_smem<T>(rb.c[3], V, ly.ch, lane, b);
+        else load_chunk<T, VEC>(y, V, ly.ch, lane, pol, b);
+        const float mm = frame_of(tab_ms(tab[ly.ch], 1).x);
+        ty.tok = rescan_regs<T, false, true>(b, b, ly.ch, ly.tc, MassY{mm, c}, lane);
+        if (ty.tok >= V) ty.tok = -1;
+    }
+    int ref = -1;
+    if (ca >= 0) {
+        if (VEC) chunk_from_smem<T>(rb.c[5], V, ca, lane, b);
+        else load_chunk<T, VEC>(y, V, ca, lane, pol, b);
+        ref = first_max_regs<T>(b, ca, ty.M);
+        if (ref >= V) ref = -1;
+    }
+    row_finish<T, true, kSampleToken, true>(P, r, tx, ty, ref, lane,
+                                            [&](int w, int v, float& xv, float& yv) {
+                                                if (VEC) {
+                                                    xv = smem_elem(rb.c[2 * w], chs[w], v, x);
+                                                    yv = smem_elem(rb.c[2 * w + 1], chs[w], v, y);
+                                                } else {
+                                                    xv = elem_value(x, v);
+                                                    yv = elem_value(y, v);
+                                                }
+                                            });
 }
 
 // Streams row r of the draft (and, with HAS_Y, of the target) once, then runs
@@ -719,14 +997,14 @@ __device__ int residual_draw(const Problem<T>& P, int r, const RowRec& rec, floa
     const T* x = P.draft + (int64_t)r * V;
     const T* y = P.target + (int64_t)r * V;
     const float c = P.ts.c;
-    const MassRes mr{rec.mx, rec.my, (float)exp(-rec.lzx), (float)exp(-rec.lzy), c};
+    const MassRes mr{rec.mx, rec.my, rec.izx, rec.izy, c};
     stream_residual<T, VEC>(rg, x, y, V, 0, P.nch, tab, mr, P.status);
     __syncthreads();
     if (warp == 0) {
-        const double Rt = table_total(tab, P.nch, 0, 0.f, c, lane);
+        const TableSum Rt = table_sum(tab, P.nch, 0, 0.f, c, lane);
         int tok = -1;
-        if (Rt > 0.0) {
-            const Located loc = table_locate(tab, P.nch, 0, 0.f, c, (double)u * Rt, lane);
+        if (Rt.Z > 0.0) {
+            const Located loc = table_locate(tab, P.nch, 0, 0.f, c, Rt, u, lane);
             if (loc.ch >= 0)
                 tok = warp_rescan<T, VEC, true, true>(x, y, V, loc.ch, loc.tc, mr, lane,
                                                       policy_evict_normal());
@@ -752,8 +1030,8 @@ __device__ int p_draw(const Problem<T>& P, int r, float u, Ring* rg, float4* tab
     __syncthreads();
     if (warp == 0) {
         const float M = table_max(tab, P.nch, 0, lane);
-        const double Z = table_total(tab, P.nch, 0, frame_of(M), c, lane);
-        const int tok = row_ok(M, Z) ? warp_sample<T, VEC>(y, nullptr, V, tab, P.nch, 0, M, Z, u,
+        const TableSum Z = table_sum(tab, P.nch, 0, frame_of(M), c, lane);
+        const int tok = row_ok(M, Z.Z) ? warp_sample<T, VEC>(y, nullptr, V, tab, P.nch, 0, M, Z, u,
                                                           c, lane, pol)
                                      : -1;
         if (lane == 0) *out = tok < V ? tok : -1;
@@ -772,43 +1050,52 @@ struct PathShared {
 };
 
 // Linear proposal path (b, s) = path: rows path*D .. path*D + D - 1.
-// path_head (warp 0): the accepted length A (first rejection by ballot) and,
-// if A < D, the record of row A.  Written to sh.A, sh.rec.
+// The accepted length A of the path (warp; first rejection by ballot).
 template <typename T>
-__device__ void path_head(const Problem<T>& P, int path, PathShared& sh) {
+__device__ __forceinline__ int path_accept_len(const Problem<T>& P, int path, int lane) {
     const int D = P.D;
     const int r0 = path * D;
+    int A = D;
+    for (int d0 = 0; d0 < D; d0 += 32) {
+        const int d = d0 + lane;
+        bool rej = false;
+        if (d < D) {
+            const RowRec rec = ld_cg(P.rows + r0 + d);
+            const float a = rec.flags ? 0.f : expf(rec.la_tok);
+            rej = rec.flags || !(__ldg(P.u_accept + r0 + d) <= a);
+        }
+        const unsigned bal = __ballot_sync(0xffffffffu, rej);
+        if (bal && A == D) A = d0 + __ffs(bal) - 1;
+    }
+    return A;
+}
+
+// path_head (warp 0): the accepted length A and, if A < D, the record of
+// row A.  Written to sh.A, sh.rec.
+template <typename T>
+__device__ void path_head(const Problem<T>& P, int path, PathShared& sh) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (warp == 0) {
-        int A = D;
-        for (int d0 = 0; d0 < D; d0 += 32) {
-            const int d = d0 + lane;
-            bool rej = false;
-            if (d < D) {
-                const RowRec rec = ld_cg(P.rows + r0 + d);
-                const double a = rec.flags ? 0.0 : exp((double)rec.la_tok);
-                rej = rec.flags || !((double)__ldg(P.u_accept + r0 + d) <= a);
-            }
-            const unsigned bal = __ballot_sync(0xffffffffu, rej);
-            if (bal && A == D) A = d0 + __ffs(bal) - 1;
-        }
+        const int A = path_accept_len<T>(P, path, lane);
         if (lane == 0) {
             sh.A = A;
-            if (A < D) sh.rec = ld_cg(P.rows + r0 + A);
+            if (A < P.D) sh.rec = ld_cg(P.rows + path * P.D + A);
         }
     }
 }
 
-// path_epilogue (warp 0): given A and the residual token at row A (-1: none
+// path_epilogue_warp (one warp): given A and the residual token at row A (-1: none
 // or no residual mass), the corrected path, alpha', the log-kappa prefix sums
 // of z~, z' and the reference (Eq. 2, warp scans), E[A] (Eq. 11); writes the
 // E-step view and the requested outputs.
+// have_rl: rlq, rla are the log q and log alpha of the residual token (else
+// they are read from the logits).
 template <typename T>
-__device__ void path_epilogue(const Problem<T>& P, int path, int A, int resid) {
+__device__ void path_epilogue_warp(const Problem<T>& P, int path, int A, int resid, int lane,
+                                   bool have_rl = false, float rlq = 0.f, float rla = 0.f) {
     const int D = P.D;
     const int r0 = path * D;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (warp == 0) {
+    {
         const int b = path / P.K;
         const double NEG = -INFINITY;
         const int64_t V = P.V;
@@ -820,19 +1107,22 @@ __device__ void path_epilogue(const Problem<T>& P, int path, int A, int resid) {
             const int r = r0 + (act ? d : 0);
             RowRec rec;
             if (act) rec = ld_cg(P.rows + r);
-            double a = 0.0, tk = 0.0, tkc = 0.0, tkr = 0.0;
+            float a = 0.f;
+            double tk = 0.0, tkc = 0.0, tkr = 0.0;
             bool acc = false;
             int zc = -1;
             float lqc = -INFINITY, lac = -INFINITY;
             if (act) {
-                a = rec.flags ? 0.0 : exp((double)rec.la_tok);
-                acc = !rec.flags && (double)__ldg(P.u_accept + r) <= a;
+                a = rec.flags ? 0.f : expf(rec.la_tok);  // alpha (Eq. 1)
+                acc = !rec.flags && __ldg(P.u_accept + r) <= a;
                 if (d < A) {
                     zc = rec.tok; lqc = rec.lq_tok; lac = rec.la_tok;
                 } else if (d == A) {
                     zc = resid >= 0 ? resid : rec.ps;  // no residual mass: draw from p (R10)
                     if (zc == rec.ps) {
                         lqc = rec.lq_ps; lac = rec.la_ps;
+                    } else if (have_rl) {
+                        lqc = rlq; lac = rla;
                     } else {
                         token_logs(P.draft + (int64_t)r * V, P.target + (int64_t)r * V, zc, rec,
                                    P.ts.invTd, &lqc, &lac);
@@ -850,7 +1140,7 @@ __device__ void path_epilogue(const Problem<T>& P, int path, int A, int resid) {
             const double lkc = ckc + warp_incl_scan(tkc, lane);
             double lkr = ckr + warp_incl_scan(tkr, lane);
             if (P.ref_logkappa && act) lkr = (double)__ldg(P.ref_logkappa + (int64_t)b * D + d);
-            EA += warp_sum(act ? exp(lk) : 0.0);  // Eq. 11
+            EA += warp_sum(act ? (double)expf((float)lk) : 0.0);  // Eq. 11
             const int lastl = min(31, D - 1 - d0);
             ck = __shfl_sync(0xffffffffu, lk, lastl);
             ckc = __shfl_sync(0xffffffffu, lkc, lastl);
@@ -865,11 +1155,11 @@ __device__ void path_epilogue(const Problem<T>& P, int path, int A, int resid) {
                 P.es.lkr[r] = (float)lkr;
                 if (o.tokens) o.tokens[r] = rec.tok;
                 if (o.logq_tok) o.logq_tok[r] = rec.lq_tok;
-                if (o.alpha) o.alpha[r] = (float)a;
+                if (o.alpha) o.alpha[r] = a;
                 if (o.accept) o.accept[r] = acc ? 1 : 0;
                 if (o.corr_tokens) o.corr_tokens[r] = zc;
                 if (o.logq_corr) o.logq_corr[r] = lqc;
-                if (o.alpha_corr) o.alpha_corr[r] = zc >= 0 ? (float)exp((double)lac) : 0.f;
+                if (o.alpha_corr) o.alpha_corr[r] = zc >= 0 ? expf(lac) : 0.f;
                 if (o.logkappa) o.logkappa[r] = (float)lk;
                 if (o.logkappa_corr) o.logkappa_corr[r] = (float)lkc;
                 if (o.logkappa_ref) o.logkappa_ref[r] = (float)lkr;
@@ -884,6 +1174,11 @@ __device__ void path_epilogue(const Problem<T>& P, int path, int A, int resid) {
             if (o.expected_len) o.expected_len[path] = (float)EA;
         }
     }
+}
+
+template <typename T>
+__device__ void path_epilogue(const Problem<T>& P, int path, int A, int resid) {
+    if ((threadIdx.x >> 5) == 0) path_epilogue_warp<T>(P, path, A, resid, threadIdx.x & 31);
 }
 
 
@@ -904,105 +1199,201 @@ __device__ void path_pass(const Problem<T>& P, int path, Ring* rg, float4* tab, 
 }
 
 // --------------------------------------------------------------- weights
+// The M-step reads its prefix's E-step view in tiles of (s, l) entries, all
+// proposals s and a run of positions l, so that each tile costs one round
+// trip to memory.  Within a tile the entries are processed in parallel
+// wherever the arithmetic allows, because double-precision latency, not
+// work, bounds a single warp here.
+constexpr int kMTile = 256;
 struct WeightsShared {
-    double ot[256], op[256], lqt[256], lqc[256], cq[256];
-    float ez[256];
-    double red[kThreads];
-    double w, cmax;
+    double lqt[256], lqc[256];  // per proposal: running sums of log q (z~, z') over l
+    // the tile: entry e = s * nd + (l - l0)
+    float lq[kMTile];    // log q(z~); then 2^{c_q - max} (CAR)
+    float lqcz[kMTile];  // log q(z')
+    unsigned char ot[kMTile], pc[kMTile];  // o~, and whether z' passes
+    int tok[kMTile], corr[kMTile];
+    double elqt[kMTile];  // running sum of log q(z~) at the entry
+    double elqc[kMTile];  // running sum of log q(z'); then the term o'(1 - o~)
+    double ecq[kMTile];   // CAR logit; then the term o'(o~ - beta zeta)
+    // per position of the tile
+    int n1[64], n0[64];  // proposals with o' != 0 and o~ = 1, with o' != 0
+    long long zs[64];    // sum of the CAR weights (fixed point, 2^-40)
+    float rz[64];        // 1 / that sum
+    float beta[64][3];   // leave-one-out beta for (o', o~) = (w, 1), (w, 0), (0, 0)
 };
 
-__device__ __forceinline__ double block_sum(double v, double* red) {
-    red[threadIdx.x] = v;
-    __syncthreads();
-    for (int o = kThreads / 2; o; o >>= 1) {
-        if (threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];
-        __syncthreads();
+// Load the tile of positions [d0, d0 + nd) of prefix b (warp).  TERMS: the
+// per-entry terms written by the forward sweep (from wscr) instead of the
+// scores.
+template <typename T, bool TERMS>
+__device__ __forceinline__ void mstep_tile(const Problem<T>& P, const EStepView& E, int b, int d0,
+                                           int nd, WeightsShared& sh, int lane) {
+    const int K = P.K, D = P.D;
+    for (int e = lane; e < K * nd; e += 32) {
+        const int s = e / nd, r = (b * K + s) * D + d0 + (e - s * nd);
+        sh.tok[e] = ld_cg(E.tok + r);
+        sh.corr[e] = ld_cg(E.corr + r);
+        if (TERMS) {
+            const double2 tm = ld_cg(P.wscr + r);
+            sh.ecq[e] = tm.x;
+            sh.elqc[e] = tm.y;
+        } else {
+            const float lkr = ld_cg(E.lkr + r);
+            sh.ot[e] = ld_cg(E.lk + r) >= lkr ? 1 : 0;
+            sh.pc[e] = ld_cg(E.lkc + r) >= lkr ? 1 : 0;
+            sh.lq[e] = ld_cg(E.lq_tok + r);
+            sh.lqcz[e] = ld_cg(E.lq_corr + r);
+        }
     }
-    const double r = red[0];
-    __syncthreads();
-    return r;
+    __syncwarp();
 }
 
-// M-step of prefix b (block; proposals s strided over the threads, K <= 256).
-// Writes coef[] for the prefix's rows, the optional weights table and
-// loss_out[b].  Arithmetic in double.
+// M-step of prefix b by one warp (K <= 256, D <= 64).  Writes coef[] for the
+// prefix's rows, the optional weights table and loss_out[b].  Arithmetic in
+// double except the CAR weights (float exponentials of double differences);
+// every sum over proposals is either an exact integer sum or taken in a fixed
+// order, so the result does not depend on timing.
+template <typename T>
+__device__ void weights_warp(const Problem<T>& P, const EStepView& E, int b, float* weights_out,
+                             float* loss_out, WeightsShared& sh, int lane) {
+    const int K = P.K, D = P.D;
+    const int dt = max(1, min(D, kMTile / K));
+    const bool one_tile = dt >= D;
+    for (int s = lane; s < K; s += 32) sh.lqt[s] = sh.lqc[s] = 0.0;
+    double Jp = 0.0, Np = 0.0;  // this lane's parts of J and N
+    for (int d0 = 0; d0 < D; d0 += dt) {
+        const int nd = min(dt, D - d0);
+        const int ne = K * nd;
+        mstep_tile<T, false>(P, E, b, d0, nd, sh, lane);
+        // running sums of log q over l, per proposal
+        for (int s = lane; s < K; s += 32) {
+            double a = sh.lqt[s], q = sh.lqc[s];
+            for (int dd = 0; dd < nd; ++dd) {
+                const int e = s * nd + dd;
+                a += (double)sh.lq[e];
+                q += (double)sh.lqcz[e];
+                sh.elqt[e] = a;
+                sh.elqc[e] = q;
+            }
+            sh.lqt[s] = a;
+            sh.lqc[s] = q;
+        }
+        __syncwarp();
+        // CAR logits (Eq. zeta): on q(z~_{1:l}) or on its log
+        for (int e = lane; e < ne; e += 32)
+            sh.ecq[e] = (P.zeta_mode == 0 ? exp(sh.elqt[e]) : sh.elqt[e]) * P.inv_tau;
+        __syncwarp();
+        // per position: the counts behind beta, and the CAR weights and their sum
+        for (int dd = 0; dd < nd; ++dd) {
+            int c1 = 0, c0 = 0;
+            float mf = -INFINITY;
+            for (int s = lane; s < K; s += 32) {
+                const int e = s * nd + dd;
+                // Algorithm 2 scores z~ (o~); Algorithm 1 keeps z~ if it
+                // passes, else z', so o' = w(l) when either passes
+                const bool ot = sh.ot[e], op = ot || sh.pc[e];
+                c1 += (op && ot) ? 1 : 0;
+                c0 += op ? 1 : 0;
+                mf = fmaxf(mf, (float)sh.ecq[e]);
+            }
+#pragma unroll
+            for (int o = 16; o; o >>= 1) {
+                c1 += __shfl_xor_sync(0xffffffffu, c1, o);
+                c0 += __shfl_xor_sync(0xffffffffu, c0, o);
+                mf = fmaxf(mf, __shfl_xor_sync(0xffffffffu, mf, o));
+            }
+            long long za = 0;  // the CAR weights are at most about 1: exact sum at 2^-40
+            for (int s = lane; s < K; s += 32) {
+                const int e = s * nd + dd;
+                const float ez = expf((float)(sh.ecq[e] - (double)mf));
+                sh.lq[e] = ez;
+                za += fixed_prod(ez, 1.f, 40);
+            }
+            za = warp_sum_ll(za);
+            if (lane == 0) {
+                sh.n1[dd] = c1;
+                sh.n0[dd] = c0;
+                sh.zs[dd] = za;
+            }
+        }
+        __syncwarp();
+        // per position, in parallel: 1 / sum, and beta (Eq. beta, leave-one-out:
+        // o' is w(l) or 0, so both of its sums are w(l) times a count)
+        for (int dd = lane; dd < nd; dd += 32) {
+            const int n1 = sh.n1[dd], n0 = sh.n0[dd];
+            const float zs = (float)sh.zs[dd] * 0x1p-40f;
+            sh.rz[dd] = zs > 0.f ? 1.f / zs : 0.f;
+            sh.beta[dd][0] = n0 - 1 > 0 ? (float)(n1 - 1) / (float)(n0 - 1) : 0.f;
+            sh.beta[dd][1] = n0 - 1 > 0 ? (float)n1 / (float)(n0 - 1) : 0.f;
+            sh.beta[dd][2] = n0 > 0 ? (float)n1 / (float)n0 : 0.f;
+            Np += P.wl[d0 + dd] * (double)n0;
+        }
+        __syncwarp();
+        // per entry, in parallel: zeta, the objective terms (Eq. advance) and
+        // the per-l gradient terms o'(o~ - beta zeta), o'(1 - o~)
+        for (int e = lane; e < ne; e += 32) {
+            const int s = e / nd, dd = e - s * nd, d = d0 + dd;
+            const bool otb = sh.ot[e], opb = otb || sh.pc[e];
+            const double w = P.wl[d];
+            const float betaf = sh.beta[dd][opb ? (otb ? 0 : 1) : 2];
+            const float zetaf = sh.lq[e] * sh.rz[dd];
+            const double beta = betaf, zeta = zetaf;
+            const double lqt = sh.elqt[e];
+            const double lqz = otb ? lqt : sh.elqc[e];
+            if (opb) Jp += w * (lqz - beta * zeta * lqt);
+            const double t0 = opb ? w * ((otb ? 1.0 : 0.0) - beta * zeta) : 0.0;
+            const double t1 = (opb && !otb) ? w : 0.0;
+            sh.ecq[e] = t0;
+            sh.elqc[e] = t1;
+            const int r = (b * K + s) * D + d;
+            if (!one_tile) P.wscr[r] = make_double2(t0, t1);
+            if (weights_out) {
+                float4* wo = reinterpret_cast<float4*>(weights_out) + ((int64_t)b * D + d) * K + s;
+                *wo = make_float4(otb ? 1.f : 0.f, opb ? (float)w : 0.f, betaf, zetaf);
+            }
+        }
+        __syncwarp();
+    }
+    const double J = warp_sum(Jp), N = warp_sum(Np);
+    const double scale = N > 0.0 ? 1.0 / ((double)P.B * N * P.ts.Td) : 0.0;
+    // suffix sums over l, from the last tile back (lqt, lqc now hold c0, c1)
+    for (int s = lane; s < K; s += 32) sh.lqt[s] = sh.lqc[s] = 0.0;
+    for (int d0 = ((D - 1) / dt) * dt; d0 >= 0; d0 -= dt) {
+        const int nd = min(dt, D - d0);
+        if (!one_tile) {
+            __syncwarp();
+            mstep_tile<T, true>(P, E, b, d0, nd, sh, lane);
+        }
+        for (int s = lane; s < K; s += 32) {
+            double c0 = sh.lqt[s], c1 = sh.lqc[s];
+            for (int dd = nd - 1; dd >= 0; --dd) {
+                const int e = s * nd + dd;
+                c0 += sh.ecq[e];
+                c1 += sh.elqc[e];
+                Coef cf;
+                cf.t0 = sh.tok[e];
+                cf.t1 = sh.corr[e];
+                double k0 = c0 * scale, k1 = c1 * scale;
+                if (cf.t1 == cf.t0) { k0 += k1; k1 = 0.0; cf.t1 = -1; }
+                cf.g = (float)((c0 + c1) * scale);
+                cf.c0 = (float)k0;
+                cf.c1 = (float)k1;
+                cf.pad0 = cf.pad1 = cf.pad2 = 0.f;
+                P.coef[(b * K + s) * D + d0 + dd] = cf;
+            }
+            sh.lqt[s] = c0;
+            sh.lqc[s] = c1;
+        }
+    }
+    if (lane == 0) loss_out[b] = (float)(N > 0.0 ? -J / N : 0.0);
+}
+
+// The M-step by a block: warp 0 runs weights_warp (the same bits as the fused
+// kernel's control warp).
 template <typename T>
 __device__ void weights_pass(const Problem<T>& P, const EStepView& E, int b, float* weights_out,
                              float* loss_out, WeightsShared& sh) {
-    const int K = P.K, D = P.D;
-    double Jp = 0.0, Np = 0.0;
-    for (int s = threadIdx.x; s < K; s += kThreads) sh.lqt[s] = sh.lqc[s] = 0.0;
-    for (int d = 0; d < D; ++d) {
-        if (threadIdx.x == 0) sh.w = pow(P.w_base, (double)(d + 1));  // w(l), App. F
-        __syncthreads();
-        const double w = sh.w;
-        for (int s = threadIdx.x; s < K; s += kThreads) {
-            const int r = (b * K + s) * D + d;
-            const double lk = ld_cg(E.lk + r), lkc = ld_cg(E.lkc + r), lkr = ld_cg(E.lkr + r);
-            sh.lqt[s] += (double)ld_cg(E.lq_tok + r);
-            sh.lqc[s] += (double)ld_cg(E.lq_corr + r);
-            // Algorithm 2 scores z~; Algorithm 1 keeps z~ if it passes, else z'.
-            const double ot = (lk >= lkr) ? 1.0 : 0.0;
-            sh.ot[s] = ot;
-            sh.op[s] = ot > 0.0 ? w : ((lkc >= lkr) ? w : 0.0);
-            sh.cq[s] = (P.zeta_mode == 0 ? exp(sh.lqt[s]) : sh.lqt[s]) / P.tau_car;
-        }
-        __syncthreads();
-        if (threadIdx.x < 32) {  // max of the CAR logits over the K proposals
-            double m = -INFINITY;
-            for (int j = threadIdx.x; j < K; j += 32) m = fmax(m, sh.cq[j]);
-#pragma unroll
-            for (int o = 16; o; o >>= 1) m = fmax(m, __shfl_xor_sync(0xffffffffu, m, o));
-            if (threadIdx.x == 0) sh.cmax = m;
-        }
-        __syncthreads();
-        for (int s = threadIdx.x; s < K; s += kThreads) sh.ez[s] = expf((float)(sh.cq[s] - sh.cmax));
-        __syncthreads();
-        for (int s = threadIdx.x; s < K; s += kThreads) {
-            double num = 0.0, den = 0.0, Zs = 0.0;
-            for (int j = 0; j < K; ++j) {
-                if (j != s) { num += sh.op[j] * sh.ot[j]; den += sh.op[j]; }
-                Zs += (double)sh.ez[j];
-            }
-            const double beta = den > 0.0 ? num / den : 0.0;  // Eq. beta (leave-one-out)
-            const double zeta = (double)sh.ez[s] / Zs;         // Eq. zeta
-            const double ot = sh.ot[s], op = sh.op[s];
-            const double lqz = ot > 0.0 ? sh.lqt[s] : sh.lqc[s];
-            if (op != 0.0) Jp += op * (lqz - beta * zeta * sh.lqt[s]);  // Eq. advance
-            Np += op;
-            // per-l terms o'(o~ - beta zeta) and o'(1 - o~) of row (s, l-1)
-            P.wscr[(b * K + s) * D + d] = make_double2(op * (ot - beta * zeta), op * (1.0 - ot));
-            if (weights_out) {
-                float4* wo = reinterpret_cast<float4*>(weights_out) + ((int64_t)b * D + d) * K + s;
-                *wo = make_float4((float)ot, (float)op, (float)beta, (float)zeta);
-            }
-        }
-        __syncthreads();
-    }
-    const double N = block_sum(Np, sh.red);
-    const double J = block_sum(Jp, sh.red);
-    const double scale = N > 0.0 ? 1.0 / ((double)P.B * N * P.ts.Td) : 0.0;
-    for (int s = threadIdx.x; s < K; s += kThreads) {
-        const int rbase = (b * K + s) * D;
-        double c0 = 0.0, c1 = 0.0;
-        for (int d = D - 1; d >= 0; --d) {
-            const int r = rbase + d;
-            const double2 tm = P.wscr[r];
-            c0 += tm.x;
-            c1 += tm.y;
-            Coef cf;
-            cf.t0 = ld_cg(E.tok + r);
-            cf.t1 = ld_cg(E.corr + r);
-            double k0 = c0 * scale, k1 = c1 * scale;
-            if (cf.t1 == cf.t0) { k0 += k1; k1 = 0.0; cf.t1 = -1; }
-            cf.g = (float)((c0 + c1) * scale);
-            cf.c0 = (float)k0;
-            cf.c1 = (float)k1;
-            cf.pad0 = cf.pad1 = cf.pad2 = 0.f;
-            P.coef[r] = cf;
-        }
-    }
-    if (threadIdx.x == 0) loss_out[b] = (float)(N > 0.0 ? -J / N : 0.0);
+    if ((threadIdx.x >> 5) == 0) weights_warp<T>(P, E, b, weights_out, loss_out, sh, threadIdx.x & 31);
 }
 
 // Mean of loss[0..B) into loss[B], summed in order (one thread).
@@ -1113,6 +1504,57 @@ __device__ void grad_pass_range(const Problem<T>& P, int r, int64_t e0, int64_t 
     }
 }
 
+// Gradient of chunks [c0, c1) of row r (warp level, through the ring; the
+// streaming warps of the fused kernel).  Same arithmetic as grad_pass_range.
+template <typename T, bool VEC, typename G>
+__device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1, G* grad) {
+    constexpr int PV = Traits<T>::kPerVec;
+    constexpr int CE = chunk_elems<T>();
+    const int64_t V = P.V;
+    if constexpr (!VEC) {
+        grad_pass_range<T, VEC, G>(P, r, (int64_t)c0 * CE, min(V, (int64_t)c1 * CE), P.rstats,
+                                   grad);
+    } else {
+        constexpr int NP = PV / 2;
+        const int lane = threadIdx.x & 31;
+        const T* x = P.draft + (int64_t)r * V;
+        G* g = grad + (int64_t)r * V;
+        const RowRec rec = ld_cg(P.rows + r);
+        const Coef cf = ld_cg(P.coef + r);
+        const float c = P.ts.c;
+        const float gq = cf.g * rec.izx;  // g / Z
+        const uint64_t pol = policy_evict_first();
+        const uint64_t mx2 = f2(rec.mx, rec.mx), c2 = f2(c, c), gq2 = f2(gq, gq);
+        ring_stream<T, false>(
+            rg, x, nullptr, V, c0, c1, pol, pol, P.status,
+            [&](int ch, const uint4 (&bx)[kLoads], const uint4 (&)[kLoads]) {
+#pragma unroll
+                for (int k = 0; k < kLoads; ++k) {
+                    const int64_t v0 = (int64_t)ch * CE + (int64_t)k * 32 * PV + lane * PV;
+                    if (v0 >= V) break;
+                    uint64_t pr[NP];
+                    vec_pairs<T>(bx[k], pr);
+                    float o[PV];
+#pragma unroll
+                    for (int q = 0; q < NP; ++q)
+                        f2split(f2mul(f2_mass(pr[q], mx2, c2), gq2), o[2 * q], o[2 * q + 1]);
+                    // the sparse terms touch at most two positions of the row
+                    if ((uint64_t)(cf.t0 - v0) < (uint64_t)PV) {
+#pragma unroll
+                        for (int e = 0; e < PV; ++e)
+                            if (v0 + e == cf.t0) o[e] -= cf.c0;
+                    }
+                    if ((uint64_t)(cf.t1 - v0) < (uint64_t)PV) {
+#pragma unroll
+                        for (int e = 0; e < PV; ++e)
+                            if (v0 + e == cf.t1) o[e] -= cf.c1;
+                    }
+                    grad_store<T, G, PV>(g, v0, o, pol);
+                }
+            });
+    }
+}
+
 template <typename T, bool VEC, typename G>
 __device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* grad) {
     grad_pass_range<T, VEC, G>(P, r, 0, P.V, rstats, grad);
@@ -1214,19 +1656,18 @@ __device__ void tree_pass(const Problem<T>& P, int b, Ring* rg, float4* tab, Tre
         const T* x = P.draft + (int64_t)r * V;
         const T* y = P.target + (int64_t)r * V;
         const float c = P.ts.c;
-        const MassRes mr{sh.rec.mx, sh.rec.my, (float)exp(-sh.rec.lzx), (float)exp(-sh.rec.lzy),
-                         c};
+        const MassRes mr{sh.rec.mx, sh.rec.my, sh.rec.izx, sh.rec.izy, c};
         stream_residual<T, VEC>(rg, x, y, V, 0, P.nch, tab, mr, P.status);
         __syncthreads();
         if (warp == 0) {
-            const double Rt = table_total(tab, P.nch, 0, 0.f, c, lane);
-            if (lane == 0) sh.rt = Rt;
-            if (Rt > 0.0) {
+            const TableSum Rt = table_sum(tab, P.nch, 0, 0.f, c, lane);
+            if (lane == 0) sh.rt = Rt.Z;
+            if (Rt.Z > 0.0) {
                 for (int n = first; n < N; ++n) {
                     if (__ldg(par + n) != u || sh.pacc[n]) continue;
                     const float un = __ldg(P.u_correct + n0 + n);
                     const Located loc =
-                        table_locate(tab, P.nch, 0, 0.f, c, (double)un * Rt, lane);
+                        table_locate(tab, P.nch, 0, 0.f, c, Rt, un, lane);
                     int tok = -1;
                     if (loc.ch >= 0)
                         tok = warp_rescan<T, VEC, true, true>(x, y, V, loc.ch, loc.tc, mr, lane,
