@@ -32,7 +32,7 @@ struct WsLayout {
 
 // Chunks per segment of the fused kernel's work items.
 #ifndef VSD_SEG_CHUNKS
-#define VSD_SEG_CHUNKS 64
+#define VSD_SEG_CHUNKS 128
 #endif
 constexpr int kSegChunks = VSD_SEG_CHUNKS;
 

@@ -112,7 +112,10 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int* status, uint64_t
 // that only move logits, and one control warp (the last) that claims work,
 // keeps the counters and runs every per-row, per-path and per-prefix step.
 constexpr int kFusedThreads = kThreads + 32;
-constexpr int kSlots = 3;  // jobs handed to the streaming warps ahead of time
+#ifndef VSD_SLOTS
+#define VSD_SLOTS 2
+#endif
+constexpr int kSlots = VSD_SLOTS;  // jobs handed to the streaming warps ahead of time
 // Named barriers (0 is __syncthreads): slot s is FULL (1 + s) when the control
 // warp has written a job into it, DONE (1 + kSlots + s) when the streaming
 // warps have finished that job.
@@ -219,8 +222,9 @@ __device__ bool claim_job(const Problem<T>& P, bool wait, int& g, Job& j) {
 }
 
 // Last-finisher counter (control warp): lane 0 adds one to *cnt after a fence
-// and every lane learns whether it completed the count n.
+// and every lane learns whether it completed the count n (n = 1: no counter).
 __device__ __forceinline__ bool warp_count_last(int* cnt, int n, int lane) {
+    if (n == 1) return true;
     int last = 0;
     if (lane == 0) {
         __threadfence();
@@ -390,7 +394,10 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
     int g = *(volatile int*)P.grad_head;
     int head = 0, tail = 0, inflight = 0;
     bool ended = false;
-    for (;;) {
+    __shared__ Job cur;
+    // Fill the free slots.  A claim may wait only when no job is in flight
+    // (then no follow-up step is owed either).
+    auto fill = [&]() {
         while (!ended && inflight < kSlots) {
             int got = 0;
             if (lane == 0) got = claim_job<T>(P, inflight == 0, g, slots[tail % kSlots]) ? 1 : 0;
@@ -406,13 +413,18 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
             }
             ++inflight;
         }
+    };
+    for (;;) {
+        fill();
         if (inflight == 0) break;
         const int s = head % kSlots;
         named_sync(bar_done(s));
-        if (slots[s].kind != kJobGrad) post_job<T, VEC>(P, E, slots[s], tab, cs, lane);
+        if (lane == 0) cur = slots[s];
         __syncwarp();
         ++head;
         --inflight;
+        if (cur.kind != kJobGrad) post_job<T, VEC>(P, E, cur, tab, cs, lane);
+        __syncwarp();
     }
 }
 
