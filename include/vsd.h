@@ -208,6 +208,38 @@ vsd_status vsd_estep_mstep_noalloc(const void* draft, const void* target, vsd_dt
                                    const float* ref_logkappa, const vsd_params* params,
                                    vsd_linear_outputs* out, void* stream);
 
+/* The draft model's LM head, the layer that produces the draft logits q is
+ * computed from (paper Sec. 5, implementation details: the draft head's output
+ * layer):  logits[M][N] = hidden[M][K] . weight[N][K]^T.
+ *   hidden  device, bf16, row-major [M][K] (K contiguous);
+ *   weight  device, bf16, row-major [N][K] (the vocabulary-by-hidden matrix);
+ *   logits  device, bf16, row-major [M][N], written (caller-owned);
+ *   ws      device workspace of at least 256 bytes whose first word is the
+ *           status word (the same as a vsd_estep_mstep workspace); cleared here.
+ * Products are exact and summed in fp32 on the tensor cores, then rounded once
+ * to bf16 (round to nearest even).  N and K must be multiples of 8 and the
+ * three pointers 16-byte aligned (VSD_ERR_INVALID_ARG otherwise); M >= 1.
+ * Asynchronous on `stream`; a device wait that runs out sets the timeout bit
+ * of the status word (vsd_device_status). */
+vsd_status vsd_lmhead_logits(const void* hidden, const void* weight, int32_t M, int32_t N,
+                             int32_t K, void* logits, void* ws, size_t ws_bytes, void* stream);
+
+/* The LM head followed by the fused E-step + M-step on its logits (config of
+ * the draft head fused with the EM step):
+ *   hidden        device, bf16 [R][H], R = B*K*D rows in the layout's row order;
+ *   weight        device, bf16 [V][H];
+ *   target        device, bf16 [R][V], the target logits;
+ *   draft_logits  device, bf16 [R][V], receives the draft logits (caller-owned);
+ * every other argument as for vsd_estep_mstep with dtype VSD_BF16 (linear
+ * layouts only).  The status word of `ws` collects the bits of both steps. */
+vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_t H,
+                                  const void* target, vsd_layout layout, float T,
+                                  const float* u_draft, const float* u_accept,
+                                  const float* u_correct, const float* ref_logkappa,
+                                  const vsd_params* params, void* draft_logits,
+                                  vsd_linear_outputs* out, void* ws, size_t ws_bytes,
+                                  void* stream);
+
 /* Waits for `stream`, then reads and clears the device status word of `ws`
  * into *status_bits (host).  Returns VSD_ERR_TIMEOUT if the timeout bit is set,
  * VSD_ERR_DEVICE_DATA for any other bit, VSD_OK if none. */

@@ -185,3 +185,22 @@ def prefix_objective(draft, T, tokens, corr_tokens, weights, N, B_total, want_gr
     J = lib().vso_prefix_objective(_ptr(draft), K, D, V, float(T), _ptr(tok), _ptr(ctok),
                                    _ptr(w), float(N), int(B_total), _ptr(g))
     return J, g
+
+
+def lmhead_logits(hidden, weight):
+    """The draft LM head (paper Sec. 5, the draft head's output layer): logits =
+    hidden . weight^T from the exact input values, in float64 (a library
+    matmul: one product per (row, vocabulary entry), no blocking of our own)."""
+    h = np.asarray(hidden, dtype=np.float64)
+    w = np.asarray(weight, dtype=np.float64)
+    return h @ w.T
+
+
+def round_bf16(x):
+    """Round float64 values to the nearest bfloat16 (8 significant bits), ties
+    to even, returned as float32 holding the bfloat16 value exactly.  Finite
+    values in the normal range of bfloat16."""
+    x = np.asarray(x, dtype=np.float64)
+    m, e = np.frexp(x)                     # x = m 2^e, 0.5 <= |m| < 1
+    r = np.rint(m * 256.0) / 256.0         # 8 significant bits; rint rounds ties to even
+    return np.ldexp(r, e).astype(np.float32)

@@ -292,7 +292,8 @@ template <typename T>
 vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float T_,
                       const float* u_draft, const float* u_accept, const float* u_correct,
                       const float* ref_logkappa, const vsd_params& p,
-                      const vsd_linear_outputs* out, void* ws, cudaStream_t s) {
+                      const vsd_linear_outputs* out, void* ws, cudaStream_t s,
+                      bool clear = true) {
     Problem<T> P = make_problem<T>(draft, target, L, T_, ws);
     set_params(P, p);
     P.u_draft = u_draft;
@@ -308,7 +309,7 @@ vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float
     if ((int64_t)ctas > tickets) ctas = (int)tickets;
     const char* env_ctas = getenv("VSD_FUSED_CTAS");
     if (env_ctas && atoi(env_ctas) > 0 && atoi(env_ctas) < ctas) ctas = atoi(env_ctas);
-    cudaError_t e = clear_counters(ws, L, s);
+    cudaError_t e = clear ? clear_counters(ws, L, s) : cudaSuccess;
     if (e == cudaSuccess) e = Launch<T>::fused(P, vec, out->grad, P.grad_bf16, ctas, s);
     return from_cuda(e);
 }
@@ -415,6 +416,46 @@ vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtyp
                                  ref_logkappa, p, out, ws, s);
     return fused_impl<__nv_bfloat16>(draft, target, layout, T, u_draft, u_accept, u_correct,
                                      ref_logkappa, p, out, ws, s);
+}
+
+vsd_status vsd_lmhead_logits(const void* hidden, const void* weight, int32_t M, int32_t N,
+                             int32_t K, void* logits, void* ws, size_t ws_bytes, void* stream) {
+    if (!lmhead_shape_ok(hidden, weight, logits, M, N, K)) return VSD_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < 256 || ((uintptr_t)ws & 255)) return VSD_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int32_t), s);
+    if (e == cudaSuccess) e = lmhead_gemm(hidden, weight, M, N, K, logits, static_cast<int*>(ws), s);
+    return from_cuda(e);
+}
+
+vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_t H,
+                                  const void* target, vsd_layout layout, float T,
+                                  const float* u_draft, const float* u_accept,
+                                  const float* u_correct, const float* ref_logkappa,
+                                  const vsd_params* params, void* draft_logits,
+                                  vsd_linear_outputs* out, void* ws, size_t ws_bytes,
+                                  void* stream) {
+    if (!layout_ok(layout) || layout.parent) return VSD_ERR_INVALID_ARG;
+    if (!target || !u_draft || !u_accept || !u_correct || !out) return VSD_ERR_INVALID_ARG;
+    if (!out->tokens || !out->accept_len || !out->corr_tokens || !out->logkappa || !out->loss ||
+        !out->grad)
+        return VSD_ERR_INVALID_ARG;
+    const int64_t R = rows_of(layout);
+    if (R > (1 << 30) || !lmhead_shape_ok(hidden, weight, draft_logits, (int)R, layout.V, H))
+        return VSD_ERR_INVALID_ARG;
+    vsd_status st = check_temperature(T);
+    if (st) return st;
+    const vsd_params p = params ? *params : default_params(VSD_BF16);
+    if ((st = check_params(p))) return st;
+    if ((st = check_ws(layout, ws, ws_bytes))) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    // the counters and the status word are cleared once, before both steps
+    cudaError_t e = clear_counters(ws, layout, s);
+    if (e == cudaSuccess)
+        e = lmhead_gemm(hidden, weight, (int)R, layout.V, H, draft_logits, static_cast<int*>(ws), s);
+    if (e != cudaSuccess) return from_cuda(e);
+    return fused_impl<__nv_bfloat16>(draft_logits, target, layout, T, u_draft, u_accept,
+                                     u_correct, ref_logkappa, p, out, ws, s, false);
 }
 
 vsd_status vsd_device_status(void* ws, void* stream, int32_t* status_bits) {

@@ -37,4 +37,11 @@ inline size_t stream_smem_bytes(int nch, bool vec) {
     return (vec ? sizeof(Ring) : 0) + table_smem_bytes(nch);
 }
 
+// The draft LM head on the tensor cores (vsd_lmhead.cu): logits = hidden .
+// weight^T, bf16 in, fp32 accumulation, bf16 out; status collects timeouts.
+bool lmhead_shape_ok(const void* hidden, const void* weight, const void* logits, int M, int N,
+                     int K);
+cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, int K, void* logits,
+                        int* status, cudaStream_t s);
+
 }  // namespace vsd

@@ -1,0 +1,392 @@
+// vsd_lmhead.cu -- the draft model's LM head on the tensor cores:
+// logits[M][N] = hidden[M][K] . weight[N][K]^T, bf16 inputs, fp32 accumulation
+// in tensor memory (TMEM), bf16 logits out (the draft head that produces q,
+// paper Sec. 5 implementation details).  Then the fused E-step + M-step on those
+// logits (vsd_lmhead_estep_mstep).
+//
+// One persistent CTA per SM computes 128 x 256 output tiles:
+//   warp 0   TMA producer: 128 x 64 hidden and 256 x 64 weight tiles (128-byte
+//            swizzle) into a 4-stage shared-memory ring;
+//   warp 1   MMA issuer: one thread issues tcgen05.mma (kind::f16, M=128,
+//            N=256, K=16) into one of two TMEM accumulators (2 x 256 columns);
+//            tcgen05.commit frees a ring stage / hands a finished accumulator on;
+//   warps 2-5 epilogue: tcgen05.ld of the accumulator (each warp its 32 TMEM
+//            lanes = 32 tile rows), rounding to bf16, 16-byte stores.
+// The epilogue of one tile overlaps the main loop of the next.  Every wait is
+// bounded; a wait that runs out sets VSD_STATUS_TIMEOUT in the status word and
+// the CTA winds down (waiting, again bounded, for its copies and MMAs in
+// flight) and frees its tensor memory.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "vsd.h"
+#include "vsd_common.cuh"
+
+namespace vsd_lm {
+
+using vsd::global_timer_ns;
+using vsd::mbar_expect_tx;
+using vsd::mbar_init;
+using vsd::mbar_init_fence;
+using vsd::mbar_try_wait;
+using vsd::smem_u32;
+
+constexpr int BM = 128, BN = 256, BK = 64;  // BK bf16 = one 128-byte swizzle row
+constexpr int kStages = 4;
+constexpr int kThreads = 192;
+constexpr int kABytes = BM * BK * 2;  // 16 KB
+constexpr int kBBytes = BN * BK * 2;  // 32 KB
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kTmemCols = 2 * BN;  // two fp32 accumulators of 128 lanes x 256 columns
+constexpr uint64_t kWaitNs = 2000000000ull;
+
+struct Bars {
+    uint64_t full[kStages];   // TMA bytes landed in stage s
+    uint64_t empty[kStages];  // the MMAs reading stage s are done
+    uint64_t acc_full[2];     // accumulator b holds a finished tile
+    uint64_t acc_empty[2];    // the epilogue has read accumulator b (4 arrivals)
+    uint64_t drain;           // the MMA warp's final commit
+    uint32_t tmem_base;
+    int err;
+};
+constexpr size_t kSmemBytes = 1024 /* alignment slack */ + kStages * kStageBytes + sizeof(Bars);
+
+// ---------------------------------------------------------------- PTX wrappers
+// 2-D tiled TMA load global -> shared, completion counted on `bar`.  x is the
+// inner (K) coordinate in elements, y the row.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y,
+                                            uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];"
+        :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y),
+           "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major bf16 tile written by TMA with
+// the 128-byte swizzle: rows of 128 bytes, 8-row groups 1024 bytes apart
+// (stride byte offset), the leading byte offset unused for this layout,
+// descriptor version 1, swizzle mode 2 (128 bytes).  The tile base is
+// 1024-byte aligned, so the base-offset field is 0; a K step of 16 elements
+// inside the 128-byte row advances the start address by 32 bytes.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // bits 0-13: start address / 16
+    d |= (uint64_t)1 << 16;                    // bits 16-29: leading byte offset / 16
+    d |= (uint64_t)(1024 >> 4) << 32;          // bits 32-45: stride byte offset / 16
+    d |= (uint64_t)1 << 46;                    // bits 46-48: version
+    d |= (uint64_t)2 << 61;                    // bits 61-63: 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, N = 256, M = 128.
+constexpr uint32_t kIdesc = (1u << 4)                      // D format f32
+                            | (1u << 7)                    // A format bf16
+                            | (1u << 10)                   // B format bf16
+                            | ((uint32_t)(BN >> 3) << 17)  // N / 8
+                            | ((uint32_t)(BM >> 4) << 24); // M / 16
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        :: "r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive on `bar` once every tcgen05.mma this thread issued so far is done.
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+        :: "r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32"
+        " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15,"
+        " %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31},"
+        " [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Bounded wait for the completion of the barrier phase with parity `parity`.
+__device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity, Bars* sb,
+                                           int* status) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*(volatile int*)&sb->err) return false;
+        if (global_timer_ns() - t0 > kWaitNs) {
+            sb->err = 1;
+            atomicOr(status, VSD_STATUS_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+// Bounded wait that ignores the error flag (winding down after an error: the
+// copies and MMAs already issued must finish before the CTA exits).
+__device__ __forceinline__ void wait_phase_drain(uint64_t* bar, uint32_t parity) {
+    const uint64_t t0 = global_timer_ns();
+    while (!mbar_try_wait(bar, parity))
+        if (global_timer_ns() - t0 > kWaitNs) return;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(uint32_t lo, uint32_t hi) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(lo), __uint_as_float(hi));
+    return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// Tiles are numbered with the M tile fastest, so the CTAs working at the same
+// time share the same few weight tiles (read from DRAM once, then from L2) and
+// the hidden states stay in L2 throughout.
+__global__ void __launch_bounds__(kThreads, 1)
+    k_lmhead(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+             __nv_bfloat16* __restrict__ out, int M, int N, int K, int* status) {
+    extern __shared__ unsigned char dsm_raw[];
+    unsigned char* dsm = dsm_raw + ((1024u - (smem_u32(dsm_raw) & 1023u)) & 1023u);
+    Bars* sb = reinterpret_cast<Bars*>(dsm + kStages * kStageBytes);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int mt = (M + BM - 1) / BM, nt = (N + BN - 1) / BN;
+    const int ntiles = mt * nt, nk = (K + BK - 1) / BK;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&sb->full[s], 1);
+            mbar_init(&sb->empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&sb->acc_full[b], 1);
+            mbar_init(&sb->acc_empty[b], 4);
+        }
+        mbar_init(&sb->drain, 1);
+        sb->err = 0;
+        mbar_init_fence();
+    }
+    if (warp == 1) {  // the whole warp allocates the two accumulators
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                     :: "r"(smem_u32(&sb->tmem_base)), "r"(kTmemCols) : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = sb->tmem_base;
+
+    if (warp == 0) {
+        // ------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            uint32_t it = 0;
+            for (int t = blockIdx.x; t < ntiles && !*(volatile int*)&sb->err; t += gridDim.x) {
+                const int m0 = (t % mt) * BM, n0 = (t / mt) * BN;
+                bool ok = true;
+                for (int kb = 0; kb < nk; ++kb) {
+                    const int s = (int)(it % kStages);
+                    const uint32_t round = it / kStages;
+                    if (round > 0 && !wait_phase(&sb->empty[s], (round - 1) & 1u, sb, status)) {
+                        ok = false;
+                        break;
+                    }
+                    unsigned char* a = dsm + s * kStageBytes;
+                    mbar_expect_tx(&sb->full[s], kStageBytes);
+                    tma_load_2d(a, &tmA, kb * BK, m0, &sb->full[s]);
+                    tma_load_2d(a + kABytes, &tmB, kb * BK, n0, &sb->full[s]);
+                    ++it;
+                }
+                if (!ok) break;
+            }
+            // the last copies issued have landed before the CTA may exit
+            for (uint32_t j = it > (uint32_t)kStages ? it - kStages : 0; j < it; ++j)
+                wait_phase_drain(&sb->full[j % kStages], (j / kStages) & 1u);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            uint32_t it = 0;
+            int lt = 0;
+            for (int t = blockIdx.x; t < ntiles && !*(volatile int*)&sb->err;
+                 t += gridDim.x, ++lt) {
+                const int buf = lt & 1;
+                const uint32_t use = (uint32_t)lt >> 1;
+                if (use > 0 && !wait_phase(&sb->acc_empty[buf], (use - 1) & 1u, sb, status)) break;
+                tc_fence_after();
+                const uint32_t d = tmem + (uint32_t)(buf * BN);
+                bool ok = true;
+                for (int kb = 0; kb < nk; ++kb) {
+                    const int s = (int)(it % kStages);
+                    if (!wait_phase(&sb->full[s], (it / kStages) & 1u, sb, status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a = smem_u32(dsm + s * kStageBytes), b = a + kABytes;
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k)
+                        mma_bf16(d, sdesc_sw128(a + 32u * k), sdesc_sw128(b + 32u * k),
+                                 (kb | k) != 0 ? 1u : 0u);
+                    mma_commit(&sb->empty[s]);  // frees the stage once these MMAs are done
+                    ++it;
+                }
+                if (!ok) break;
+                mma_commit(&sb->acc_full[buf]);
+            }
+            // every MMA this thread issued is complete once this arrives
+            mma_commit(&sb->drain);
+            wait_phase_drain(&sb->drain, 0);
+        }
+    } else {
+        // ------------------------------------------------------ epilogue
+        const int q = warp & 3;  // this warp may access TMEM lanes 32q .. 32q + 31
+        int lt = 0;
+        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++lt) {
+            const int buf = lt & 1;
+            const uint32_t use = (uint32_t)lt >> 1;
+            if (!wait_phase(&sb->acc_full[buf], use & 1u, sb, status)) break;
+            tc_fence_after();
+            const int m0 = (t % mt) * BM, n0 = (t / mt) * BN;
+            const int row = m0 + 32 * q + lane;
+            const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN);
+#pragma unroll 1
+            for (int c = 0; c < BN / 32; ++c) {
+                uint32_t r[32];
+                tmem_ld32(taddr + 32u * c, r);
+                const int col = n0 + 32 * c;
+                if (row < M && col < N) {
+                    __nv_bfloat16* o = out + (size_t)row * N + col;
+#pragma unroll
+                    for (int v = 0; v < 4; ++v)
+                        if (col + 8 * v < N)
+                            *reinterpret_cast<uint4*>(o + 8 * v) =
+                                make_uint4(pack_bf16(r[8 * v + 0], r[8 * v + 1]),
+                                           pack_bf16(r[8 * v + 2], r[8 * v + 3]),
+                                           pack_bf16(r[8 * v + 4], r[8 * v + 5]),
+                                           pack_bf16(r[8 * v + 6], r[8 * v + 7]));
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sb->acc_empty[buf]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;"
+                     :: "r"(tmem), "r"(kTmemCols) : "memory");
+    }
+}
+
+// ---------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no link
+// against the driver library).
+EncodeTiledFn encode_fn() {
+    static std::once_flag once;
+    static EncodeTiledFn fn = nullptr;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// Tensor map of a row-major bf16 matrix [rows][cols] read in boxes of
+// box_rows x 64 columns with the 128-byte swizzle; out-of-range elements read
+// as zero (they add nothing to a dot product).
+bool make_map(CUtensorMap* m, const void* base, int rows, int cols, int box_rows) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
+
+}  // namespace vsd_lm
+
+namespace vsd {
+
+bool lmhead_shape_ok(const void* hidden, const void* weight, const void* logits, int M, int N,
+                     int K) {
+    if (!hidden || !weight || !logits) return false;
+    if (M < 1 || N < 8 || K < 8) return false;
+    if (N % 8 || K % 8) return false;  // 16-byte rows for TMA and for the stores
+    if (((uintptr_t)hidden | (uintptr_t)weight | (uintptr_t)logits) & 15) return false;
+    return true;
+}
+
+cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, int K, void* logits,
+                        int* status, cudaStream_t s) {
+    using vsd_lm::k_lmhead;
+    using vsd_lm::make_map;
+    CUtensorMap ta, tb;
+    if (!make_map(&ta, hidden, M, K, vsd_lm::BM) || !make_map(&tb, weight, N, K, vsd_lm::BN))
+        return cudaErrorInvalidValue;
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    {  // the shared-memory opt-in, once per device
+        static std::mutex mu;
+        static bool done[256];
+        std::lock_guard<std::mutex> lock(mu);
+        if (dev < 0 || dev >= 256) return cudaErrorInvalidDevice;
+        if (!done[dev]) {
+            e = cudaFuncSetAttribute(k_lmhead, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)vsd_lm::kSmemBytes);
+            if (e != cudaSuccess) return e;
+            done[dev] = true;
+        }
+    }
+    const long long ntiles =
+        (long long)((M + vsd_lm::BM - 1) / vsd_lm::BM) * ((N + vsd_lm::BN - 1) / vsd_lm::BN);
+    const int grid = (int)(ntiles < sms ? ntiles : sms);
+    // (qualified: the enclosing namespace has a kThreads of its own)
+    k_lmhead<<<grid, vsd_lm::kThreads, vsd_lm::kSmemBytes, s>>>(
+        ta, tb, static_cast<__nv_bfloat16*>(logits), M, N, K, status);
+    return cudaGetLastError();
+}
+
+}  // namespace vsd

@@ -192,3 +192,23 @@ def lmhead_problem(B, K, D, V, H, device="cpu", seed=BASE_SEED):
                 weight=weight.contiguous(), target=t.to(torch.bfloat16).contiguous(),
                 u_draft=uniforms(R, device, seed + 3), u_accept=uniforms(R, device, seed + 4),
                 u_correct=uniforms(R, device, seed + 5))
+
+
+def lmhead_exact_problem(B, K, D, V, H, device="cpu", seed=BASE_SEED):
+    """LM-head inputs whose products and partial sums are all exact in float32:
+    hidden in {-2, ..., 2}, weight in {-64, ..., 64} / 256, so every product is
+    a multiple of 2^-8 of magnitude at most 1/2 and every partial sum a
+    multiple of 2^-8 below H/2: exact in float32 (24 bits) for H < 2^17.  Any
+    summation order then gives the exact logits before the one rounding to
+    bf16.  Target logits and uniforms as in lmhead_problem."""
+    R = B * K * D
+    g = _gen(device, seed + 9)
+    hidden = torch.randint(-2, 3, (R, H), generator=g, device=device).to(torch.bfloat16)
+    weight = (torch.randint(-64, 65, (V, H), generator=g, device=device).float() / 256.0).to(
+        torch.bfloat16)
+    t = logits_spiked(R, V, 3.0, min(50, V), 8.0, device, seed + 1) + logits_gaussian(
+        R, V, 1.0, device, seed + 2)
+    return dict(B=B, K=K, D=D, V=V, H=H, dtype="bf16", hidden=hidden.contiguous(),
+                weight=weight.contiguous(), target=t.to(torch.bfloat16).contiguous(),
+                u_draft=uniforms(R, device, seed + 3), u_accept=uniforms(R, device, seed + 4),
+                u_correct=uniforms(R, device, seed + 5))

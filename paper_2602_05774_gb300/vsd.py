@@ -22,7 +22,8 @@ _STATUS_NAMES = {0: "VSD_OK", 1: "VSD_ERR_INVALID_ARG", 2: "VSD_ERR_UNSUPPORTED"
 
 SYMBOLS = ("vsd_workspace_bytes", "vsd_sample_paths", "vsd_verify_paths",
            "vsd_weighted_loss_fwd_bwd", "vsd_estep_mstep", "vsd_device_status",
-           "vsd_status_string", "vsd_version", "vsd_estep_mstep_noalloc")
+           "vsd_status_string", "vsd_version", "vsd_estep_mstep_noalloc",
+           "vsd_lmhead_logits", "vsd_lmhead_estep_mstep")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -90,12 +91,18 @@ def _lib():
         lib.vsd_estep_mstep_noalloc.argtypes = [vp, vp, C.c_int, Layout, C.c_float, vp, vp, vp,
                                                 vp, C.POINTER(Params), C.POINTER(LinearOutputs),
                                                 vp]
+        lib.vsd_lmhead_logits.argtypes = [vp, vp, C.c_int32, C.c_int32, C.c_int32, vp, vp,
+                                          C.c_size_t, vp]
+        lib.vsd_lmhead_estep_mstep.argtypes = [vp, vp, C.c_int32, vp, Layout, C.c_float, vp, vp,
+                                               vp, vp, C.POINTER(Params), vp,
+                                               C.POINTER(LinearOutputs), vp, C.c_size_t, vp]
         lib.vsd_device_status.argtypes = [vp, vp, C.POINTER(C.c_int32)]
         lib.vsd_status_string.argtypes = [C.c_int]
         lib.vsd_status_string.restype = C.c_char_p
         lib.vsd_version.restype = C.c_char_p
         for name in ("vsd_sample_paths", "vsd_verify_paths", "vsd_weighted_loss_fwd_bwd",
-                     "vsd_estep_mstep", "vsd_device_status", "vsd_estep_mstep_noalloc"):
+                     "vsd_estep_mstep", "vsd_device_status", "vsd_estep_mstep_noalloc",
+                     "vsd_lmhead_logits", "vsd_lmhead_estep_mstep"):
             getattr(lib, name).restype = C.c_int
         _LIB = lib
     return _LIB
@@ -316,6 +323,54 @@ def estep_mstep(draft, target, u_draft, u_accept, u_correct, K, D, T, ref_logkap
                                   _ptr(u_draft), _ptr(u_accept), _ptr(u_correct),
                                   _ptr(ref_logkappa), C.byref(prm), C.byref(st), _ptr(ws),
                                   ws.numel(), _stream(dev)), "vsd_estep_mstep")
+    return out
+
+
+def lmhead_logits(hidden, weight, out=None, workspace=None):
+    """Draft logits [M][N] = hidden [M][K] . weight [N][K]^T on the tensor cores
+    (bf16 in, fp32 accumulation, bf16 out)."""
+    _need_cuda(hidden, weight)
+    if hidden.dtype != torch.bfloat16 or weight.dtype != torch.bfloat16:
+        raise ValueError("the LM head takes bf16 hidden states and weights")
+    M, K = hidden.shape
+    N = weight.shape[0]
+    if weight.shape[1] != K:
+        raise ValueError("hidden and weight disagree on the hidden size")
+    dev = hidden.device
+    if out is None:
+        out = torch.empty(M, N, dtype=torch.bfloat16, device=dev)
+    ws = workspace if workspace is not None else torch.empty(256, dtype=torch.uint8, device=dev)
+    _check(_lib().vsd_lmhead_logits(_ptr(hidden), _ptr(weight), M, N, K, _ptr(out), _ptr(ws),
+                                    ws.numel(), _stream(dev)), "vsd_lmhead_logits")
+    return out
+
+
+def lmhead_estep_mstep(hidden, weight, target, u_draft, u_accept, u_correct, K, D, T,
+                       ref_logkappa=None, prm=None, workspace=None, out=None, draft_logits=None,
+                       full=True):
+    """The LM head, then the fused E-step + M-step on its logits.  Returns the
+    outputs of estep_mstep() plus "draft_logits"."""
+    _need_cuda(hidden, weight, target, u_draft, u_accept, u_correct, ref_logkappa)
+    V = weight.shape[0]
+    H = hidden.shape[-1]
+    R = hidden.numel() // H
+    B = R // (K * D)
+    lay = layout(B, K, D, V)
+    dev = hidden.device
+    ws = _ws(workspace, lay, dev)
+    prm = prm or params(like=target)
+    if draft_logits is None:
+        draft_logits = torch.empty(R, V, dtype=torch.bfloat16, device=dev)
+    if out is None:
+        gdt = torch.bfloat16 if prm.grad_dtype == VSD_BF16 else torch.float32
+        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full)
+    st = _linear_struct(out)
+    _check(_lib().vsd_lmhead_estep_mstep(_ptr(hidden), _ptr(weight), H, _ptr(target), lay,
+                                         float(T), _ptr(u_draft), _ptr(u_accept),
+                                         _ptr(u_correct), _ptr(ref_logkappa), C.byref(prm),
+                                         _ptr(draft_logits), C.byref(st), _ptr(ws), ws.numel(),
+                                         _stream(dev)), "vsd_lmhead_estep_mstep")
+    out["draft_logits"] = draft_logits
     return out
 
 

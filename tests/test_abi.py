@@ -100,3 +100,29 @@ def test_binding_refuses_cpu_tensors(vsd):
     u = torch.zeros(4)
     with pytest.raises(ValueError):
         vsd.sample_paths(x, u, 1, 4, 1.0)
+
+
+def test_lmhead_argument_checks_before_any_launch(vsd):
+    lib = vsd.load()
+    fake = C.c_void_p(0x1000)  # never dereferenced: every call below fails its checks
+    ws = C.c_void_p(0x100000)
+    # N and K must be multiples of 8, M >= 1, pointers 16-byte aligned
+    assert lib.vsd_lmhead_logits(fake, fake, 128, 260, 64, fake, ws, 256, None) == 1
+    assert lib.vsd_lmhead_logits(fake, fake, 128, 256, 60, fake, ws, 256, None) == 1
+    assert lib.vsd_lmhead_logits(fake, fake, 0, 256, 64, fake, ws, 256, None) == 1
+    assert lib.vsd_lmhead_logits(C.c_void_p(0x1008), fake, 128, 256, 64, fake, ws, 256,
+                                 None) == 1
+    assert lib.vsd_lmhead_logits(None, fake, 128, 256, 64, fake, ws, 256, None) == 1
+    # workspace: present, 256 bytes, 256-byte aligned
+    assert lib.vsd_lmhead_logits(fake, fake, 128, 256, 64, fake, None, 256, None) == 5
+    assert lib.vsd_lmhead_logits(fake, fake, 128, 256, 64, fake, ws, 16, None) == 5
+    # the fused variant: linear layouts only, H a multiple of 8
+    lay = vsd.layout(2, 4, 4, 1024)
+    o = vsd.LinearOutputs(*([0x1000] * len(vsd.LINEAR_FIELDS)))
+    assert lib.vsd_lmhead_estep_mstep(fake, fake, 100, fake, lay, 1.0, fake, fake, fake, None,
+                                      None, fake, C.byref(o), ws, 1 << 30, None) == 1
+    tlay = vsd.Layout(2, 1, 1, 1024, 60, 0x1000)
+    assert lib.vsd_lmhead_estep_mstep(fake, fake, 128, fake, tlay, 1.0, fake, fake, fake, None,
+                                      None, fake, C.byref(o), ws, 1 << 30, None) == 1
+    assert lib.vsd_lmhead_estep_mstep(fake, fake, 128, fake, lay, 0.0, fake, fake, fake, None,
+                                      None, fake, C.byref(o), ws, 1 << 30, None) == 2

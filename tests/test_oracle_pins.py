@@ -438,3 +438,47 @@ def test_theorems_by_enumeration(oracle):
     assert abs(elbo_star - math.log(Z)) < 1e-12  # Theorem 2, equality
     assert elbo_star > elbo_kl  # Theorem 2, strict when kappa varies
     assert elbo <= elbo_star + 1e-12  # the posterior maximises the ELBO
+
+
+# --------------------------------------------------------------------------
+# The draft LM head (Sec. 5, the draft head's output layer) and bf16 rounding
+
+
+def test_lmhead_one_hot_rows_pick_weight_columns(oracle):
+    """A one-hot hidden state e_k gives logits W[:, k]; e_i + e_j gives the sum
+    of two columns.  A transposed operand or a dropped term fails here."""
+    rng = np.random.default_rng(5)
+    V, H = 7, 5
+    W = rng.integers(-9, 10, size=(V, H)).astype(np.float64) / 4
+    hid = np.zeros((3, H))
+    hid[0, 2] = 1.0
+    hid[1, 4] = 1.0
+    hid[2, 0] = hid[2, 3] = 1.0
+    lg = oracle.lmhead_logits(hid, W)
+    assert lg.shape == (3, V)
+    assert np.array_equal(lg[0], W[:, 2])
+    assert np.array_equal(lg[1], W[:, 4])
+    assert np.array_equal(lg[2], W[:, 0] + W[:, 3])
+
+
+def test_lmhead_closed_form_sums(oracle):
+    """hidden = all ones, W[v, k] = v - k: logits[v] = H v - H (H - 1) / 2."""
+    V, H = 6, 9
+    W = np.subtract.outer(np.arange(V), np.arange(H)).astype(np.float64)
+    lg = oracle.lmhead_logits(np.ones((2, H)), W)
+    want = H * np.arange(V) - H * (H - 1) / 2
+    assert np.array_equal(lg[0], want) and np.array_equal(lg[1], want)
+
+
+def test_round_bf16_ties_to_even_and_matches_torch(oracle):
+    one = 1.0
+    # halfway cases: 1 + 2^-8 lies between 1 and 1 + 2^-7 -> even (1);
+    # 1 + 3 * 2^-8 between 1 + 2^-7 and 1 + 2^-6 -> even (1 + 2^-6)
+    x = np.array([one + 2.0**-8, one + 3 * 2.0**-8, -(one + 2.0**-8), 2.0**-9 * 3, 0.0])
+    r = oracle.round_bf16(x)
+    assert r.tolist() == [1.0, 1.0 + 2.0**-6, -1.0, 2.0**-9 * 3, 0.0]
+    # on float32 inputs (no double rounding) it is torch's round-to-nearest-even cast
+    torch = pytest.importorskip("torch")
+    f = np.random.default_rng(3).standard_normal(20000).astype(np.float32) * 40
+    want = torch.from_numpy(f).to(torch.bfloat16).float().numpy()
+    assert np.array_equal(oracle.round_bf16(f.astype(np.float64)), want)
