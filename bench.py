@@ -20,12 +20,17 @@ import sys
 import threading
 import time
 
+# The oracle baseline is single-threaded: keep numpy's BLAS (the oracle's LM
+# head) on one core so that "cores": 1 holds.
+for _v in ("OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = ("draft-logit rows/s and achieved HBM GB/s (fraction of GB300 roofline) for fused "
           "E/M step")
-WORKLOADS = ("vocab128k", "vocab32k", "tiny")
+WORKLOADS = ("vocab128k", "vocab32k", "tiny", "lmhead")
 
 
 def parse():
@@ -57,6 +62,16 @@ def peaks():
         return float(d["hbm_gbs"]), "measured"
     except Exception:
         return 6800.0, "fallback"
+
+
+def tensor_peak():
+    """Measured cuBLAS bf16 throughput (burst: the GEMM is timed on its own)."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(path))
+        return float(d["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
 
 
 def kernel_source_hash():
@@ -343,9 +358,193 @@ def run_ours(args):
     print(json.dumps(line), flush=True)
 
 
+
+def oracle_lmhead_sample(prob, rows, T):
+    """The oracle's LM head (fp64 matmul, one bf16 rounding) and E/M step on the
+    first `rows` rows: seconds."""
+    from oracle import oracle
+    K, D = prob["K"], prob["D"]
+    h = prob["hidden"][:rows].float().cpu().numpy()
+    w = prob["weight"].float().cpu().numpy()
+    sub = {k: prob[k][:rows].float().cpu().numpy() for k in
+           ("target", "u_draft", "u_accept", "u_correct")}
+    t0 = time.perf_counter()
+    draft = oracle.round_bf16(oracle.lmhead_logits(h, w))
+    oracle.linear(draft, sub["target"], T, sub["u_draft"], sub["u_accept"], sub["u_correct"],
+                  min(K, rows // D), D)
+    return time.perf_counter() - t0
+
+
+def run_reference_lmhead(args):
+    """The oracle on the host cores for the LM-head workload: each step the LM
+    head and E/M step of one path (D rows) of one prefix."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2602_05774_gb300 import inputs
+    from oracle.build import build_oracle
+    build_oracle()
+    c = inputs.CONFIGS["lmhead"]
+    K, D, V, H = c["K"], c["D"], c["V"], c["H"]
+    small = inputs.lmhead_problem(1, K, D, V, H, device="cpu", seed=inputs.BASE_SEED + 99)
+    rows = D
+    for i in range(args.warmup):
+        oracle_lmhead_sample(small, rows, 1.0)
+    t = sum(oracle_lmhead_sample(small, rows, 1.0) for _ in range(args.steps))
+    ms = t / args.steps * 1e3
+    val = rows / (ms / 1e3)
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": val, "unit": "rows/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; same recipe)",
+        "config": {"workload": "lmhead", "B": c["B"], "K": K, "D": D, "V": V, "H": H,
+                   "sample_per_step": "1 path x %d rows of one prefix" % D},
+        "cpu_baseline": {"value": val, "unit": "rows/s", "cores": 1, "kind": "oracle",
+                         "sample": "%d rows per step (one path of one prefix)" % rows},
+        "e2e": {"value": val, "unit": "rows/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def run_lmhead(args):
+    """Config 5: the LM head on the tensor cores fused with the E/M step.  The
+    step is vsd_lmhead_estep_mstep; the roofline is the GEMM's (tensor), timed
+    on its own with CUDA events per launch."""
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2602_05774_gb300 import build, inputs, vsd
+    build.build_library()
+    vsd.load()
+    seed = inputs.BASE_SEED + list(inputs.CONFIGS).index("lmhead") + 1000 * rank
+    prob = inputs.config("lmhead", device=dev, seed=seed, B=args.prefixes or None)
+    B, K, D, V, H = prob["B"], prob["K"], prob["D"], prob["V"], prob["H"]
+    R = B * K * D
+    T = 1.0
+    prm = vsd.params(like=prob["target"])
+    ws = vsd.new_workspace(vsd.layout(B, K, D, V), dev)
+    out = vsd.linear_outputs(B, K, D, V, dev, grad_dtype=torch.bfloat16, full=True)
+    dl = torch.empty(R, V, dtype=torch.bfloat16, device=dev)
+
+    def step(i):
+        vsd.lmhead_estep_mstep(prob["hidden"], prob["weight"], prob["target"], prob["u_draft"],
+                               prob["u_accept"], prob["u_correct"], K, D, T, prm=prm,
+                               workspace=ws, out=out, draft_logits=dl)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    def timed(fn, n):
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(n)]
+        stream = torch.cuda.current_stream(dev)
+        barrier()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for i in range(n):
+            ev[i][0].record(stream)
+            fn(i)
+            ev[i][1].record(stream)
+        t1.record(stream)
+        barrier()
+        return t0.elapsed_time(t1), statistics.mean(a.elapsed_time(b) for a, b in ev)
+
+    for i in range(args.warmup):
+        step(i)
+    barrier()
+    if vsd.device_status(ws)[0] != 0:
+        raise RuntimeError("device status after warm-up: %s" % (vsd.device_status(ws),))
+    with ClockSampler(local) as clk:
+        total_ms, _ = timed(step, args.steps)
+        # the GEMM alone, per launch (the roofline's kernel)
+        gws = torch.zeros(256, dtype=torch.uint8, device=dev)
+        for _ in range(3):
+            vsd.lmhead_logits(prob["hidden"], prob["weight"], out=dl, workspace=gws)
+        _, gemm_ms = timed(lambda i: vsd.lmhead_logits(prob["hidden"], prob["weight"], out=dl,
+                                                       workspace=gws), args.steps)
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = tt.item()
+    ms = total_ms / args.steps
+    if vsd.device_status(ws)[0] != 0 or vsd.device_status(gws)[0] != 0:
+        raise RuntimeError("device status after timing")
+
+    e2e = None
+    if not args.no_e2e:  # the same step from pinned host buffers, loss read back
+        h_hidden = prob["hidden"].cpu().pin_memory()
+        h_target = prob["target"].cpu().pin_memory()
+        h_u = torch.stack([prob["u_draft"], prob["u_accept"], prob["u_correct"]]).cpu().pin_memory()
+        d_hidden = torch.empty_like(prob["hidden"])
+        d_target = torch.empty_like(prob["target"])
+        d_u = torch.empty(3, R, dtype=torch.float32, device=dev)
+        h_loss = torch.empty(B + 1, dtype=torch.float32).pin_memory()
+
+        def e2e_step(i):
+            d_hidden.copy_(h_hidden, non_blocking=True)
+            d_target.copy_(h_target, non_blocking=True)
+            d_u.copy_(h_u, non_blocking=True)
+            vsd.lmhead_estep_mstep(d_hidden, prob["weight"], d_target, d_u[0], d_u[1], d_u[2],
+                                   K, D, T, prm=prm, workspace=ws, out=out, draft_logits=dl)
+            h_loss.copy_(out["loss"], non_blocking=True)
+
+        e_steps = max(3, min(args.steps, 20))
+        for i in range(2):
+            e2e_step(i)
+        e_total, _ = timed(e2e_step, e_steps)
+        e_ms = e_total / e_steps
+        e2e = {"value": R * world / (e_ms / 1e3), "unit": "rows/s",
+               "h2d_bytes_per_step": (h_hidden.numel() * 2 + h_target.numel() * 2
+                                      + h_u.numel() * 4),
+               "d2h_bytes_per_step": h_loss.numel() * 4, "ms_per_step": e_ms,
+               "steps": e_steps, "weights": "resident on the device"}
+    if rank != 0:
+        return
+    peak, peak_kind = tensor_peak()
+    flops = 2.0 * R * V * H
+    achieved = flops / (gemm_ms / 1e3) / 1e12
+    line = {
+        "metric": METRIC, "value": R * world / (ms / 1e3), "unit": "rows/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; hidden ~N(0,1), LM-head weight ~N(0,0.02^2), spiked target)",
+        "config": {"workload": "lmhead", "B": B, "K": K, "D": D, "V": V, "H": H,
+                   "logits": "bf16", "grad": "bf16", "temperatures": [T],
+                   "l2": "inputs larger than L2 (no flush)", "rows_per_gpu": R},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
+                     "kernel": "k_lmhead", "flops_per_launch": flops, "launch_ms": gemm_ms},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clk.summary(),
+    }
+    if e2e is not None:
+        line["e2e"] = e2e
+    if world == 1 and not args.no_cpu_baseline:
+        rows = D
+        secs = oracle_lmhead_sample(prob, rows, T)
+        if secs < 8.0:  # about 12 s of oracle work, at most four prefixes
+            rows = D * min(4 * K, max(1, int(12.0 / max(secs, 1e-3))))
+            secs = oracle_lmhead_sample(prob, rows, T)
+        line["cpu_baseline"] = {"value": rows / secs, "unit": "rows/s", "cores": 1,
+                                "kind": "oracle", "seconds": secs,
+                                "sample": "the first %d rows (LM head in fp64 + E/M step)" % rows}
+    print(json.dumps(line), flush=True)
+
 def main():
     args = parse()
-    if args.impl == "reference":
+    if args.config == "lmhead":
+        run_reference_lmhead(args) if args.impl == "reference" else run_lmhead(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)
