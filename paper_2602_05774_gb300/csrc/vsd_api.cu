@@ -147,8 +147,12 @@ vsd_status check_params(const vsd_params& p) {
 // w(l) = w_base^l for l = 1 .. D, with the host's pow, and 1 / tau_car.
 template <typename T>
 void fill_wl(Problem<T>& P) {
-    for (int d = 0; d < 64; ++d) P.wl[d] = d < P.D ? pow(P.w_base, (double)(d + 1)) : 0.0;
+    for (int d = 0; d < 64; ++d) {
+        P.wl[d] = d < P.D ? pow(P.w_base, (double)(d + 1)) : 0.0;
+        P.wlf[d] = (float)P.wl[d];
+    }
     P.inv_tau = 1.0 / P.tau_car;
+    P.inv_tau_f = (float)P.inv_tau;
 }
 
 template <typename T>

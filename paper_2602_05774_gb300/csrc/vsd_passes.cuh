@@ -106,7 +106,9 @@ struct Problem {
     const int32_t* parent;        // tree [B][N]
     double w_base, tau_car;
     double wl[64];  // w(l) = w_base^l for l = 1 .. D (App. F), computed on the host
+    float wlf[64];  // the same in float
     double inv_tau;  // 1 / tau_car
+    float inv_tau_f;
     int zeta_mode;
     int grad_bf16;
     int inject_wait_fault;
@@ -412,6 +414,40 @@ __device__ __forceinline__ long long warp_incl_scan_ll(long long v, int lane) {
     return v;
 }
 
+// Whether t sc 2^E <= num exactly, for finite t, sc >= 0 and num >= 0 (integer
+// arithmetic on the two 24-bit significands).
+__device__ __forceinline__ bool prod_le(float t, float sc, int E, long long num) {
+    if (!(t > 0.f) || !(sc > 0.f)) return true;
+    const unsigned bt = __float_as_uint(t), bc = __float_as_uint(sc);
+    const int xt = (bt >> 23) & 0xFF, xc = (bc >> 23) & 0xFF;
+    const unsigned long long mt = xt ? ((bt & 0x7FFFFFu) | 0x800000u) : (bt & 0x7FFFFFu);
+    const unsigned long long mc = xc ? ((bc & 0x7FFFFFu) | 0x800000u) : (bc & 0x7FFFFFu);
+    const unsigned long long pm = mt * mc;  // t sc 2^E = pm 2^sh
+    const int sh = (xt ? xt : 1) + (xc ? xc : 1) - 300 + E;
+    const unsigned long long n = (unsigned long long)num;
+    if (sh >= 0) return sh < 64 && pm <= (n >> sh);
+    const int k = -sh;
+    if (k >= 64) return n >= 1;
+    const unsigned long long q = pm >> k, r = pm & ((1ull << k) - 1ull);
+    return q < n || (q == n && r == 0);
+}
+
+// The largest float t >= 0 with t sc <= num 2^-E (num >= 0, sc > 0): a float
+// estimate, then exact tests one float step at a time.
+__device__ __forceinline__ float fixed_quotient_rd(long long num, float sc, int E) {
+    const float nf = (float)(int)(num >> 32) * 4294967296.f + (float)(unsigned)(num & 0xFFFFFFFFull);
+    float t = ldexpf(nf, -E) / sc;
+    if (!(t >= 0.f)) t = 0.f;
+    if (t > 3.0e38f) t = 3.0e38f;
+    for (int i = 0; i < 16 && !prod_le(t, sc, E, num); ++i) t = nextafterf(t, 0.f);
+    for (int i = 0; i < 16; ++i) {
+        const float up = nextafterf(t, INFINITY);
+        if (!prod_le(up, sc, E, num)) break;
+        t = up;
+    }
+    return t;
+}
+
 // A table total: Z = Zi 2^-E (NaN if a weight is not finite).
 struct TableSum {
     long long Zi;
@@ -475,9 +511,9 @@ __device__ __forceinline__ Located table_locate(const float4* tab, int nch, int 
             const int L = __ffs(hit) - 1;
             const long long before = __shfl_sync(0xffffffffu, base + inc - w, L);
             const float scL = __shfl_sync(0xffffffffu, sc, L);
-            // ti - before < w_L < 2^52: exact in double, as is the scaling
-            const double rem = (double)(ti - before) * pow2_neg(S.E);
-            return Located{g + L, __double2float_rd(__ddiv_rd(rem, (double)scL))};
+            // the threshold in the chunk's frame, (ti - before) 2^-E / sc,
+            // rounded down to a float
+            return Located{g + L, fixed_quotient_rd(ti - before, scL, S.E)};
         }
         if (pos) last = g + 31 - __clz(pos);
         base += __shfl_sync(0xffffffffu, inc, 31);
@@ -1205,22 +1241,54 @@ __device__ void path_pass(const Problem<T>& P, int path, Ring* rg, float4* tab, 
 // wherever the arithmetic allows, because double-precision latency, not
 // work, bounds a single warp here.
 constexpr int kMTile = 256;
+constexpr int kLqE = 32;  // fixed-point scale 2^-32 of the M-step's sums
 struct WeightsShared {
-    double lqt[256], lqc[256];  // per proposal: running sums of log q (z~, z') over l
+    // per proposal: running sums over l of log q(z~) and log q(z') (fixed point)
+    long long lqt[256], lqc[256];
     // the tile: entry e = s * nd + (l - l0)
-    float lq[kMTile];    // log q(z~); then 2^{c_q - max} (CAR)
+    float lq[kMTile];    // log q(z~); then the CAR weight
     float lqcz[kMTile];  // log q(z')
     unsigned char ot[kMTile], pc[kMTile];  // o~, and whether z' passes
     int tok[kMTile], corr[kMTile];
-    double elqt[kMTile];  // running sum of log q(z~) at the entry
-    double elqc[kMTile];  // running sum of log q(z'); then the term o'(1 - o~)
-    double ecq[kMTile];   // CAR logit; then the term o'(o~ - beta zeta)
+    long long elqt[kMTile];  // running sum of log q(z~) at the entry
+    long long elqc[kMTile];  // running sum of log q(z'); then the term o'(1 - o~)
+    long long et0[kMTile];   // the term o'(o~ - beta zeta)
     // per position of the tile
-    int n1[64], n0[64];  // proposals with o' != 0 and o~ = 1, with o' != 0
-    long long zs[64];    // sum of the CAR weights (fixed point, 2^-40)
-    float rz[64];        // 1 / that sum
-    float beta[64][3];   // leave-one-out beta for (o', o~) = (w, 1), (w, 0), (0, 0)
+    int n1[64], n0[64];          // proposals with o' != 0 and o~ = 1, with o' != 0
+    long long lmax[64];          // max over proposals of the running log q(z~)
+    unsigned long long zs[64];   // sum of the CAR weights (fixed point, 2^-40)
+    float rz[64];                // 1 / that sum
+    float beta[64][3];           // leave-one-out beta for (o', o~) = (w, 1), (w, 0), (0, 0)
+    float cmax[64];              // zeta_mode 0: exp(lmax) / tau
 };
+
+// x 2^E rounded toward zero, |x| clamped to 2^20 (a non-finite log-probability
+// of an invalid row becomes -2^20); exact for |x| >= 2^(23-E).
+__device__ __forceinline__ long long to_fixed(float x, int E) {
+    float a = fabsf(x);
+    if (!(a <= 1048576.f)) a = 1048576.f;
+    const long long m = fixed_prod(a, 1.f, E);
+    return (x < 0.f || x != x) ? -m : m;
+}
+// q 2^-E as a float (two 32-bit conversions: relative error below 2^-23).
+__device__ __forceinline__ float from_fixed(long long q, int E) {
+    const float hi = (float)(int)(q >> 32) * 4294967296.f;
+    const float lo = (float)(unsigned)(q & 0xFFFFFFFFull);
+    return ldexpf(hi + lo, -E);
+}
+
+// f(e) for the entries e = lane, lane + 32, ... < ne, four at a time so that
+// their independent loads and double-precision chains overlap.
+template <class F>
+__device__ __forceinline__ void each_entry(int ne, int lane, F&& f) {
+    for (int e0 = lane; e0 < ne; e0 += 128) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int e = e0 + 32 * u;
+            if (e < ne) f(e);
+        }
+    }
+}
 
 // Load the tile of positions [d0, d0 + nd) of prefix b (warp).  TERMS: the
 // per-entry terms written by the forward sweep (from wscr) instead of the
@@ -1229,14 +1297,14 @@ template <typename T, bool TERMS>
 __device__ __forceinline__ void mstep_tile(const Problem<T>& P, const EStepView& E, int b, int d0,
                                            int nd, WeightsShared& sh, int lane) {
     const int K = P.K, D = P.D;
-    for (int e = lane; e < K * nd; e += 32) {
+    each_entry(K * nd, lane, [&](int e) {
         const int s = e / nd, r = (b * K + s) * D + d0 + (e - s * nd);
         sh.tok[e] = ld_cg(E.tok + r);
         sh.corr[e] = ld_cg(E.corr + r);
         if (TERMS) {
             const double2 tm = ld_cg(P.wscr + r);
-            sh.ecq[e] = tm.x;
-            sh.elqc[e] = tm.y;
+            sh.et0[e] = to_fixed((float)tm.x, kLqE);
+            sh.elqc[e] = to_fixed((float)tm.y, kLqE);
         } else {
             const float lkr = ld_cg(E.lkr + r);
             sh.ot[e] = ld_cg(E.lk + r) >= lkr ? 1 : 0;
@@ -1244,120 +1312,127 @@ __device__ __forceinline__ void mstep_tile(const Problem<T>& P, const EStepView&
             sh.lq[e] = ld_cg(E.lq_tok + r);
             sh.lqcz[e] = ld_cg(E.lq_corr + r);
         }
-    }
+    });
     __syncwarp();
 }
 
 // M-step of prefix b by one warp (K <= 256, D <= 64).  Writes coef[] for the
-// prefix's rows, the optional weights table and loss_out[b].  Arithmetic in
-// double except the CAR weights (float exponentials of double differences);
-// every sum over proposals is either an exact integer sum or taken in a fixed
-// order, so the result does not depend on timing.
+// prefix's rows, the optional weights table and loss_out[b].  No dependent
+// double-precision chains (GB300's FP64 latency would dominate): sums over l
+// and over entries are exact 64-bit fixed-point sums of float terms, the CAR
+// weights come from exact differences of those sums, and every reduction is
+// exact, so the result does not depend on the order of the entries.
 template <typename T>
 __device__ void weights_warp(const Problem<T>& P, const EStepView& E, int b, float* weights_out,
                              float* loss_out, WeightsShared& sh, int lane) {
     const int K = P.K, D = P.D;
     const int dt = max(1, min(D, kMTile / K));
     const bool one_tile = dt >= D;
-    for (int s = lane; s < K; s += 32) sh.lqt[s] = sh.lqc[s] = 0.0;
-    double Jp = 0.0, Np = 0.0;  // this lane's parts of J and N
+    const float inv_tau = P.inv_tau_f;
+    for (int s = lane; s < K; s += 32) sh.lqt[s] = sh.lqc[s] = 0;
+    long long Jq = 0, Nq = 0;  // this lane's parts of J and N (fixed point, 2^-24)
     for (int d0 = 0; d0 < D; d0 += dt) {
         const int nd = min(dt, D - d0);
         const int ne = K * nd;
         mstep_tile<T, false>(P, E, b, d0, nd, sh, lane);
         // running sums of log q over l, per proposal
         for (int s = lane; s < K; s += 32) {
-            double a = sh.lqt[s], q = sh.lqc[s];
+            long long a = sh.lqt[s], q = sh.lqc[s];
             for (int dd = 0; dd < nd; ++dd) {
                 const int e = s * nd + dd;
-                a += (double)sh.lq[e];
-                q += (double)sh.lqcz[e];
+                a += to_fixed(sh.lq[e], kLqE);
+                q += to_fixed(sh.lqcz[e], kLqE);
                 sh.elqt[e] = a;
                 sh.elqc[e] = q;
             }
             sh.lqt[s] = a;
             sh.lqc[s] = q;
         }
-        __syncwarp();
-        // CAR logits (Eq. zeta): on q(z~_{1:l}) or on its log
-        for (int e = lane; e < ne; e += 32)
-            sh.ecq[e] = (P.zeta_mode == 0 ? exp(sh.elqt[e]) : sh.elqt[e]) * P.inv_tau;
-        __syncwarp();
-        // per position: the counts behind beta, and the CAR weights and their sum
-        for (int dd = 0; dd < nd; ++dd) {
-            int c1 = 0, c0 = 0;
-            float mf = -INFINITY;
-            for (int s = lane; s < K; s += 32) {
-                const int e = s * nd + dd;
-                // Algorithm 2 scores z~ (o~); Algorithm 1 keeps z~ if it
-                // passes, else z', so o' = w(l) when either passes
-                const bool ot = sh.ot[e], op = ot || sh.pc[e];
-                c1 += (op && ot) ? 1 : 0;
-                c0 += op ? 1 : 0;
-                mf = fmaxf(mf, (float)sh.ecq[e]);
-            }
-#pragma unroll
-            for (int o = 16; o; o >>= 1) {
-                c1 += __shfl_xor_sync(0xffffffffu, c1, o);
-                c0 += __shfl_xor_sync(0xffffffffu, c0, o);
-                mf = fmaxf(mf, __shfl_xor_sync(0xffffffffu, mf, o));
-            }
-            long long za = 0;  // the CAR weights are at most about 1: exact sum at 2^-40
-            for (int s = lane; s < K; s += 32) {
-                const int e = s * nd + dd;
-                const float ez = expf((float)(sh.ecq[e] - (double)mf));
-                sh.lq[e] = ez;
-                za += fixed_prod(ez, 1.f, 40);
-            }
-            za = warp_sum_ll(za);
-            if (lane == 0) {
-                sh.n1[dd] = c1;
-                sh.n0[dd] = c0;
-                sh.zs[dd] = za;
-            }
+        for (int dd = lane; dd < nd; dd += 32) {
+            sh.n1[dd] = sh.n0[dd] = 0;
+            sh.lmax[dd] = (long long)0x8000000000000000ull;
+            sh.zs[dd] = 0;
         }
+        __syncwarp();
+        // per position: the counts behind beta and the largest running log q,
+        // gathered from every entry at once with shared-memory integer atomics
+        each_entry(ne, lane, [&](int e) {
+            const int dd = e % nd;
+            // Algorithm 2 scores z~ (o~); Algorithm 1 keeps z~ if it passes,
+            // else z', so o' = w(l) when either passes
+            const bool ot = sh.ot[e], op = ot || sh.pc[e];
+            if (op) {
+                atomicAdd(&sh.n0[dd], 1);
+                if (ot) atomicAdd(&sh.n1[dd], 1);
+            }
+            atomicMax(&sh.lmax[dd], sh.elqt[e]);
+        });
+        __syncwarp();
+        if (P.zeta_mode == 0)  // exp(lmax) / tau, with the float split hi + lo of lmax
+            for (int dd = lane; dd < nd; dd += 32) {
+                const long long m = sh.lmax[dd];
+                const float hi = from_fixed(m, kLqE);
+                const float lo = from_fixed(m - to_fixed(hi, kLqE), kLqE);
+                sh.cmax[dd] = expf(hi) * (1.f + lo) * inv_tau;
+            }
+        __syncwarp();
+        // CAR weights (Eq. zeta) relative to the proposal with the largest
+        // logit: exp((Q_s - Q_max) / tau) with Q = q(z~_{1:l}) (zeta_mode 0:
+        // Q_s - Q_max = Q_max expm1(d)) or Q = log q(z~_{1:l}) (zeta_mode 1:
+        // Q_s - Q_max = d), d = the exact difference of the running sums
+        each_entry(ne, lane, [&](int e) {
+            const int dd = e % nd;
+            const float d = from_fixed(sh.elqt[e] - sh.lmax[dd], kLqE);
+            const float arg = P.zeta_mode == 0 ? sh.cmax[dd] * expm1f(d) : d * inv_tau;
+            const float ez = expf(arg);
+            sh.lq[e] = ez;
+            // at most 1: exact sum at 2^-40
+            const long long z = fixed_prod(ez, 1.f, 40);
+            if (z) atomicAdd(&sh.zs[dd], (unsigned long long)z);
+        });
         __syncwarp();
         // per position, in parallel: 1 / sum, and beta (Eq. beta, leave-one-out:
         // o' is w(l) or 0, so both of its sums are w(l) times a count)
         for (int dd = lane; dd < nd; dd += 32) {
             const int n1 = sh.n1[dd], n0 = sh.n0[dd];
-            const float zs = (float)sh.zs[dd] * 0x1p-40f;
+            const float zs = (float)(long long)sh.zs[dd] * 0x1p-40f;
             sh.rz[dd] = zs > 0.f ? 1.f / zs : 0.f;
             sh.beta[dd][0] = n0 - 1 > 0 ? (float)(n1 - 1) / (float)(n0 - 1) : 0.f;
             sh.beta[dd][1] = n0 - 1 > 0 ? (float)n1 / (float)(n0 - 1) : 0.f;
             sh.beta[dd][2] = n0 > 0 ? (float)n1 / (float)n0 : 0.f;
-            Np += P.wl[d0 + dd] * (double)n0;
         }
         __syncwarp();
         // per entry, in parallel: zeta, the objective terms (Eq. advance) and
         // the per-l gradient terms o'(o~ - beta zeta), o'(1 - o~)
-        for (int e = lane; e < ne; e += 32) {
+        each_entry(ne, lane, [&](int e) {
             const int s = e / nd, dd = e - s * nd, d = d0 + dd;
             const bool otb = sh.ot[e], opb = otb || sh.pc[e];
-            const double w = P.wl[d];
-            const float betaf = sh.beta[dd][opb ? (otb ? 0 : 1) : 2];
-            const float zetaf = sh.lq[e] * sh.rz[dd];
-            const double beta = betaf, zeta = zetaf;
-            const double lqt = sh.elqt[e];
-            const double lqz = otb ? lqt : sh.elqc[e];
-            if (opb) Jp += w * (lqz - beta * zeta * lqt);
-            const double t0 = opb ? w * ((otb ? 1.0 : 0.0) - beta * zeta) : 0.0;
-            const double t1 = (opb && !otb) ? w : 0.0;
-            sh.ecq[e] = t0;
-            sh.elqc[e] = t1;
+            const float w = P.wlf[d];
+            const float beta = sh.beta[dd][opb ? (otb ? 0 : 1) : 2];
+            const float zeta = sh.lq[e] * sh.rz[dd];
+            if (opb) {
+                const float lqt = from_fixed(sh.elqt[e], kLqE);
+                const float lqz = otb ? lqt : from_fixed(sh.elqc[e], kLqE);
+                Jq += to_fixed(w * (lqz - beta * zeta * lqt), 24);
+                Nq += to_fixed(w, 24);
+            }
+            const float t0 = opb ? w * ((otb ? 1.f : 0.f) - beta * zeta) : 0.f;
+            const float t1 = (opb && !otb) ? w : 0.f;
+            sh.et0[e] = to_fixed(t0, kLqE);
+            sh.elqc[e] = to_fixed(t1, kLqE);
             const int r = (b * K + s) * D + d;
             if (!one_tile) P.wscr[r] = make_double2(t0, t1);
             if (weights_out) {
                 float4* wo = reinterpret_cast<float4*>(weights_out) + ((int64_t)b * D + d) * K + s;
-                *wo = make_float4(otb ? 1.f : 0.f, opb ? (float)w : 0.f, betaf, zetaf);
+                *wo = make_float4(otb ? 1.f : 0.f, opb ? w : 0.f, beta, zeta);
             }
-        }
+        });
         __syncwarp();
     }
-    const double J = warp_sum(Jp), N = warp_sum(Np);
-    const double scale = N > 0.0 ? 1.0 / ((double)P.B * N * P.ts.Td) : 0.0;
+    const float J = from_fixed(warp_sum_ll(Jq), 24), N = from_fixed(warp_sum_ll(Nq), 24);
+    const float scale = N > 0.f ? 1.f / ((float)P.B * N * P.ts.T) : 0.f;
     // suffix sums over l, from the last tile back (lqt, lqc now hold c0, c1)
-    for (int s = lane; s < K; s += 32) sh.lqt[s] = sh.lqc[s] = 0.0;
+    for (int s = lane; s < K; s += 32) sh.lqt[s] = sh.lqc[s] = 0;
     for (int d0 = ((D - 1) / dt) * dt; d0 >= 0; d0 -= dt) {
         const int nd = min(dt, D - d0);
         if (!one_tile) {
@@ -1365,19 +1440,24 @@ __device__ void weights_warp(const Problem<T>& P, const EStepView& E, int b, flo
             mstep_tile<T, true>(P, E, b, d0, nd, sh, lane);
         }
         for (int s = lane; s < K; s += 32) {
-            double c0 = sh.lqt[s], c1 = sh.lqc[s];
+            long long c0 = sh.lqt[s], c1 = sh.lqc[s];
             for (int dd = nd - 1; dd >= 0; --dd) {
                 const int e = s * nd + dd;
-                c0 += sh.ecq[e];
+                c0 += sh.et0[e];
                 c1 += sh.elqc[e];
                 Coef cf;
                 cf.t0 = sh.tok[e];
                 cf.t1 = sh.corr[e];
-                double k0 = c0 * scale, k1 = c1 * scale;
-                if (cf.t1 == cf.t0) { k0 += k1; k1 = 0.0; cf.t1 = -1; }
-                cf.g = (float)((c0 + c1) * scale);
-                cf.c0 = (float)k0;
-                cf.c1 = (float)k1;
+                const float g = from_fixed(c0 + c1, kLqE) * scale;
+                if (cf.t1 == cf.t0) {
+                    cf.c0 = g;
+                    cf.c1 = 0.f;
+                    cf.t1 = -1;
+                } else {
+                    cf.c0 = from_fixed(c0, kLqE) * scale;
+                    cf.c1 = from_fixed(c1, kLqE) * scale;
+                }
+                cf.g = g;
                 cf.pad0 = cf.pad1 = cf.pad2 = 0.f;
                 P.coef[(b * K + s) * D + d0 + dd] = cf;
             }
@@ -1385,7 +1465,7 @@ __device__ void weights_warp(const Problem<T>& P, const EStepView& E, int b, flo
             sh.lqc[s] = c1;
         }
     }
-    if (lane == 0) loss_out[b] = (float)(N > 0.0 ? -J / N : 0.0);
+    if (lane == 0) loss_out[b] = N > 0.f ? -J / N : 0.f;
 }
 
 // The M-step by a block: warp 0 runs weights_warp (the same bits as the fused
