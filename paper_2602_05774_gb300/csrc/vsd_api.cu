@@ -205,6 +205,10 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.row_seg_cnt = at<int>(ws, w.row_seg_cnt);
     P.res_seg_cnt = at<int>(ws, w.res_seg_cnt);
     P.path_A = at<int>(ws, w.path_A);
+    // the tree layout has no E-step view and no path lengths: their arrays
+    // hold its residual lists
+    P.tlist = at<int>(ws, w.es_tok);
+    P.tcount = at<int>(ws, w.path_A);
     P.resq = at<int>(ws, w.resq);
     P.resq_flag = at<int>(ws, w.resq_flag);
     P.resq_head = at<int>(ws, w.resq_head);

@@ -62,14 +62,29 @@ __global__ void __launch_bounds__(kThreads) k_paths(Problem<T> P) {
     path_pass<T, VEC>(P, blockIdx.x, rg, tab, sh);
 }
 
-template <typename T, bool VEC>
+template <typename T>
 __global__ void __launch_bounds__(kThreads) k_tree(Problem<T> P) {
-    extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ TreeShared sh;
+    tree_nodes<T>(P, blockIdx.x, sh);
+}
+
+// kTreeBlocks blocks per tree share its residual rows.
+constexpr int kTreeBlocks = 4;
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kThreads) k_tree_residuals(Problem<T> P) {
+    extern __shared__ __align__(128) unsigned char dsm[];
+    __shared__ int s_tok;
     Ring* rg;
     float4* tab;
     smem_views<VEC>(dsm, rg, tab);
-    tree_pass<T, VEC>(P, blockIdx.x, rg, tab, sh);
+    tree_residuals<T, VEC>(P, blockIdx.x / kTreeBlocks, blockIdx.x % kTreeBlocks, kTreeBlocks, rg,
+                           tab, &s_tok);
+}
+
+template <typename T>
+__global__ void k_tree_bonus(Problem<T> P) {
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b < P.B) tree_bonus<T>(P, b);
 }
 
 template <typename T>
@@ -487,16 +502,25 @@ cudaError_t Launch<VSD_T>::paths(const Problem<VSD_T>& P, bool vec, cudaStream_t
 
 template <>
 cudaError_t Launch<VSD_T>::tree(const Problem<VSD_T>& P, bool vec, cudaStream_t s) {
+    // per node (one block per tree), then the residual rows (kTreeBlocks per
+    // tree), then the bonus tokens
+    k_tree<VSD_T><<<P.B, kThreads, 0, s>>>(P);
+    cudaError_t e = cudaGetLastError();
+    if (e) return e;
     const size_t smem = stream_smem_bytes(P.nch, vec);
+    const int grid = P.B * kTreeBlocks;
     if (vec) {
-        cudaError_t e = prep(k_tree<VSD_T, true>, smem);
+        e = prep(k_tree_residuals<VSD_T, true>, smem);
         if (e) return e;
-        k_tree<VSD_T, true><<<P.B, kThreads, smem, s>>>(P);
+        k_tree_residuals<VSD_T, true><<<grid, kThreads, smem, s>>>(P);
     } else {
-        cudaError_t e = prep(k_tree<VSD_T, false>, smem);
+        e = prep(k_tree_residuals<VSD_T, false>, smem);
         if (e) return e;
-        k_tree<VSD_T, false><<<P.B, kThreads, smem, s>>>(P);
+        k_tree_residuals<VSD_T, false><<<grid, kThreads, smem, s>>>(P);
     }
+    e = cudaGetLastError();
+    if (e) return e;
+    k_tree_bonus<VSD_T><<<(P.B + 127) / 128, 128, 0, s>>>(P);
     return cudaGetLastError();
 }
 

@@ -19,9 +19,10 @@
 //                the per-row gradient coefficients.
 //   grad_pass    one streaming read of a draft row and write of its gradient:
 //                grad[v] = g q(v) - c0 [v = t0] - c1 [v = t1].
-//   tree_pass    per draft tree: acceptance per node at its parent's row, the
-//                AND-scan along parent pointers, log kappa, residual draws at
-//                the parents of first-rejected nodes, deepest node, bonus.
+//   tree_nodes / tree_residuals / tree_bonus   per draft tree: acceptance per
+//                node at its parent's row, the AND-scan along parent pointers,
+//                log kappa, the deepest node; residual draws at the parents of
+//                rejected nodes (several blocks per tree); the bonus token.
 #pragma once
 
 #include "vsd_common.cuh"
@@ -134,6 +135,8 @@ struct Problem {
     int* row_seg_cnt;             // [R] segments of a row completed
     int* res_seg_cnt;             // [B*K] residual segments of a path completed
     int* path_A;                  // [B*K] accepted length of a path
+    int* tlist;                   // tree layout: [R] residual rows of each tree (its rows' slots)
+    int* tcount;                  // tree layout: [B] length of each tree's list
     int* resq;                    // [B*K*nseg] residual segment items (path*nseg + seg)
     int* resq_flag;               // [B*K*nseg] item written
     int* resq_head;               // next item to take
@@ -243,10 +246,11 @@ __device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, in
     };
     const int nrange = ch1 - ch0;
     const int nj = nrange > warp ? (nrange - warp + kWarps - 1) / kWarps : 0;
+    const int cfirst = ch0 + warp, cstride = kWarps;
     const int pos = *posp;
     bool broken = rg->broken[warp] != 0;
     auto issue = [&](int j) {
-        const int ch = ch0 + warp + j * kWarps;
+        const int ch = cfirst + j * cstride;
         const int slot = (pos + j) % NS;
         const int64_t e0 = (int64_t)ch * CE;
         const int64_t ne = V - e0 < CE ? V - e0 : CE;
@@ -264,7 +268,7 @@ __device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, in
         const uint32_t parity = (uint32_t)((pos + j) / NS) & 1u;
         bool ok = broken ? false : ring_wait(&bars[slot], parity, status);
         broken = __any_sync(0xffffffffu, !ok);
-        const int ch = ch0 + warp + j * kWarps;
+        const int ch = cfirst + j * cstride;
         const int64_t e0 = (int64_t)ch * CE;
         const uint4* sx = xbuf(slot);
         uint4 bx[kLoads], by[kLoads];
@@ -1054,30 +1058,6 @@ __device__ int residual_draw(const Problem<T>& P, int r, const RowRec& rec, floa
     return tok;
 }
 
-// Inverse-CDF draw from p at row r with uniform u (block; streams the target row).
-template <typename T, bool VEC>
-__device__ int p_draw(const Problem<T>& P, int r, float u, Ring* rg, float4* tab, int* out) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t V = P.V;
-    const T* y = P.target + (int64_t)r * V;
-    const float c = P.ts.c;
-    const uint64_t pol = policy_evict_normal();
-    stream_tables<T, VEC, false>(rg, y, nullptr, V, 0, P.nch, tab, c, pol, pol, P.status);
-    __syncthreads();
-    if (warp == 0) {
-        const float M = table_max(tab, P.nch, 0, lane);
-        const TableSum Z = table_sum(tab, P.nch, 0, frame_of(M), c, lane);
-        const int tok = row_ok(M, Z.Z) ? warp_sample<T, VEC>(y, nullptr, V, tab, P.nch, 0, M, Z, u,
-                                                          c, lane, pol)
-                                     : -1;
-        if (lane == 0) *out = tok < V ? tok : -1;
-    }
-    __syncthreads();
-    const int tok = *out;
-    __syncthreads();
-    return tok;
-}
-
 // --------------------------------------------------------------- path pass
 struct PathShared {
     int A;
@@ -1642,24 +1622,30 @@ __device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* g
 
 // --------------------------------------------------------------- tree pass
 struct TreeShared {
-    int bad, deepest, bonus, resid;
-    double rt;
-    RowRec rec;
-    unsigned char pacc[1024];
+    int bad, deepest, maxdepth;
+    unsigned char acc[1024], pacc[1024], hasrej[1024];
     int depth[1024];
+    float la[1024];
     double lk[1024];
 };
 
-// One draft tree per block; rows of tree b are b*N .. b*N + N - 1, row n is
-// the distribution node n's children were drafted from (App. E tree).
-template <typename T, bool VEC>
-__device__ void tree_pass(const Problem<T>& P, int b, Ring* rg, float4* tab, TreeShared& sh) {
+// Tree verification, one draft tree b of N nodes per block; rows of tree b
+// are b*N .. b*N + N - 1, row n is the distribution node n's children were
+// drafted from (App. E tree).  This pass:
+//   1. every node, in parallel: alpha and the accept bit of its token against
+//      its parent's row (Eq. 1);
+//   2. in node order (parents come first): the accepted-path bit and the
+//      depth; then log kappa level by level (each node adds its log alpha to
+//      its parent's); the deepest accepted node;
+//   3. the list of residual rows (accepted nodes with a rejected child) for
+//      tree_residuals, in tlist[b*N ..], its length in tcount[b].
+template <typename T>
+__device__ void tree_nodes(const Problem<T>& P, int b, TreeShared& sh) {
     const int N = P.N;
     const int64_t V = P.V;
     const int n0 = b * N;
     const int32_t* par = P.parent + (int64_t)n0;
     const vsd_tree_outputs& o = P.tout;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
         int bad = (__ldg(par) != -1);
         for (int n = 1; n < N && !bad; ++n) {
@@ -1681,103 +1667,170 @@ __device__ void tree_pass(const Problem<T>& P, int b, Ring* rg, float4* tab, Tre
             o.logkappa[n0 + n] = -INFINITY;
             o.corr_tokens[n0 + n] = -1;
         }
-        if (threadIdx.x == 0) { o.deepest[b] = -1; o.accept_len[b] = -1; o.bonus[b] = -1; }
+        if (threadIdx.x == 0) {
+            o.deepest[b] = -1;
+            o.accept_len[b] = -1;
+            o.bonus[b] = -1;
+            P.tcount[b] = 0;
+        }
         return;
     }
-    if (threadIdx.x == 0) {
-        o.alpha[n0] = 1.f; o.accept[n0] = 1; o.path_accept[n0] = 1; o.logkappa[n0] = 0.f;
-        o.corr_tokens[n0] = -1;
-        sh.pacc[0] = 1;
-        sh.depth[0] = 0;
-        double* lk = sh.lk;
-        lk[0] = 0.0;
-        int deepest = 0;
-        for (int n = 1; n < N; ++n) {
+    // 1. per node
+    for (int n = threadIdx.x; n < N; n += kThreads) {
+        float la = 0.f;
+        bool acc = true;
+        if (n > 0) {
             const int pn = __ldg(par + n);
             const RowRec rec = ld_cg(P.rows + n0 + pn);
             const int tok = __ldg(P.given_tokens + n0 + n);
-            double la = -INFINITY;
+            la = -INFINITY;
             if (tok < 0 || tok >= V) {
                 atomicOr(P.status, VSD_STATUS_BAD_TOKEN);
             } else if (!rec.flags) {
-                float lq, laf;
+                float lq;
                 token_logs(P.draft + (int64_t)(n0 + pn) * V, P.target + (int64_t)(n0 + pn) * V,
-                           tok, rec, P.ts.invTd, &lq, &laf);
-                la = (double)laf;
+                           tok, rec, P.ts.invTd, &lq, &la);
             }
-            const double a = exp(la);
-            const bool acc = la > -INFINITY && (double)__ldg(P.u_accept + n0 + n) <= a;
-            sh.pacc[n] = (unsigned char)(acc && sh.pacc[pn]);
-            sh.depth[n] = sh.depth[pn] + 1;
-            lk[n] = lk[pn] + la;
-            o.alpha[n0 + n] = (float)a;
+            const float a = expf(la);
+            acc = la > -INFINITY && __ldg(P.u_accept + n0 + n) <= a;
+            o.alpha[n0 + n] = a;
             o.accept[n0 + n] = acc ? 1 : 0;
-            o.path_accept[n0 + n] = sh.pacc[n];
-            o.logkappa[n0 + n] = (float)lk[n];
-            o.corr_tokens[n0 + n] = -1;
+        }
+        sh.la[n] = la;
+        sh.acc[n] = acc ? 1 : 0;
+        sh.hasrej[n] = 0;
+    }
+    __syncthreads();
+    // 2. accepted-path bits, depths, the deepest accepted node
+    if (threadIdx.x == 0) {
+        sh.pacc[0] = 1;
+        sh.depth[0] = 0;
+        sh.lk[0] = 0.0;
+        int deepest = 0, maxd = 0;
+        for (int n = 1; n < N; ++n) {
+            const int pn = __ldg(par + n);
+            sh.pacc[n] = (unsigned char)(sh.acc[n] && sh.pacc[pn]);
+            sh.depth[n] = sh.depth[pn] + 1;
+            maxd = max(maxd, sh.depth[n]);
             if (sh.pacc[n] && sh.depth[n] > sh.depth[deepest]) deepest = n;
         }
         sh.deepest = deepest;
+        sh.maxdepth = maxd;
+        o.alpha[n0] = 1.f;
+        o.accept[n0] = 1;
+        o.path_accept[n0] = 1;
+        o.logkappa[n0] = 0.f;
+        o.corr_tokens[n0] = -1;
+        o.deepest[b] = deepest;
+        o.accept_len[b] = sh.depth[deepest];
     }
     __syncthreads();
-    // Residual draws (Sec. 3): every node on an accepted path whose children
-    // include rejected ones streams its row once; each rejected child then
-    // draws with its own uniform.
-    for (int u = 0; u < N; ++u) {
-        if (!sh.pacc[u]) continue;
-        int first = -1;
-        for (int n = u + 1; n < N; ++n)
-            if (__ldg(par + n) == u && !sh.pacc[n]) { first = n; break; }
-        if (first < 0) continue;
-        if (threadIdx.x == 0) sh.rec = ld_cg(P.rows + n0 + u);
+    for (int L = 1; L <= sh.maxdepth; ++L) {  // log kappa along each branch (Eq. 2)
+        for (int n = threadIdx.x; n < N; n += kThreads)
+            if (sh.depth[n] == L) sh.lk[n] = sh.lk[__ldg(par + n)] + (double)sh.la[n];
         __syncthreads();
-        if (sh.rec.flags) { __syncthreads(); continue; }
+    }
+    for (int n = 1 + threadIdx.x; n < N; n += kThreads) {
+        o.path_accept[n0 + n] = sh.pacc[n];
+        o.logkappa[n0 + n] = (float)sh.lk[n];
+        o.corr_tokens[n0 + n] = -1;
+        const int pn = __ldg(par + n);
+        if (sh.pacc[pn] && !sh.pacc[n]) sh.hasrej[pn] = 1;
+    }
+    __syncthreads();
+    // 3. the residual rows, in node order
+    if (threadIdx.x == 0) {
+        int k = 0;
+        for (int u = 0; u < N; ++u)
+            if (sh.pacc[u] && sh.hasrej[u]) P.tlist[n0 + k++] = u;
+        P.tcount[b] = k;
+    }
+}
+
+// Residual rows of tree b, items g, g + G, ... of its list (block): stream
+// the row's residual max(0, p - q) (Sec. 3) and draw each rejected child's
+// token with the child's own uniform; if the residual has no mass, a draw
+// from p instead (reading R10).
+template <typename T, bool VEC>
+__device__ void tree_residuals(const Problem<T>& P, int b, int g, int G, Ring* rg, float4* tab,
+                               int* s_tok) {
+    const int N = P.N;
+    const int64_t V = P.V;
+    const int n0 = b * N;
+    const int nch = P.nch;
+    const int32_t* par = P.parent + (int64_t)n0;
+    const vsd_tree_outputs& o = P.tout;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const float c = P.ts.c;
+    const uint64_t pol = policy_evict_normal();
+    const int cnt = ld_cg(P.tcount + b);
+    for (int i = g; i < cnt; i += G) {
+        const int u = ld_cg(P.tlist + n0 + i);
         const int r = n0 + u;
+        const RowRec rec = ld_cg(P.rows + r);
+        if (rec.flags) continue;
         const T* x = P.draft + (int64_t)r * V;
         const T* y = P.target + (int64_t)r * V;
-        const float c = P.ts.c;
-        const MassRes mr{sh.rec.mx, sh.rec.my, sh.rec.izx, sh.rec.izy, c};
-        stream_residual<T, VEC>(rg, x, y, V, 0, P.nch, tab, mr, P.status);
+        const MassRes mr{rec.mx, rec.my, rec.izx, rec.izy, c};
+        stream_residual<T, VEC>(rg, x, y, V, 0, nch, tab, mr, P.status);
         __syncthreads();
-        if (warp == 0) {
-            const TableSum Rt = table_sum(tab, P.nch, 0, 0.f, c, lane);
-            if (lane == 0) sh.rt = Rt.Z;
-            if (Rt.Z > 0.0) {
-                for (int n = first; n < N; ++n) {
-                    if (__ldg(par + n) != u || sh.pacc[n]) continue;
-                    const float un = __ldg(P.u_correct + n0 + n);
+        {  // every warp computes the total; the rejected children are shared out
+            const TableSum Rt = table_sum(tab, nch, 0, 0.f, c, lane);
+            if (threadIdx.x == 0) *s_tok = Rt.Z > 0.0;
+            int k = 0;
+            if (Rt.Z > 0.0)
+                for (int n = u + 1; n < N; ++n) {
+                    if (__ldg(par + n) != u || ld_cg(o.path_accept + n0 + n)) continue;
+                    if (k++ % kWarps != warp) continue;
                     const Located loc =
-                        table_locate(tab, P.nch, 0, 0.f, c, Rt, un, lane);
+                        table_locate(tab, nch, 0, 0.f, c, Rt, __ldg(P.u_correct + n0 + n), lane);
                     int tok = -1;
                     if (loc.ch >= 0)
                         tok = warp_rescan<T, VEC, true, true>(x, y, V, loc.ch, loc.tc, mr, lane,
-                                                              policy_evict_normal());
+                                                              pol);
+                    if (lane == 0) o.corr_tokens[n0 + n] = tok < V ? tok : -1;
+                }
+        }
+        __syncthreads();
+        if (!*s_tok) {  // no residual mass: each rejected child draws from p
+            stream_tables<T, VEC, false>(rg, y, nullptr, V, 0, nch, tab, c, pol, pol, P.status);
+            __syncthreads();
+            {
+                const float M = table_max(tab, nch, 0, lane);
+                const TableSum S = table_sum(tab, nch, 0, frame_of(M), c, lane);
+                int k = 0;
+                for (int n = u + 1; n < N; ++n) {
+                    if (__ldg(par + n) != u || ld_cg(o.path_accept + n0 + n)) continue;
+                    if (k++ % kWarps != warp) continue;
+                    const int tok =
+                        row_ok(M, S.Z) ? warp_sample<T, VEC>(y, nullptr, V, tab, nch, 0, M, S,
+                                                             __ldg(P.u_correct + n0 + n), c,
+                                                             lane, pol)
+                                       : -1;
                     if (lane == 0) o.corr_tokens[n0 + n] = tok < V ? tok : -1;
                 }
             }
         }
         __syncthreads();
-        if (!(sh.rt > 0.0)) {
-            // no residual mass: each rejected child draws from p (reading R10)
-            for (int n = first; n < N; ++n) {
-                if (__ldg(par + n) != u || sh.pacc[n]) continue;
-                const int tok = p_draw<T, VEC>(P, r, __ldg(P.u_correct + n0 + n), rg, tab, &sh.resid);
-                if (threadIdx.x == 0) o.corr_tokens[n0 + n] = tok;
-            }
-        }
-        __syncthreads();
     }
-    if (threadIdx.x == 0) {
-        const int best = sh.deepest;
-        o.deepest[b] = best;
-        o.accept_len[b] = sh.depth[best];
-        int bonus = -1;
-        bool has_child = false;
-        for (int n = best + 1; n < N; ++n)
-            if (__ldg(par + n) == best) { bonus = o.corr_tokens[n0 + n]; has_child = true; break; }
-        if (!has_child) bonus = ld_cg(P.rows + n0 + best).ps;  // leaf: p-draw at its row
-        o.bonus[b] = bonus;
-    }
+}
+
+// The bonus token of tree b: the residual (or p) draw of the deepest accepted
+// node's first child, or, at a leaf, the p-draw at its row (one thread).
+template <typename T>
+__device__ void tree_bonus(const Problem<T>& P, int b) {
+    const int N = P.N;
+    const int n0 = b * N;
+    const int32_t* par = P.parent + (int64_t)n0;
+    const vsd_tree_outputs& o = P.tout;
+    const int best = ld_cg(o.deepest + b);
+    if (best < 0) return;  // invalid tree: already written
+    int bonus = -1;
+    bool has_child = false;
+    for (int n = best + 1; n < N; ++n)
+        if (__ldg(par + n) == best) { bonus = ld_cg(o.corr_tokens + n0 + n); has_child = true; break; }
+    if (!has_child) bonus = ld_cg(P.rows + n0 + best).ps;
+    o.bonus[b] = bonus;
 }
 
 }  // namespace vsd
