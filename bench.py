@@ -30,7 +30,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = ("draft-logit rows/s and achieved HBM GB/s (fraction of GB300 roofline) for fused "
           "E/M step")
-WORKLOADS = ("vocab128k", "vocab32k", "tiny", "lmhead")
+WORKLOADS = ("vocab128k", "vocab32k", "tiny", "lmhead", "tree60")
 
 
 def parse():
@@ -540,10 +540,180 @@ def run_lmhead(args):
                                 "sample": "the first %d rows (LM head in fp64 + E/M step)" % rows}
     print(json.dumps(line), flush=True)
 
+
+def oracle_tree_sample(prob, trees, T):
+    """The oracle's tree verification of the first `trees` trees: seconds."""
+    from oracle import oracle
+    N = prob["parent"].shape[1]
+    rows = trees * N
+    t0 = time.perf_counter()
+    oracle.tree(prob["draft"][:rows].float().cpu().numpy(),
+                prob["target"][:rows].float().cpu().numpy(), T,
+                prob["parent"][:trees].cpu().numpy(), prob["tokens"][:trees].cpu().numpy(),
+                prob["u_accept"][:trees].cpu().numpy(), prob["u_correct"][:trees].cpu().numpy())
+    return time.perf_counter() - t0
+
+
+def run_reference_tree(args):
+    """The oracle on the host cores for the tree workload: one tree per step."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2602_05774_gb300 import inputs
+    from oracle.build import build_oracle
+    build_oracle()
+    c = inputs.CONFIGS["tree60"]
+    small = inputs.config("tree60", device="cpu", seed=inputs.BASE_SEED + 99, B=1)
+    N = small["parent"].shape[1]
+    for _ in range(args.warmup):
+        oracle_tree_sample(small, 1, 1.0)
+    t = sum(oracle_tree_sample(small, 1, 1.0) for _ in range(args.steps))
+    ms = t / args.steps * 1e3
+    val = N / (ms / 1e3)
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": val, "unit": "rows/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; same recipe)",
+        "config": {"workload": "tree60", "B": c["B"], "N": N, "V": c["V"],
+                   "sample_per_step": "1 tree of %d nodes" % N},
+        "cpu_baseline": {"value": val, "unit": "rows/s", "cores": 1, "kind": "oracle",
+                         "sample": "one tree (%d rows) per step" % N},
+        "e2e": {"value": val, "unit": "rows/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def run_tree(args):
+    """Config 4: verification of B draft trees (vsd_verify_paths with a tree
+    layout); HBM roofline on the two logit reads."""
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2602_05774_gb300 import build, inputs, vsd
+    build.build_library()
+    vsd.load()
+    seed = inputs.BASE_SEED + list(inputs.CONFIGS).index("tree60") + 1000 * rank
+    prob = inputs.config("tree60", device=dev, seed=seed, B=args.prefixes or None)
+    B, N = prob["parent"].shape
+    V = prob["draft"].shape[-1]
+    R = B * N
+    T = 1.0
+    ws = vsd.new_workspace(vsd.layout(B, V=V, N=N, parent=prob["parent"]), dev)
+
+    def step(i):
+        return vsd.verify_tree(prob["draft"], prob["target"], prob["parent"], prob["tokens"],
+                               prob["u_accept"], prob["u_correct"], T, workspace=ws)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for i in range(args.warmup):
+        step(i)
+    barrier()
+    if vsd.device_status(ws)[0] != 0:
+        raise RuntimeError("device status after warm-up: %s" % (vsd.device_status(ws),))
+    stream = torch.cuda.current_stream(dev)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        barrier()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for i in range(args.steps):
+            ev[i][0].record(stream)
+            step(i)
+            ev[i][1].record(stream)
+        t1.record(stream)
+        barrier()
+    total_ms = t0.elapsed_time(t1)
+    launch_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = tt.item()
+    ms = total_ms / args.steps
+    if vsd.device_status(ws)[0] != 0:
+        raise RuntimeError("device status after timing")
+    e2e = None
+    if not args.no_e2e:  # inputs from pinned host buffers, accepted lengths read back
+        names = ("draft", "target", "parent", "tokens", "u_accept", "u_correct")
+        host = {k: prob[k].cpu().pin_memory() for k in names}
+        dv = {k: torch.empty_like(prob[k]) for k in names}
+        h_len = torch.empty(B, dtype=torch.int32).pin_memory()
+
+        def e2e_step(i):
+            for k in names:
+                dv[k].copy_(host[k], non_blocking=True)
+            o = vsd.verify_tree(dv["draft"], dv["target"], dv["parent"], dv["tokens"],
+                                dv["u_accept"], dv["u_correct"], T, workspace=ws)
+            h_len.copy_(o["accept_len"], non_blocking=True)
+
+        e_steps = max(3, min(args.steps, 20))
+        for i in range(2):
+            e2e_step(i)
+        barrier()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(e_steps):
+            e2e_step(i)
+        b.record(stream)
+        barrier()
+        e_ms = a.elapsed_time(b) / e_steps
+        e2e = {"value": R * world / (e_ms / 1e3), "unit": "rows/s",
+               "h2d_bytes_per_step": sum(host[k].numel() * host[k].element_size() for k in names),
+               "d2h_bytes_per_step": B * 4, "ms_per_step": e_ms, "steps": e_steps}
+    if rank != 0:
+        return
+    peak, peak_kind = peaks()
+    elem = prob["draft"].element_size()
+    alg = 2 * R * V * elem + R * 16  # both logit rows once; token, parent, two uniforms
+    achieved = alg / (launch_ms / 1e3) / 1e9
+    line = {
+        "metric": METRIC, "value": R * world / (ms / 1e3), "unit": "rows/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if elem == 2 else "f32",
+        "data": "synthetic (seeded; EAGLE-2-style trees, spiked logits)",
+        "config": {"workload": "tree60", "B": B, "N": N, "V": V, "logits": "bf16",
+                   "temperatures": [T], "l2": "inputs larger than L2 (no flush)",
+                   "rows_per_gpu": R},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
+                     "kernel": "k_rows_verify + k_tree + k_tree_residuals + k_tree_bonus",
+                     "algorithmic_bytes_per_launch": alg, "launch_ms": launch_ms},
+        "gpu_launches": 4 * args.steps,
+        "clocks": clk.summary(),
+    }
+    if e2e is not None:
+        line["e2e"] = e2e
+    if world == 1 and not args.no_cpu_baseline:
+        trees = 1
+        secs = oracle_tree_sample(prob, trees, T)
+        if secs < 8.0:
+            trees = min(B, max(1, int(12.0 / max(secs, 1e-3))))
+            secs = oracle_tree_sample(prob, trees, T)
+        line["cpu_baseline"] = {"value": trees * N / secs, "unit": "rows/s", "cores": 1,
+                                "kind": "oracle", "seconds": secs,
+                                "sample": "the first %d trees (%d rows)" % (trees, trees * N)}
+    print(json.dumps(line), flush=True)
+
 def main():
     args = parse()
     if args.config == "lmhead":
         run_reference_lmhead(args) if args.impl == "reference" else run_lmhead(args)
+    elif args.config == "tree60":
+        run_reference_tree(args) if args.impl == "reference" else run_tree(args)
     elif args.impl == "reference":
         run_reference(args)
     else:

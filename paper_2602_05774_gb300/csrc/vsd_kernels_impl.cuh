@@ -69,7 +69,7 @@ __global__ void __launch_bounds__(kThreads) k_tree(Problem<T> P) {
 }
 
 // kTreeBlocks blocks per tree share its residual rows.
-constexpr int kTreeBlocks = 4;
+constexpr int kTreeBlocks = 8;
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads) k_tree_residuals(Problem<T> P) {
     extern __shared__ __align__(128) unsigned char dsm[];

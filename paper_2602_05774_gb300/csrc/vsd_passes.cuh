@@ -1638,7 +1638,9 @@ struct TreeShared {
 //      depth; then log kappa level by level (each node adds its log alpha to
 //      its parent's); the deepest accepted node;
 //   3. the list of residual rows (accepted nodes with a rejected child) for
-//      tree_residuals, in tlist[b*N ..], its length in tcount[b].
+//      tree_residuals, in tlist[b*N ..], its length in tcount[b]; the first
+//      child of the deepest accepted node (or -1) in tlist[b*N + N - 1], a
+//      slot the list never reaches (node N - 1 has no children).
 template <typename T>
 __device__ void tree_nodes(const Problem<T>& P, int b, TreeShared& sh) {
     const int N = P.N;
@@ -1716,6 +1718,10 @@ __device__ void tree_nodes(const Problem<T>& P, int b, TreeShared& sh) {
         }
         sh.deepest = deepest;
         sh.maxdepth = maxd;
+        int first = -1;
+        for (int n = deepest + 1; n < N && first < 0; ++n)
+            if (__ldg(par + n) == deepest) first = n;
+        P.tlist[n0 + N - 1] = first;
         o.alpha[n0] = 1.f;
         o.accept[n0] = 1;
         o.path_accept[n0] = 1;
@@ -1821,16 +1827,11 @@ template <typename T>
 __device__ void tree_bonus(const Problem<T>& P, int b) {
     const int N = P.N;
     const int n0 = b * N;
-    const int32_t* par = P.parent + (int64_t)n0;
     const vsd_tree_outputs& o = P.tout;
     const int best = ld_cg(o.deepest + b);
     if (best < 0) return;  // invalid tree: already written
-    int bonus = -1;
-    bool has_child = false;
-    for (int n = best + 1; n < N; ++n)
-        if (__ldg(par + n) == best) { bonus = ld_cg(o.corr_tokens + n0 + n); has_child = true; break; }
-    if (!has_child) bonus = ld_cg(P.rows + n0 + best).ps;
-    o.bonus[b] = bonus;
+    const int child = ld_cg(P.tlist + n0 + N - 1);
+    o.bonus[b] = child >= 0 ? ld_cg(o.corr_tokens + n0 + child) : ld_cg(P.rows + n0 + best).ps;
 }
 
 }  // namespace vsd
