@@ -35,6 +35,11 @@ struct WsLayout {
 #define VSD_SEG_CHUNKS 128
 #endif
 constexpr int kSegChunks = VSD_SEG_CHUNKS;
+// Longest row (in chunks) whose tail the streaming warps run themselves.
+#ifndef VSD_STREAM_TAIL_CHUNKS
+#define VSD_STREAM_TAIL_CHUNKS 48
+#endif
+constexpr int kStreamTailChunks = VSD_STREAM_TAIL_CHUNKS;
 
 // Upper bounds of the chunk count and segment count of a row over both logit
 // dtypes (the smaller float32 chunk gives the larger count).
@@ -207,6 +212,7 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.path_A = at<int>(ws, w.path_A);
     // the tree layout has no E-step view and no path lengths: their arrays
     // hold its residual lists
+    P.stream_tails = 0;
     P.tlist = at<int>(ws, w.es_tok);
     P.tcount = at<int>(ws, w.path_A);
     P.resq = at<int>(ws, w.resq);
@@ -312,6 +318,10 @@ vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float
     const size_t gelem = P.grad_bf16 ? 2 : 4;
     const bool vec = vec_ok(draft, target, out->grad, L.V, sizeof(T), gelem);
     const int per_sm = Launch<T>::fused_blocks_per_sm(P, vec, P.grad_bf16);
+    // rows of one short segment: the streaming warps run the row tails
+    // themselves (three warps at once) instead of leaving them to the
+    // control warp, which would otherwise bound the kernel
+    P.stream_tails = (P.nseg == 1 && P.nch <= kStreamTailChunks) ? 1 : 0;
     const int64_t tickets = 2 * (int64_t)P.R * P.nseg;
     int ctas = per_sm * num_sms();
     if ((int64_t)ctas > tickets) ctas = (int)tickets;

@@ -136,6 +136,7 @@ constexpr int kSlots = VSD_SLOTS;  // jobs handed to the streaming warps ahead o
 // warps have finished that job.
 __device__ __forceinline__ int bar_full(int s) { return 1 + s; }
 __device__ __forceinline__ int bar_done(int s) { return 1 + kSlots + s; }
+constexpr int kStreamBar = 1 + 2 * kSlots;  // the streaming warps among themselves
 __device__ __forceinline__ void named_sync(int id) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(kFusedThreads) : "memory");
 }
@@ -285,7 +286,7 @@ __device__ void post_job(const Problem<T>& P, const EStepView& E, const Job& j, 
     if (j.kind == kJobRow) {
         const int r = j.r;
         if (!warp_count_last(P.row_seg_cnt + r, nseg, lane)) return;
-        row_tail_warp<T, VEC>(P, r, tab, cs.rb, lane);
+        if (!P.stream_tails) row_tail_warp<T, VEC>(P, r, tab, cs.rb, lane);
         __syncwarp();
         const int path = r / D;
         if (!warp_count_last(P.path_cnt + path, D, lane)) return;
@@ -374,6 +375,7 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ CtlShared cs;
     __shared__ Job slots[kSlots];
+    __shared__ RowShared rsh;
     Ring* rg;
     float4* tab;
     smem_views<VEC>(dsm, rg, tab);
@@ -388,9 +390,14 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
             const T* x = P.draft + (int64_t)j.r * V;
             if (j.kind == kJobRow) {
                 // The draft row is read again for the gradient: ask L2 to keep it.
+                float4* rtab = P.gtab + (int64_t)j.r * P.nch_ws;
                 stream_tables<T, VEC, true>(rg, x, P.target + (int64_t)j.r * V, V, j.c0, j.c1,
-                                            P.gtab + (int64_t)j.r * P.nch_ws, P.ts.c,
-                                            policy_evict_last(), policy_evict_first(), P.status);
+                                            rtab, P.ts.c, policy_evict_last(),
+                                            policy_evict_first(), P.status);
+                if (P.stream_tails) {  // short rows: the tail here, three draws at once
+                    asm volatile("bar.sync %0, %1;" ::"r"(kStreamBar), "r"(kThreads) : "memory");
+                    row_tail<T, VEC, true, kSampleToken, true, kStreamBar>(P, j.r, rtab, rsh);
+                }
             } else if (j.kind == kJobResidual) {
                 // row A's table was consumed by its row tail: reuse it
                 stream_residual<T, VEC>(rg, x, P.target + (int64_t)j.r * V, V, j.c0, j.c1,

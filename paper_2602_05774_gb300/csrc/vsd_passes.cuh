@@ -134,6 +134,7 @@ struct Problem {
     float4* gtab;                 // [R][nch_ws] per-chunk tables of each row
     int* row_seg_cnt;             // [R] segments of a row completed
     int* res_seg_cnt;             // [B*K] residual segments of a path completed
+    int stream_tails;             // fused kernel: the streaming warps run the row tails
     int* path_A;                  // [B*K] accepted length of a path
     int* tlist;                   // tree layout: [R] residual rows of each tree (its rows' slots)
     int* tcount;                  // tree layout: [B] length of each tree's list
@@ -809,17 +810,21 @@ struct RowShared {
     RowTask t[3];
 };
 
-// The per-row work once the row's chunk table tab[0..nch) is complete in
-// shared memory (block): warps 0, 1 and 2 take the three tasks at once, warp
-// 0 then writes the record.
-template <typename T, bool VEC, bool HAS_Y, int XMODE, bool ARGMAX>
+// The per-row work once the row's chunk table tab[0..nch) is complete
+// (block, or with BAR > 0 the kThreads threads 0 .. kThreads-1 that meet at
+// named barrier BAR): warps 0, 1 and 2 take the three tasks at once, warp 0
+// then writes the record.
+template <typename T, bool VEC, bool HAS_Y, int XMODE, bool ARGMAX, int BAR = 0>
 __device__ void row_tail(const Problem<T>& P, int r, const float4* tab, RowShared& sh) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (warp == 0 || (HAS_Y && (warp == 1 || (ARGMAX && warp == 2)))) {
         const RowTask t = row_task<T, VEC, XMODE>(P, r, tab, warp, lane);
         if (lane == 0) sh.t[warp] = t;
     }
-    __syncthreads();
+    if (BAR == 0)
+        __syncthreads();
+    else
+        asm volatile("bar.sync %0, %1;" ::"r"(BAR), "r"(kThreads) : "memory");
     if (warp == 0) {
         RowTask ty = sh.t[1];
         if (!HAS_Y) ty = RowTask{0.f, TableSum{0, 0, 0.0}, -1};
