@@ -30,11 +30,18 @@ struct WsLayout {
     int nch_ws, nseg_ws;
 };
 
-// Chunks per segment of the fused kernel's work items.
+// Chunks per segment of the fused kernel's row and residual jobs, and of its
+// gradient jobs.  Gradient jobs are cut finer: they need no follow-up step, and
+// small ones let the last prefixes' gradients spread over every block instead
+// of leaving most blocks idle at the end of the kernel.
 #ifndef VSD_SEG_CHUNKS
 #define VSD_SEG_CHUNKS 128
 #endif
 constexpr int kSegChunks = VSD_SEG_CHUNKS;
+#ifndef VSD_GRAD_SEG_CHUNKS
+#define VSD_GRAD_SEG_CHUNKS 16
+#endif
+constexpr int kGradSegChunks = VSD_GRAD_SEG_CHUNKS;
 // Longest row (in chunks) whose tail the streaming warps run themselves.
 #ifndef VSD_STREAM_TAIL_CHUNKS
 #define VSD_STREAM_TAIL_CHUNKS 48
@@ -205,6 +212,8 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.wscr = at<double2>(ws, w.wscr);
     P.segc = kSegChunks;
     P.nseg = (P.nch + kSegChunks - 1) / kSegChunks;
+    P.gsegc = kGradSegChunks;
+    P.gnseg = (P.nch + kGradSegChunks - 1) / kGradSegChunks;
     P.nch_ws = w.nch_ws;
     P.gtab = at<float4>(ws, w.gtab);
     P.row_seg_cnt = at<int>(ws, w.row_seg_cnt);
@@ -322,7 +331,7 @@ vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float
     // themselves (three warps at once) instead of leaving them to the
     // control warp, which would otherwise bound the kernel
     P.stream_tails = (P.nseg == 1 && P.nch <= kStreamTailChunks) ? 1 : 0;
-    const int64_t tickets = 2 * (int64_t)P.R * P.nseg;
+    const int64_t tickets = (int64_t)P.R * (P.nseg + P.gnseg);
     int ctas = per_sm * num_sms();
     if ((int64_t)ctas > tickets) ctas = (int)tickets;
     const char* env_ctas = getenv("VSD_FUSED_CTAS");

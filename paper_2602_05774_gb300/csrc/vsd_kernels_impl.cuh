@@ -166,7 +166,6 @@ template <typename T>
 __device__ bool claim_job(const Problem<T>& P, bool wait, int& g, Job& j) {
     const int B = P.B, nseg = P.nseg, segc = P.segc;
     const int row_items = P.R * nseg;
-    const int grad_items = P.K * P.D * nseg;  // per prefix
     uint64_t idle_since = 0;
     j.kind = kJobEnd;
     for (;;) {
@@ -197,13 +196,14 @@ __device__ bool claim_job(const Problem<T>& P, bool wait, int& g, Job& j) {
             return true;
         }
         if (rdy) {
+            const int gn = P.gnseg, gs = P.gsegc;
             const int t = atomicAdd(P.grad_cnt + g, 1);
-            if (t < grad_items) {
-                const int seg = t % nseg;
+            if (t < P.K * P.D * gn) {
+                const int seg = t % gn;
                 j.kind = kJobGrad;
-                j.r = g * P.K * P.D + t / nseg;
-                j.c0 = seg * segc;
-                j.c1 = min(P.nch, j.c0 + segc);
+                j.r = g * P.K * P.D + t / gn;
+                j.c0 = seg * gs;
+                j.c1 = min(P.nch, j.c0 + gs);
                 return true;
             }
             atomicMax(P.grad_head, g + 1);

@@ -36,13 +36,19 @@ using vsd::mbar_init_fence;
 using vsd::mbar_try_wait;
 using vsd::smem_u32;
 
-constexpr int BM = 128, BN = 256, BK = 64;  // BK bf16 = one 128-byte swizzle row
-constexpr int kStages = 4;
+#ifndef VSD_LM_BN
+#define VSD_LM_BN 256
+#endif
+#ifndef VSD_LM_STAGES
+#define VSD_LM_STAGES 4
+#endif
+constexpr int BM = 128, BN = VSD_LM_BN, BK = 64;  // BK bf16 = one 128-byte swizzle row
+constexpr int kStages = VSD_LM_STAGES;
 constexpr int kThreads = 192;
 constexpr int kABytes = BM * BK * 2;  // 16 KB
 constexpr int kBBytes = BN * BK * 2;  // 32 KB
 constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kTmemCols = 2 * BN;  // two fp32 accumulators of 128 lanes x 256 columns
+constexpr int kTmemCols = 2 * BN;  // two fp32 accumulators of 128 lanes x BN columns
 constexpr uint64_t kWaitNs = 2000000000ull;
 
 struct Bars {
@@ -382,7 +388,11 @@ cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, in
     }
     const long long ntiles =
         (long long)((M + vsd_lm::BM - 1) / vsd_lm::BM) * ((N + vsd_lm::BN - 1) / vsd_lm::BN);
-    const int grid = (int)(ntiles < sms ? ntiles : sms);
+#ifndef VSD_LM_CTAS_PER_SM
+#define VSD_LM_CTAS_PER_SM 1
+#endif
+    const long long slots = (long long)sms * VSD_LM_CTAS_PER_SM;
+    const int grid = (int)(ntiles < slots ? ntiles : slots);
     // (qualified: the enclosing namespace has a kThreads of its own)
     k_lmhead<<<grid, vsd_lm::kThreads, vsd_lm::kSmemBytes, s>>>(
         ta, tb, static_cast<__nv_bfloat16*>(logits), M, N, K, status);

@@ -131,6 +131,7 @@ struct Problem {
     // fused kernel: rows, residual rows and gradient rows are split into
     // segments of segc chunks (nseg per row)
     int segc, nseg, nch_ws;       // nch_ws: row stride of gtab (>= nch)
+    int gsegc, gnseg;             // gradient jobs: chunks per segment, segments per row
     float4* gtab;                 // [R][nch_ws] per-chunk tables of each row
     int* row_seg_cnt;             // [R] segments of a row completed
     int* res_seg_cnt;             // [B*K] residual segments of a path completed

@@ -76,6 +76,11 @@ SHAPES = [
     (1, 7, 3, 5000, "bf16", "zipf", 1.0),
     (3, 1, 6, 2048, "bf16", "spiked", 1.0),
     (2, 16, 1, 1536, "f32", "gauss", 1.0),
+    # rows longer than one work segment (several segments per row and per
+    # residual row): V above 128 chunks of 1024 bf16 / 512 f32 values
+    (1, 3, 3, 140000, "bf16", "zipf", 1.0),
+    (2, 2, 2, 70001, "f32", "gauss", 0.9),
+    (1, 2, 4, 262400, "bf16", "spiked", 1.0),
 ]
 
 
