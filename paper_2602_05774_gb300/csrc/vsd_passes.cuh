@@ -1591,6 +1591,37 @@ __device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1
         const float gq = cf.g * rec.izx;  // g / Z
         const uint64_t pol = policy_evict_first();
         const uint64_t mx2 = f2(rec.mx, rec.mx), c2 = f2(c, c), gq2 = f2(gq, gq);
+        // the sparse terms touch at most two positions of the row
+        auto emit = [&](int64_t v0, float (&o)[PV]) {
+            if ((uint64_t)(cf.t0 - v0) < (uint64_t)PV) {
+#pragma unroll
+                for (int e = 0; e < PV; ++e)
+                    if (v0 + e == cf.t0) o[e] -= cf.c0;
+            }
+            if ((uint64_t)(cf.t1 - v0) < (uint64_t)PV) {
+#pragma unroll
+                for (int e = 0; e < PV; ++e)
+                    if (v0 + e == cf.t1) o[e] -= cf.c1;
+            }
+            grad_store<T, G, PV>(g, v0, o, pol);
+        };
+        if (cf.g == 0.f && isfinite(rec.mx)) {
+            // No dense part: g q(v) is +0 for every mass in [0, 1], so the
+            // draft row is not read (rows no objective term reaches).
+            const int warp = threadIdx.x >> 5;
+            for (int ch = c0 + warp; ch < c1; ch += kWarps) {
+#pragma unroll
+                for (int k = 0; k < kLoads; ++k) {
+                    const int64_t v0 = (int64_t)ch * CE + (int64_t)k * 32 * PV + lane * PV;
+                    if (v0 >= V) break;
+                    float o[PV];
+#pragma unroll
+                    for (int e = 0; e < PV; ++e) o[e] = 0.f;
+                    emit(v0, o);
+                }
+            }
+            return;
+        }
         ring_stream<T, false>(
             rg, x, nullptr, V, c0, c1, pol, pol, P.status,
             [&](int ch, const uint4 (&bx)[kLoads], const uint4 (&)[kLoads]) {
@@ -1604,18 +1635,7 @@ __device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1
 #pragma unroll
                     for (int q = 0; q < NP; ++q)
                         f2split(f2mul(f2_mass(pr[q], mx2, c2), gq2), o[2 * q], o[2 * q + 1]);
-                    // the sparse terms touch at most two positions of the row
-                    if ((uint64_t)(cf.t0 - v0) < (uint64_t)PV) {
-#pragma unroll
-                        for (int e = 0; e < PV; ++e)
-                            if (v0 + e == cf.t0) o[e] -= cf.c0;
-                    }
-                    if ((uint64_t)(cf.t1 - v0) < (uint64_t)PV) {
-#pragma unroll
-                        for (int e = 0; e < PV; ++e)
-                            if (v0 + e == cf.t1) o[e] -= cf.c1;
-                    }
-                    grad_store<T, G, PV>(g, v0, o, pol);
+                    emit(v0, o);
                 }
             });
     }
