@@ -690,9 +690,9 @@ def run_tree(args):
                    "rows_per_gpu": R},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
-                     "kernel": "k_rows_verify + k_tree + k_tree_residuals + k_tree_bonus",
+                     "kernel": "k_tree_fused",
                      "algorithmic_bytes_per_launch": alg, "launch_ms": launch_ms},
-        "gpu_launches": 4 * args.steps,
+        "gpu_launches": args.steps,
         "clocks": clk.summary(),
     }
     if e2e is not None:

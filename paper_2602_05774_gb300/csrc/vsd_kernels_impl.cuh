@@ -39,17 +39,14 @@ __global__ void __launch_bounds__(kThreads) k_sample(Problem<T> P) {
     }
 }
 
-template <typename T, bool VEC, bool TREE>
+template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads) k_rows_verify(Problem<T> P) {
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ RowShared sh;
     Ring* rg;
     float4* tab;
     smem_views<VEC>(dsm, rg, tab);
-    if (TREE)
-        row_pass<T, VEC, true, kNoToken, false>(P, blockIdx.x, rg, tab, sh);
-    else
-        row_pass<T, VEC, true, kGivenToken, true>(P, blockIdx.x, rg, tab, sh);
+    row_pass<T, VEC, true, kGivenToken, true>(P, blockIdx.x, rg, tab, sh);
 }
 
 template <typename T, bool VEC>
@@ -60,31 +57,6 @@ __global__ void __launch_bounds__(kThreads) k_paths(Problem<T> P) {
     float4* tab;
     smem_views<VEC>(dsm, rg, tab);
     path_pass<T, VEC>(P, blockIdx.x, rg, tab, sh);
-}
-
-template <typename T>
-__global__ void __launch_bounds__(kThreads) k_tree(Problem<T> P) {
-    __shared__ TreeShared sh;
-    tree_nodes<T>(P, blockIdx.x, sh);
-}
-
-// kTreeBlocks blocks per tree share its residual rows.
-constexpr int kTreeBlocks = 8;
-template <typename T, bool VEC>
-__global__ void __launch_bounds__(kThreads) k_tree_residuals(Problem<T> P) {
-    extern __shared__ __align__(128) unsigned char dsm[];
-    __shared__ int s_tok;
-    Ring* rg;
-    float4* tab;
-    smem_views<VEC>(dsm, rg, tab);
-    tree_residuals<T, VEC>(P, blockIdx.x / kTreeBlocks, blockIdx.x % kTreeBlocks, kTreeBlocks, rg,
-                           tab, &s_tok);
-}
-
-template <typename T>
-__global__ void k_tree_bonus(Problem<T> P) {
-    const int b = blockIdx.x * blockDim.x + threadIdx.x;
-    if (b < P.B) tree_bonus<T>(P, b);
 }
 
 template <typename T>
@@ -121,6 +93,39 @@ __device__ __forceinline__ bool wait_flag(const int* flag, int* status, uint64_t
         if (global_timer_ns() - t0 > timeout_ns) return false;
         __nanosleep(1000);
     }
+}
+
+// Residual queue: producers reserve slots (resq_tail), write the items,
+// release each slot's flag and then add the items to resq_avail.  A consumer
+// reserves one published item with one atomic on resq_avail (returned at once
+// if none was left) and takes the next slot with one atomic on resq_head, so
+// claims pipeline in L2 instead of queueing behind a compare-and-swap.  The
+// slot may belong to a producer that reserved it but has not released it yet
+// (it is running, past its reservation): a bounded wait on the flag.
+// Callers look at resq_avail first.  Returns the item, -1 if none was left,
+// -2 if the wait ran out (status bit set).
+__device__ __forceinline__ int take_residual(int* head, int* avail, const int* flags,
+                                             const int* items, int* status,
+                                             uint64_t timeout_ns) {
+    if (atomicSub(avail, 1) <= 0) {
+        atomicAdd(avail, 1);
+        return -1;
+    }
+    const int h = atomicAdd(head, 1);
+    if (!wait_flag(flags + h, status, timeout_ns)) {
+        atomicOr(status, VSD_STATUS_TIMEOUT);
+        return -2;
+    }
+    return ld_cg(items + h);
+}
+
+__device__ __forceinline__ void publish_residuals(int* tail, int* avail, int* flags, int* items,
+                                                  int first, int n, bool sem) {
+    const int base = atomicAdd(tail, n);
+    for (int i = 0; i < n; ++i) items[base + i] = first + i;
+    __threadfence();
+    for (int i = 0; i < n; ++i) st_release(flags + base + i, 1);
+    if (sem) atomicAdd(avail, n);
 }
 
 // The fused kernel's block: kWarps streaming warps (threads 0 .. kThreads-1)
@@ -171,16 +176,25 @@ __device__ bool claim_job(const Problem<T>& P, bool wait, int& g, Job& j) {
     for (;;) {
         // independent reads first (one round trip), then at most one attempt
         // per kind of work
-        const int h = *(volatile int*)P.resq_head;
-        const int tl = *(volatile int*)P.resq_tail;
         const int tk = *(volatile int*)P.ticket;
         const int rdy = g < B ? ld_acquire(P.ready + g) : 0;
-        if (h < tl && atomicCAS(P.resq_head, h, h + 1) == h) {
-            if (!wait_flag(P.resq_flag + h, P.status, P.timeout_ns)) {
-                atomicOr(P.status, VSD_STATUS_TIMEOUT);
-                return true;  // end
+        int it = -1, av;
+        if (P.resq_sem) {  // short rows: claims must not queue (the chain bounds the kernel)
+            av = *(volatile int*)P.resq_avail > 0;
+            if (av)
+                it = take_residual(P.resq_head, P.resq_avail, P.resq_flag, P.resq, P.status,
+                                   P.timeout_ns);
+        } else {  // long rows: one compare-and-swap, fewer round trips per claim
+            const int h = *(volatile int*)P.resq_head;
+            const int tl = *(volatile int*)P.resq_tail;
+            av = h < tl;
+            if (av && atomicCAS(P.resq_head, h, h + 1) == h) {
+                it = wait_flag(P.resq_flag + h, P.status, P.timeout_ns) ? ld_cg(P.resq + h) : -2;
+                if (it == -2) atomicOr(P.status, VSD_STATUS_TIMEOUT);
             }
-            const int it = ld_cg(P.resq + h);
+        }
+        if (it == -2) return true;  // a wait ran out: end
+        if (it >= 0) {
             const int path = it / nseg, seg = it - path * nseg;
             const int A = ld_cg(P.path_A + path);
             const int rA = path * P.D + A;
@@ -225,7 +239,7 @@ __device__ bool claim_job(const Problem<T>& P, bool wait, int& g, Job& j) {
         if (g >= B) return true;  // every gradient segment has been claimed: end
         if (*(volatile int*)P.status & VSD_STATUS_TIMEOUT) return true;
         if (!wait) return false;
-        if (h < tl) continue;  // residual work is pending: try again at once
+        if (av) continue;  // residual work is pending: try again at once
         const uint64_t now = global_timer_ns();
         if (idle_since == 0) {
             idle_since = now;
@@ -295,10 +309,8 @@ __device__ void post_job(const Problem<T>& P, const EStepView& E, const Job& j, 
         if (A < D && !flags) {
             if (lane == 0) {  // queue the residual row's segments
                 P.path_A[path] = A;
-                const int base = atomicAdd(P.resq_tail, nseg);
-                for (int sg = 0; sg < nseg; ++sg) P.resq[base + sg] = path * nseg + sg;
-                __threadfence();
-                for (int sg = 0; sg < nseg; ++sg) st_release(P.resq_flag + base + sg, 1);
+                publish_residuals(P.resq_tail, P.resq_avail, P.resq_flag, P.resq, path * nseg,
+                                  nseg, P.resq_sem != 0);
             }
         } else {
             finish_path_warp<T>(P, E, path, A, -1, false, 0.f, 0.f, cs, lane);
@@ -450,6 +462,110 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
     }
 }
 
+// ------------------------------------------------------------ fused tree kernel
+// Tree verification in one launch of plain 128-thread blocks, R + tail
+// blocks.  Each block first takes a ticket: a ticket below R is a node row
+// (its tables and p-draw, then its children's acceptance); the block completing a
+// tree's last row runs the per-node pass for that tree (its shared memory is
+// the idle ring) and queues the tree's residual rows.  After its row a block
+// takes queued residual rows (the rejected children's draws) while any are
+// ready; the block completing a tree's last residual row writes its bonus
+// token.  A block whose ticket is R or more was started after every row had
+// been claimed, so every job it may wait for is held by a running block: it
+// waits for residual rows (bounded, status bit on expiry) until every tree is
+// done.
+template <typename T>
+__device__ int claim_residual(const Problem<T>& P, bool wait) {
+    uint64_t idle_since = 0;
+    for (;;) {
+        const int it = *(volatile int*)P.resq_avail > 0
+                           ? take_residual(P.resq_head, P.resq_avail, P.resq_flag, P.resq,
+                                           P.status, P.timeout_ns)
+                           : -1;
+        if (it >= 0) return it;
+        if (it == -2) return -1;
+        if (!wait) return -1;
+        if (*(volatile int*)P.prefix_done >= P.B) return -1;
+        if (*(volatile int*)P.status & VSD_STATUS_TIMEOUT) return -1;
+        const uint64_t now = global_timer_ns();
+        if (idle_since == 0) {
+            idle_since = now;
+        } else if (now - idle_since > P.timeout_ns) {
+            atomicOr(P.status, VSD_STATUS_TIMEOUT);
+            return -1;
+        }
+        __nanosleep(1000);
+    }
+}
+
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
+    extern __shared__ __align__(128) unsigned char dsm[];
+    __shared__ RowShared sh;
+    __shared__ int s_t, s_last, s_tok;
+    Ring* rg;
+    float4* tab;
+    smem_views<VEC>(dsm, rg, tab);
+    // The per-node pass runs between streams: on the vector path its shared
+    // memory is the ring's data (no copy is in flight then), else it follows
+    // the chunk table.
+    static_assert(sizeof(TreeShared) <= sizeof(Ring::data), "TreeShared fits the ring");
+    TreeShared* tsh = VEC ? reinterpret_cast<TreeShared*>(rg->data)
+                          : reinterpret_cast<TreeShared*>(tab + P.nch);
+    const int N = P.N;
+    if (threadIdx.x == 0) s_t = atomicAdd(P.ticket, 1);
+    __syncthreads();
+    const int t = s_t;
+    if (t < P.R) {
+        const int b = t / N;
+        row_pass<T, VEC, true, kNoToken, false>(P, t, rg, tab, sh);
+        __syncthreads();
+        tree_children<T>(P, b, t - b * N);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            __threadfence();
+            s_last = atomicAdd(P.path_cnt + b, 1) == N - 1;
+            if (s_last) __threadfence();
+        }
+        __syncthreads();
+        if (s_last) {
+            tree_nodes<T>(P, b, *tsh);
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                const int cnt = ld_cg(P.tcount + b);
+                if (cnt == 0) {
+                    tree_bonus<T>(P, b);
+                    __threadfence();
+                    atomicAdd(P.prefix_done, 1);
+                } else {  // queue the tree's residual rows (list positions)
+                    publish_residuals(P.resq_tail, P.resq_avail, P.resq_flag, P.resq, b * N,
+                                      cnt, true);
+                }
+            }
+            __syncthreads();
+        }
+    }
+    const bool wait = t >= P.R;
+    for (;;) {
+        if (threadIdx.x == 0) s_t = claim_residual<T>(P, wait);
+        __syncthreads();
+        const int item = s_t;
+        if (item < 0) break;
+        const int b = item / N;
+        tree_residual_row<T, VEC>(P, b, ld_cg(P.tlist + item), rg, tab, &s_tok);
+        if (threadIdx.x == 0) {
+            __threadfence();
+            if (atomicAdd(P.res_seg_cnt + b, 1) == ld_cg(P.tcount + b) - 1) {
+                __threadfence();
+                tree_bonus<T>(P, b);
+                __threadfence();
+                atomicAdd(P.prefix_done, 1);
+            }
+        }
+        __syncthreads();
+    }
+}
+
 // ------------------------------------------------------------ launchers
 // Static plus dynamic shared memory above 48 KB needs the kernel's opt-in.
 template <typename K>
@@ -474,20 +590,12 @@ cudaError_t Launch<VSD_T>::sample(const Problem<VSD_T>& P, bool vec, cudaStream_
 }
 
 template <>
-cudaError_t Launch<VSD_T>::rows_verify(const Problem<VSD_T>& P, bool vec, bool tree,
-                                       cudaStream_t s) {
+cudaError_t Launch<VSD_T>::rows_verify(const Problem<VSD_T>& P, bool vec, cudaStream_t s) {
     const size_t smem = stream_smem_bytes(P.nch, vec);
-#define VSD_ROWS(V_, T_)                                              \
-    do {                                                              \
-        cudaError_t e = prep(k_rows_verify<VSD_T, V_, T_>, smem);     \
-        if (e) return e;                                              \
-        k_rows_verify<VSD_T, V_, T_><<<P.R, kThreads, smem, s>>>(P);  \
-    } while (0)
-    if (vec && tree) VSD_ROWS(true, true);
-    else if (vec) VSD_ROWS(true, false);
-    else if (tree) VSD_ROWS(false, true);
-    else VSD_ROWS(false, false);
-#undef VSD_ROWS
+    auto kern = vec ? k_rows_verify<VSD_T, true> : k_rows_verify<VSD_T, false>;
+    cudaError_t e = prep(kern, smem);
+    if (e) return e;
+    kern<<<P.R, kThreads, smem, s>>>(P);
     return cudaGetLastError();
 }
 
@@ -507,27 +615,26 @@ cudaError_t Launch<VSD_T>::paths(const Problem<VSD_T>& P, bool vec, cudaStream_t
     return cudaGetLastError();
 }
 
+#ifndef VSD_TREE_TAIL_PER_SM
+#define VSD_TREE_TAIL_PER_SM 1
+#endif
 template <>
 cudaError_t Launch<VSD_T>::tree(const Problem<VSD_T>& P, bool vec, cudaStream_t s) {
-    // per node (one block per tree), then the residual rows (kTreeBlocks per
-    // tree), then the bonus tokens
-    k_tree<VSD_T><<<P.B, kThreads, 0, s>>>(P);
-    cudaError_t e = cudaGetLastError();
+    // one block per node row, then tail blocks for the last trees' residual rows
+    const size_t smem = stream_smem_bytes(P.nch, vec) + (vec ? 0 : sizeof(TreeShared));
+    auto kern = vec ? k_tree_fused<VSD_T, true> : k_tree_fused<VSD_T, false>;
+    cudaError_t e = prep(kern, smem);
     if (e) return e;
-    const size_t smem = stream_smem_bytes(P.nch, vec);
-    const int grid = P.B * kTreeBlocks;
-    if (vec) {
-        e = prep(k_tree_residuals<VSD_T, true>, smem);
-        if (e) return e;
-        k_tree_residuals<VSD_T, true><<<grid, kThreads, smem, s>>>(P);
-    } else {
-        e = prep(k_tree_residuals<VSD_T, false>, smem);
-        if (e) return e;
-        k_tree_residuals<VSD_T, false><<<grid, kThreads, smem, s>>>(P);
-    }
-    e = cudaGetLastError();
+    int dev = 0, sms = 0;
+    e = cudaGetDevice(&dev);
     if (e) return e;
-    k_tree_bonus<VSD_T><<<(P.B + 127) / 128, 128, 0, s>>>(P);
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e) return e;
+    long long tail = (long long)sms * VSD_TREE_TAIL_PER_SM;
+    const long long most = (long long)P.B * (P.N - 1);  // residual rows at most
+    if (tail > most) tail = most;
+    if (tail < 1) tail = 1;
+    kern<<<(unsigned)(P.R + tail), kThreads, smem, s>>>(P);
     return cudaGetLastError();
 }
 

@@ -11,11 +11,12 @@ namespace vsd {
 template <typename T> struct Launch {
     // z~ ~ q per row, tokens/logq/row_stats written from the row records
     static cudaError_t sample(const Problem<T>& P, bool vec, cudaStream_t s);
-    // row statistics of draft+target with given tokens (linear) or none (tree)
-    static cudaError_t rows_verify(const Problem<T>& P, bool vec, bool tree, cudaStream_t s);
+    // row statistics of draft+target with given tokens (linear paths)
+    static cudaError_t rows_verify(const Problem<T>& P, bool vec, cudaStream_t s);
     // accepted lengths, residual draws, corrected paths, log-kappa (linear)
     static cudaError_t paths(const Problem<T>& P, bool vec, cudaStream_t s);
-    // tree acceptance scan, residual draws, deepest node, bonus
+    // tree verification in one persistent launch: node rows, acceptance scan,
+    // residual draws, deepest node, bonus
     static cudaError_t tree(const Problem<T>& P, bool vec, cudaStream_t s);
     // M-step weights and loss from an E-step view
     static cudaError_t weights(const Problem<T>& P, const EStepView& E, float* weights,

@@ -19,10 +19,11 @@
 //                the per-row gradient coefficients.
 //   grad_pass    one streaming read of a draft row and write of its gradient:
 //                grad[v] = g q(v) - c0 [v = t0] - c1 [v = t1].
-//   tree_nodes / tree_residuals / tree_bonus   per draft tree: acceptance per
-//                node at its parent's row, the AND-scan along parent pointers,
-//                log kappa, the deepest node; residual draws at the parents of
-//                rejected nodes (several blocks per tree); the bonus token.
+//   tree_nodes / tree_residual_row / tree_bonus   per draft tree: acceptance
+//                per node at its parent's row, the AND-scan along parent
+//                pointers, log kappa, the deepest node; the residual draws at
+//                each accepted parent of rejected nodes (one block per such
+//                row); the bonus token.
 #pragma once
 
 #include "vsd_common.cuh"
@@ -139,10 +140,14 @@ struct Problem {
     int* path_A;                  // [B*K] accepted length of a path
     int* tlist;                   // tree layout: [R] residual rows of each tree (its rows' slots)
     int* tcount;                  // tree layout: [B] length of each tree's list
-    int* resq;                    // [B*K*nseg] residual segment items (path*nseg + seg)
-    int* resq_flag;               // [B*K*nseg] item written
+    float* tla;                   // tree layout: [R] log alpha of each node's token
+    int* resq;                    // [B*K*nseg] residual segment items (path*nseg + seg);
+                                  // trees: [B*N] positions b*N + i in the residual list
+    int* resq_flag;               // item written
     int* resq_head;               // next item to take
     int* resq_tail;               // next free slot
+    int* resq_avail;              // items published and not yet reserved (may dip below 0)
+    int resq_sem;                 // fused kernel claims residual items through resq_avail
     // outputs (device, caller-owned; null = not written)
     vsd_linear_outputs out;
     vsd_tree_outputs tout;
@@ -1140,7 +1145,7 @@ __device__ void path_epilogue_warp(const Problem<T>& P, int path, int A, int res
                 if (d < A) {
                     zc = rec.tok; lqc = rec.lq_tok; lac = rec.la_tok;
                 } else if (d == A) {
-                    zc = resid >= 0 ? resid : rec.ps;  // no residual mass: draw from p (R10)
+                    zc = resid >= 0 ? resid : rec.ps;  // no residual mass: draw from p
                     if (zc == rec.ps) {
                         lqc = rec.lq_ps; lac = rec.la_ps;
                     } else if (have_rl) {
@@ -1650,10 +1655,44 @@ __device__ void grad_pass(const Problem<T>& P, int r, const float4* rstats, G* g
 struct TreeShared {
     int bad, deepest, maxdepth;
     unsigned char acc[1024], pacc[1024], hasrej[1024];
+    int par[1024];
     int depth[1024];
     float la[1024];
     double lk[1024];
 };
+
+// The children of node u of tree b at row u (block, right after the row's
+// pass, while the row is still in L2): alpha, the accept bit (Eq. 1) and log
+// alpha of each child's token, for the per-node pass; and the row's
+// statistics output.
+template <typename T>
+__device__ void tree_children(const Problem<T>& P, int b, int u) {
+    const int N = P.N;
+    const int64_t V = P.V;
+    const int n0 = b * N, r = n0 + u;
+    const int32_t* par = P.parent + (int64_t)n0;
+    const vsd_tree_outputs& o = P.tout;
+    if (threadIdx.x == 0 && o.row_stats)
+        reinterpret_cast<float4*>(o.row_stats)[r] = ld_cg(P.rstats + r);
+    for (int n = u + 1 + threadIdx.x; n < N; n += kThreads) {
+        if (__ldg(par + n) != u) continue;
+        const RowRec rec = ld_cg(P.rows + r);
+        const int tok = __ldg(P.given_tokens + n0 + n);
+        float la = -INFINITY;
+        if (tok < 0 || tok >= V) {
+            atomicOr(P.status, VSD_STATUS_BAD_TOKEN);
+        } else if (!rec.flags) {
+            float lq;
+            token_logs(P.draft + (int64_t)r * V, P.target + (int64_t)r * V, tok, rec,
+                       P.ts.invTd, &lq, &la);
+        }
+        const float a = expf(la);
+        const bool acc = la > -INFINITY && __ldg(P.u_accept + n0 + n) <= a;
+        o.alpha[n0 + n] = a;
+        o.accept[n0 + n] = acc ? 1 : 0;
+        P.tla[n0 + n] = la;
+    }
+}
 
 // Tree verification, one draft tree b of N nodes per block; rows of tree b
 // are b*N .. b*N + N - 1, row n is the distribution node n's children were
@@ -1664,30 +1703,26 @@ struct TreeShared {
 //      depth; then log kappa level by level (each node adds its log alpha to
 //      its parent's); the deepest accepted node;
 //   3. the list of residual rows (accepted nodes with a rejected child) for
-//      tree_residuals, in tlist[b*N ..], its length in tcount[b]; the first
+//      tree_residual_row, in tlist[b*N ..], its length in tcount[b]; the first
 //      child of the deepest accepted node (or -1) in tlist[b*N + N - 1], a
 //      slot the list never reaches (node N - 1 has no children).
 template <typename T>
 __device__ void tree_nodes(const Problem<T>& P, int b, TreeShared& sh) {
     const int N = P.N;
-    const int64_t V = P.V;
     const int n0 = b * N;
     const int32_t* par = P.parent + (int64_t)n0;
     const vsd_tree_outputs& o = P.tout;
-    if (threadIdx.x == 0) {
-        int bad = (__ldg(par) != -1);
-        for (int n = 1; n < N && !bad; ++n) {
-            const int pn = __ldg(par + n);
-            if (pn < 0 || pn >= n) bad = 1;
-        }
-        sh.bad = bad;
-        if (bad) atomicOr(P.status, VSD_STATUS_BAD_TREE);
+    // parents into shared memory; a tree is valid if node 0 is the root and
+    // every other node's parent precedes it
+    int badl = 0;
+    for (int n = threadIdx.x; n < N; n += kThreads) {
+        const int pn = __ldg(par + n);
+        sh.par[n] = pn;
+        badl |= n == 0 ? pn != -1 : (pn < 0 || pn >= n);
     }
-    __syncthreads();
-    if (o.row_stats)
-        for (int n = threadIdx.x; n < N; n += kThreads)
-            reinterpret_cast<float4*>(o.row_stats)[n0 + n] = ld_cg(P.rstats + n0 + n);
-    if (sh.bad) {
+    const int bad = __syncthreads_or(badl);
+    if (bad) {
+        if (threadIdx.x == 0) atomicOr(P.status, VSD_STATUS_BAD_TREE);
         for (int n = threadIdx.x; n < N; n += kThreads) {
             o.alpha[n0 + n] = 0.f;
             o.accept[n0 + n] = 0;
@@ -1703,29 +1738,10 @@ __device__ void tree_nodes(const Problem<T>& P, int b, TreeShared& sh) {
         }
         return;
     }
-    // 1. per node
+    // 1. per node: log alpha and the accept bit from the parents' row blocks
     for (int n = threadIdx.x; n < N; n += kThreads) {
-        float la = 0.f;
-        bool acc = true;
-        if (n > 0) {
-            const int pn = __ldg(par + n);
-            const RowRec rec = ld_cg(P.rows + n0 + pn);
-            const int tok = __ldg(P.given_tokens + n0 + n);
-            la = -INFINITY;
-            if (tok < 0 || tok >= V) {
-                atomicOr(P.status, VSD_STATUS_BAD_TOKEN);
-            } else if (!rec.flags) {
-                float lq;
-                token_logs(P.draft + (int64_t)(n0 + pn) * V, P.target + (int64_t)(n0 + pn) * V,
-                           tok, rec, P.ts.invTd, &lq, &la);
-            }
-            const float a = expf(la);
-            acc = la > -INFINITY && __ldg(P.u_accept + n0 + n) <= a;
-            o.alpha[n0 + n] = a;
-            o.accept[n0 + n] = acc ? 1 : 0;
-        }
-        sh.la[n] = la;
-        sh.acc[n] = acc ? 1 : 0;
+        sh.la[n] = n > 0 ? ld_cg(P.tla + n0 + n) : 0.f;
+        sh.acc[n] = n > 0 ? ld_cg(o.accept + n0 + n) : 1;
         sh.hasrej[n] = 0;
     }
     __syncthreads();
@@ -1736,7 +1752,7 @@ __device__ void tree_nodes(const Problem<T>& P, int b, TreeShared& sh) {
         sh.lk[0] = 0.0;
         int deepest = 0, maxd = 0;
         for (int n = 1; n < N; ++n) {
-            const int pn = __ldg(par + n);
+            const int pn = sh.par[n];
             sh.pacc[n] = (unsigned char)(sh.acc[n] && sh.pacc[pn]);
             sh.depth[n] = sh.depth[pn] + 1;
             maxd = max(maxd, sh.depth[n]);
@@ -1746,7 +1762,7 @@ __device__ void tree_nodes(const Problem<T>& P, int b, TreeShared& sh) {
         sh.maxdepth = maxd;
         int first = -1;
         for (int n = deepest + 1; n < N && first < 0; ++n)
-            if (__ldg(par + n) == deepest) first = n;
+            if (sh.par[n] == deepest) first = n;
         P.tlist[n0 + N - 1] = first;
         o.alpha[n0] = 1.f;
         o.accept[n0] = 1;
@@ -1759,14 +1775,14 @@ __device__ void tree_nodes(const Problem<T>& P, int b, TreeShared& sh) {
     __syncthreads();
     for (int L = 1; L <= sh.maxdepth; ++L) {  // log kappa along each branch (Eq. 2)
         for (int n = threadIdx.x; n < N; n += kThreads)
-            if (sh.depth[n] == L) sh.lk[n] = sh.lk[__ldg(par + n)] + (double)sh.la[n];
+            if (sh.depth[n] == L) sh.lk[n] = sh.lk[sh.par[n]] + (double)sh.la[n];
         __syncthreads();
     }
     for (int n = 1 + threadIdx.x; n < N; n += kThreads) {
         o.path_accept[n0 + n] = sh.pacc[n];
         o.logkappa[n0 + n] = (float)sh.lk[n];
         o.corr_tokens[n0 + n] = -1;
-        const int pn = __ldg(par + n);
+        const int pn = sh.par[n];
         if (sh.pacc[pn] && !sh.pacc[n]) sh.hasrej[pn] = 1;
     }
     __syncthreads();
@@ -1779,13 +1795,12 @@ __device__ void tree_nodes(const Problem<T>& P, int b, TreeShared& sh) {
     }
 }
 
-// Residual rows of tree b, items g, g + G, ... of its list (block): stream
-// the row's residual max(0, p - q) (Sec. 3) and draw each rejected child's
-// token with the child's own uniform; if the residual has no mass, a draw
-// from p instead (reading R10).
+// Residual row of node u of tree b (block): stream the row's residual
+// max(0, p - q) (Sec. 3) and draw each rejected child's token with the
+// child's own uniform; if the residual has no mass, a draw from p instead.
 template <typename T, bool VEC>
-__device__ void tree_residuals(const Problem<T>& P, int b, int g, int G, Ring* rg, float4* tab,
-                               int* s_tok) {
+__device__ void tree_residual_row(const Problem<T>& P, int b, int u, Ring* rg, float4* tab,
+                                  int* s_tok) {
     const int N = P.N;
     const int64_t V = P.V;
     const int n0 = b * N;
@@ -1795,56 +1810,48 @@ __device__ void tree_residuals(const Problem<T>& P, int b, int g, int G, Ring* r
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const float c = P.ts.c;
     const uint64_t pol = policy_evict_normal();
-    const int cnt = ld_cg(P.tcount + b);
-    for (int i = g; i < cnt; i += G) {
-        const int u = ld_cg(P.tlist + n0 + i);
-        const int r = n0 + u;
-        const RowRec rec = ld_cg(P.rows + r);
-        if (rec.flags) continue;
-        const T* x = P.draft + (int64_t)r * V;
-        const T* y = P.target + (int64_t)r * V;
-        const MassRes mr{rec.mx, rec.my, rec.izx, rec.izy, c};
-        stream_residual<T, VEC>(rg, x, y, V, 0, nch, tab, mr, P.status);
-        __syncthreads();
-        {  // every warp computes the total; the rejected children are shared out
-            const TableSum Rt = table_sum(tab, nch, 0, 0.f, c, lane);
-            if (threadIdx.x == 0) *s_tok = Rt.Z > 0.0;
-            int k = 0;
-            if (Rt.Z > 0.0)
-                for (int n = u + 1; n < N; ++n) {
-                    if (__ldg(par + n) != u || ld_cg(o.path_accept + n0 + n)) continue;
-                    if (k++ % kWarps != warp) continue;
-                    const Located loc =
-                        table_locate(tab, nch, 0, 0.f, c, Rt, __ldg(P.u_correct + n0 + n), lane);
-                    int tok = -1;
-                    if (loc.ch >= 0)
-                        tok = warp_rescan<T, VEC, true, true>(x, y, V, loc.ch, loc.tc, mr, lane,
-                                                              pol);
-                    if (lane == 0) o.corr_tokens[n0 + n] = tok < V ? tok : -1;
-                }
-        }
-        __syncthreads();
-        if (!*s_tok) {  // no residual mass: each rejected child draws from p
-            stream_tables<T, VEC, false>(rg, y, nullptr, V, 0, nch, tab, c, pol, pol, P.status);
-            __syncthreads();
-            {
-                const float M = table_max(tab, nch, 0, lane);
-                const TableSum S = table_sum(tab, nch, 0, frame_of(M), c, lane);
-                int k = 0;
-                for (int n = u + 1; n < N; ++n) {
-                    if (__ldg(par + n) != u || ld_cg(o.path_accept + n0 + n)) continue;
-                    if (k++ % kWarps != warp) continue;
-                    const int tok =
-                        row_ok(M, S.Z) ? warp_sample<T, VEC>(y, nullptr, V, tab, nch, 0, M, S,
-                                                             __ldg(P.u_correct + n0 + n), c,
-                                                             lane, pol)
-                                       : -1;
-                    if (lane == 0) o.corr_tokens[n0 + n] = tok < V ? tok : -1;
-                }
+    const int r = n0 + u;
+    const RowRec rec = ld_cg(P.rows + r);
+    if (rec.flags) return;
+    const T* x = P.draft + (int64_t)r * V;
+    const T* y = P.target + (int64_t)r * V;
+    const MassRes mr{rec.mx, rec.my, rec.izx, rec.izy, c};
+    stream_residual<T, VEC>(rg, x, y, V, 0, nch, tab, mr, P.status);
+    __syncthreads();
+    {  // every warp computes the total; the rejected children are shared out
+        const TableSum Rt = table_sum(tab, nch, 0, 0.f, c, lane);
+        if (threadIdx.x == 0) *s_tok = Rt.Z > 0.0;
+        int k = 0;
+        if (Rt.Z > 0.0)
+            for (int n = u + 1; n < N; ++n) {
+                if (__ldg(par + n) != u || ld_cg(o.path_accept + n0 + n)) continue;
+                if (k++ % kWarps != warp) continue;
+                const Located loc =
+                    table_locate(tab, nch, 0, 0.f, c, Rt, __ldg(P.u_correct + n0 + n), lane);
+                int tok = -1;
+                if (loc.ch >= 0)
+                    tok = warp_rescan<T, VEC, true, true>(x, y, V, loc.ch, loc.tc, mr, lane, pol);
+                if (lane == 0) o.corr_tokens[n0 + n] = tok < V ? tok : -1;
             }
-        }
-        __syncthreads();
     }
+    __syncthreads();
+    if (!*s_tok) {  // no residual mass: each rejected child draws from p
+        stream_tables<T, VEC, false>(rg, y, nullptr, V, 0, nch, tab, c, pol, pol, P.status);
+        __syncthreads();
+        const float M = table_max(tab, nch, 0, lane);
+        const TableSum S = table_sum(tab, nch, 0, frame_of(M), c, lane);
+        int k = 0;
+        for (int n = u + 1; n < N; ++n) {
+            if (__ldg(par + n) != u || ld_cg(o.path_accept + n0 + n)) continue;
+            if (k++ % kWarps != warp) continue;
+            const int tok = row_ok(M, S.Z)
+                                ? warp_sample<T, VEC>(y, nullptr, V, tab, nch, 0, M, S,
+                                                      __ldg(P.u_correct + n0 + n), c, lane, pol)
+                                : -1;
+            if (lane == 0) o.corr_tokens[n0 + n] = tok < V ? tok : -1;
+        }
+    }
+    __syncthreads();
 }
 
 // The bonus token of tree b: the residual (or p) draw of the deepest accepted
