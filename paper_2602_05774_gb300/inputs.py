@@ -150,6 +150,9 @@ def tree_shapes(B, N, depth, topk, seed):
                     pool.append((sc_k, dep, pi, k))
             layer.sort(key=lambda i: -pool[i][0])
             frontier = layer[:topk]
+        if len(pool) < N:
+            raise ValueError("depth %d and top-%d give %d candidates, fewer than N = %d"
+                             % (depth, topk, len(pool), N))
         order = sorted(range(1, len(pool)), key=lambda i: -pool[i][0])[: N - 1]
         keep = [0] + sorted(order, key=lambda i: (pool[i][1], -pool[i][0]))
         pos = {pi: n for n, pi in enumerate(keep)}

@@ -200,6 +200,46 @@ def test_small_trees_matches_oracle(vsd, oracle):
         compare_tree(g, orc)
 
 
+
+def _tree_case(B, N, V, parent, seed, same=False):
+    """Random spiked logits (target = draft if same) for a given parent array,
+    node tokens drawn among each parent row's 8 largest draft logits."""
+    g = torch.Generator().manual_seed(seed)
+    draft = torch.randn(B * N, V, generator=g) * 3.0
+    target = draft.clone() if same else draft + torch.randn(B * N, V, generator=g)
+    parent = torch.as_tensor(parent, dtype=torch.int32).view(1, N).repeat(B, 1)
+    top = draft.topk(min(8, V), dim=1).indices.to(torch.int32)
+    rows = (torch.arange(B).view(B, 1) * N + parent.clamp(min=0).long()).view(-1)
+    pick = torch.randint(0, min(8, V), (B * N,), generator=g)
+    tokens = top[rows, pick].view(B, N)
+    tokens[:, 0] = 0
+    return dict(B=B, N=N, V=V, draft=draft.to(torch.bfloat16), target=target.to(torch.bfloat16),
+                parent=parent, tokens=tokens,
+                u_accept=torch.rand(B, N, generator=g), u_correct=torch.rand(B, N, generator=g))
+
+
+def test_tree_edge_shapes(vsd, oracle):
+    """Root-only trees, the largest tree (1024 nodes), a chain whose every
+    token is accepted (target = draft: no residual row, the bonus is the leaf
+    row's p-draw) and a star (every node a child of the root)."""
+    from paper_2602_05774_gb300 import inputs
+    cases = [inputs.tree_problem(3, 1, 1, 1, 100, seed=5),
+             inputs.tree_problem(2, 1024, 17, 8, 64, seed=6),
+             _tree_case(2, 8, 50, [-1, 0, 1, 2, 3, 4, 5, 6], seed=7, same=True),
+             _tree_case(3, 9, 300, [-1] + [0] * 8, seed=8)]
+    for i, prob in enumerate(cases):
+        orc = oracle.tree(_np32(prob["draft"]), _np32(prob["target"]), 1.0,
+                          prob["parent"].numpy(), prob["tokens"].numpy(),
+                          _np32(prob["u_accept"]), _np32(prob["u_correct"]))
+        p = to_cuda(prob)
+        g = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"], p["u_accept"],
+                            p["u_correct"], 1.0)
+        torch.cuda.synchronize()
+        compare_tree(g, orc)
+        if i == 2:  # the chain: every node accepted, so the accepted length is N - 1
+            assert (g["accept_len"].cpu() == 7).all()
+
+
 @pytest.mark.parametrize("T", [1.0, 0.7])
 def test_vocab128k_full_size_sampled_prefixes(vsd, oracle, T):
     """The benchmark's workload and launch; the oracle checks two sampled prefixes."""
