@@ -49,10 +49,8 @@ def parse():
 
 
 def dist_env():
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return rank, world, local
+    from paper_2602_05774_gb300 import multirank
+    return multirank.env()
 
 
 def peaks():
@@ -217,16 +215,15 @@ def run_reference(args):
 def run_ours(args):
     import torch
     rank, world, local = dist_env()
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
+    from paper_2602_05774_gb300 import multirank
+    multirank.init(world, "nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     from paper_2602_05774_gb300 import build, inputs, vsd
     build.build_library()
     vsd.load()
     c = inputs.CONFIGS[args.config]
-    seed = inputs.BASE_SEED + list(inputs.CONFIGS).index(args.config) + 1000 * rank
+    seed = multirank.rank_seed(inputs.BASE_SEED + list(inputs.CONFIGS).index(args.config), rank)
     prob = inputs.config(args.config, device=dev, seed=seed, B=args.prefixes or None)
     torch.cuda.empty_cache()
     B, K, D, V = prob["B"], prob["K"], prob["D"], prob["V"]
@@ -253,10 +250,7 @@ def run_ours(args):
         raise RuntimeError("device status %d (bits %d) after warm-up" % (code, bits))
 
     def barrier():
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
-        torch.cuda.synchronize(dev)
+        multirank.barrier(world, dev)
 
     stream = torch.cuda.current_stream(dev)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -274,11 +268,7 @@ def run_ours(args):
         barrier()
     total_ms = t0.elapsed_time(t1)
     launch_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
-    if world > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = tt.item()
+    total_ms = multirank.max_over_ranks(total_ms, world, dev)
     ms = total_ms / args.steps
     code, bits = vsd.device_status(ws)
     if code != 0:
@@ -303,12 +293,8 @@ def run_ours(args):
         b.record(stream)
         barrier()
         e_ms = a.elapsed_time(b) / e_steps
-        if world > 1:
-            import torch.distributed as dist
-            tt = torch.tensor([e_ms], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e_ms = tt.item()
-        e2e = {"value": R * world / (e_ms / 1e3), "unit": "rows/s",
+        e_ms = multirank.max_over_ranks(e_ms, world, dev)
+        e2e = {"value": multirank.job_rate(R, world, e_ms), "unit": "rows/s",
                "h2d_bytes_per_step": hs.h2d_bytes(), "d2h_bytes_per_step": hs.d2h_bytes(),
                "ms_per_step": e_ms, "steps": e_steps}
         assert torch.isfinite(loss).all()
@@ -320,7 +306,7 @@ def run_ours(args):
     alg = algorithmic_bytes(R, V, elem, gelem)
     achieved = alg / (launch_ms / 1e3) / 1e9
     traffic = ncu_traffic(args.config)
-    value = R * world / (ms / 1e3)
+    value = multirank.job_rate(R, world, ms)
     line = {
         "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
@@ -413,15 +399,14 @@ def run_lmhead(args):
     on its own with CUDA events per launch."""
     import torch
     rank, world, local = dist_env()
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
+    from paper_2602_05774_gb300 import multirank
+    multirank.init(world, "nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     from paper_2602_05774_gb300 import build, inputs, vsd
     build.build_library()
     vsd.load()
-    seed = inputs.BASE_SEED + list(inputs.CONFIGS).index("lmhead") + 1000 * rank
+    seed = multirank.rank_seed(inputs.BASE_SEED + list(inputs.CONFIGS).index("lmhead"), rank)
     prob = inputs.config("lmhead", device=dev, seed=seed, B=args.prefixes or None)
     B, K, D, V, H = prob["B"], prob["K"], prob["D"], prob["V"], prob["H"]
     R = B * K * D
@@ -437,10 +422,7 @@ def run_lmhead(args):
                                workspace=ws, out=out, draft_logits=dl)
 
     def barrier():
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
-        torch.cuda.synchronize(dev)
+        multirank.barrier(world, dev)
 
     def timed(fn, n):
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -471,11 +453,7 @@ def run_lmhead(args):
             vsd.lmhead_logits(prob["hidden"], prob["weight"], out=dl, workspace=gws)
         _, gemm_ms = timed(lambda i: vsd.lmhead_logits(prob["hidden"], prob["weight"], out=dl,
                                                        workspace=gws), args.steps)
-    if world > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = tt.item()
+    total_ms = multirank.max_over_ranks(total_ms, world, dev)
     ms = total_ms / args.steps
     if vsd.device_status(ws)[0] != 0 or vsd.device_status(gws)[0] != 0:
         raise RuntimeError("device status after timing")
@@ -502,8 +480,8 @@ def run_lmhead(args):
         for i in range(2):
             e2e_step(i)
         e_total, _ = timed(e2e_step, e_steps)
-        e_ms = e_total / e_steps
-        e2e = {"value": R * world / (e_ms / 1e3), "unit": "rows/s",
+        e_ms = multirank.max_over_ranks(e_total / e_steps, world, dev)
+        e2e = {"value": multirank.job_rate(R, world, e_ms), "unit": "rows/s",
                "h2d_bytes_per_step": (h_hidden.numel() * 2 + h_target.numel() * 2
                                       + h_u.numel() * 4),
                "d2h_bytes_per_step": h_loss.numel() * 4, "ms_per_step": e_ms,
@@ -514,7 +492,7 @@ def run_lmhead(args):
     flops = 2.0 * R * V * H
     achieved = flops / (gemm_ms / 1e3) / 1e12
     line = {
-        "metric": METRIC, "value": R * world / (ms / 1e3), "unit": "rows/s", "n_gpus": world,
+        "metric": METRIC, "value": multirank.job_rate(R, world, ms), "unit": "rows/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; hidden ~N(0,1), LM-head weight ~N(0,0.02^2), spiked target)",
@@ -589,15 +567,14 @@ def run_tree(args):
     layout); HBM roofline on the two logit reads."""
     import torch
     rank, world, local = dist_env()
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
+    from paper_2602_05774_gb300 import multirank
+    multirank.init(world, "nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     from paper_2602_05774_gb300 import build, inputs, vsd
     build.build_library()
     vsd.load()
-    seed = inputs.BASE_SEED + list(inputs.CONFIGS).index("tree60") + 1000 * rank
+    seed = multirank.rank_seed(inputs.BASE_SEED + list(inputs.CONFIGS).index("tree60"), rank)
     prob = inputs.config("tree60", device=dev, seed=seed, B=args.prefixes or None)
     B, N = prob["parent"].shape
     V = prob["draft"].shape[-1]
@@ -610,10 +587,7 @@ def run_tree(args):
                                prob["u_accept"], prob["u_correct"], T, workspace=ws)
 
     def barrier():
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
-        torch.cuda.synchronize(dev)
+        multirank.barrier(world, dev)
 
     for i in range(args.warmup):
         step(i)
@@ -636,11 +610,7 @@ def run_tree(args):
         barrier()
     total_ms = t0.elapsed_time(t1)
     launch_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
-    if world > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = tt.item()
+    total_ms = multirank.max_over_ranks(total_ms, world, dev)
     ms = total_ms / args.steps
     if vsd.device_status(ws)[0] != 0:
         raise RuntimeError("device status after timing")
@@ -669,8 +639,8 @@ def run_tree(args):
             e2e_step(i)
         b.record(stream)
         barrier()
-        e_ms = a.elapsed_time(b) / e_steps
-        e2e = {"value": R * world / (e_ms / 1e3), "unit": "rows/s",
+        e_ms = multirank.max_over_ranks(a.elapsed_time(b) / e_steps, world, dev)
+        e2e = {"value": multirank.job_rate(R, world, e_ms), "unit": "rows/s",
                "h2d_bytes_per_step": sum(host[k].numel() * host[k].element_size() for k in names),
                "d2h_bytes_per_step": B * 4, "ms_per_step": e_ms, "steps": e_steps}
     if rank != 0:
@@ -680,7 +650,7 @@ def run_tree(args):
     alg = 2 * R * V * elem + R * 16  # both logit rows once; token, parent, two uniforms
     achieved = alg / (launch_ms / 1e3) / 1e9
     line = {
-        "metric": METRIC, "value": R * world / (ms / 1e3), "unit": "rows/s", "n_gpus": world,
+        "metric": METRIC, "value": multirank.job_rate(R, world, ms), "unit": "rows/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16" if elem == 2 else "f32",
