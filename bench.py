@@ -296,7 +296,9 @@ def run_ours(args):
         e_ms = multirank.max_over_ranks(e_ms, world, dev)
         e2e = {"value": multirank.job_rate(R, world, e_ms), "unit": "rows/s",
                "h2d_bytes_per_step": hs.h2d_bytes(), "d2h_bytes_per_step": hs.d2h_bytes(),
-               "ms_per_step": e_ms, "steps": e_steps}
+               "ms_per_step": e_ms, "steps": e_steps,
+               "inputs": "double-buffered: a step's copies overlap the previous step's kernels"}
+        torch.cuda.synchronize(dev)
         assert torch.isfinite(loss).all()
         del hs, h_draft, h_target, h_u
 
@@ -463,18 +465,11 @@ def run_lmhead(args):
         h_hidden = prob["hidden"].cpu().pin_memory()
         h_target = prob["target"].cpu().pin_memory()
         h_u = torch.stack([prob["u_draft"], prob["u_accept"], prob["u_correct"]]).cpu().pin_memory()
-        d_hidden = torch.empty_like(prob["hidden"])
-        d_target = torch.empty_like(prob["target"])
-        d_u = torch.empty(3, R, dtype=torch.float32, device=dev)
-        h_loss = torch.empty(B + 1, dtype=torch.float32).pin_memory()
+        hs = vsd.HostLMHeadStep(prob["weight"], B, K, D, V, prm=prm)
+        losses = []
 
         def e2e_step(i):
-            d_hidden.copy_(h_hidden, non_blocking=True)
-            d_target.copy_(h_target, non_blocking=True)
-            d_u.copy_(h_u, non_blocking=True)
-            vsd.lmhead_estep_mstep(d_hidden, prob["weight"], d_target, d_u[0], d_u[1], d_u[2],
-                                   K, D, T, prm=prm, workspace=ws, out=out, draft_logits=dl)
-            h_loss.copy_(out["loss"], non_blocking=True)
+            losses.append(hs(h_hidden, h_target, h_u, T))
 
         e_steps = max(3, min(args.steps, 20))
         for i in range(2):
@@ -482,10 +477,11 @@ def run_lmhead(args):
         e_total, _ = timed(e2e_step, e_steps)
         e_ms = multirank.max_over_ranks(e_total / e_steps, world, dev)
         e2e = {"value": multirank.job_rate(R, world, e_ms), "unit": "rows/s",
-               "h2d_bytes_per_step": (h_hidden.numel() * 2 + h_target.numel() * 2
-                                      + h_u.numel() * 4),
-               "d2h_bytes_per_step": h_loss.numel() * 4, "ms_per_step": e_ms,
-               "steps": e_steps, "weights": "resident on the device"}
+               "h2d_bytes_per_step": hs.h2d_bytes(), "d2h_bytes_per_step": hs.d2h_bytes(),
+               "ms_per_step": e_ms, "steps": e_steps, "weights": "resident on the device",
+               "inputs": "double-buffered: a step's copies overlap the previous step's kernels"}
+        assert torch.isfinite(losses[-1]).all()
+        del hs
     if rank != 0:
         return
     peak, peak_kind = tensor_peak()
@@ -618,15 +614,10 @@ def run_tree(args):
     if not args.no_e2e:  # inputs from pinned host buffers, accepted lengths read back
         names = ("draft", "target", "parent", "tokens", "u_accept", "u_correct")
         host = {k: prob[k].cpu().pin_memory() for k in names}
-        dv = {k: torch.empty_like(prob[k]) for k in names}
-        h_len = torch.empty(B, dtype=torch.int32).pin_memory()
+        hs = vsd.HostTreeStep(B, N, V, prob["draft"].dtype, dev)
 
         def e2e_step(i):
-            for k in names:
-                dv[k].copy_(host[k], non_blocking=True)
-            o = vsd.verify_tree(dv["draft"], dv["target"], dv["parent"], dv["tokens"],
-                                dv["u_accept"], dv["u_correct"], T, workspace=ws)
-            h_len.copy_(o["accept_len"], non_blocking=True)
+            hs(host, T)
 
         e_steps = max(3, min(args.steps, 20))
         for i in range(2):
@@ -641,8 +632,10 @@ def run_tree(args):
         barrier()
         e_ms = multirank.max_over_ranks(a.elapsed_time(b) / e_steps, world, dev)
         e2e = {"value": multirank.job_rate(R, world, e_ms), "unit": "rows/s",
-               "h2d_bytes_per_step": sum(host[k].numel() * host[k].element_size() for k in names),
-               "d2h_bytes_per_step": B * 4, "ms_per_step": e_ms, "steps": e_steps}
+               "h2d_bytes_per_step": hs.h2d_bytes(), "d2h_bytes_per_step": hs.d2h_bytes(),
+               "ms_per_step": e_ms, "steps": e_steps,
+               "inputs": "double-buffered: a step's copies overlap the previous step's kernels"}
+        del hs
     if rank != 0:
         return
     peak, peak_kind = peaks()

@@ -254,7 +254,21 @@ def verify_paths(draft, target, tokens, u_accept, u_correct, K, D, T, ref_logkap
     return o
 
 
-def verify_tree(draft, target, parent, tokens, u_accept, u_correct, T, workspace=None):
+def tree_outputs(B, N, device):
+    """Output tensors of verify_tree, to pass as out= and reuse across calls."""
+    f = dict(device=device)
+    return dict(alpha=torch.empty(B, N, dtype=torch.float32, **f),
+                accept=torch.empty(B, N, dtype=torch.uint8, **f),
+                path_accept=torch.empty(B, N, dtype=torch.uint8, **f),
+                logkappa=torch.empty(B, N, dtype=torch.float32, **f),
+                corr_tokens=torch.empty(B, N, dtype=torch.int32, **f),
+                deepest=torch.empty(B, dtype=torch.int32, **f),
+                accept_len=torch.empty(B, dtype=torch.int32, **f),
+                bonus=torch.empty(B, dtype=torch.int32, **f),
+                row_stats=torch.empty(B * N, 4, dtype=torch.float32, **f))
+
+
+def verify_tree(draft, target, parent, tokens, u_accept, u_correct, T, workspace=None, out=None):
     """Tree verification (App. E tree, Eq. 1 per node, Sec. 3 residual)."""
     _need_cuda(draft, target, parent, tokens, u_accept, u_correct)
     V = draft.shape[-1]
@@ -262,16 +276,7 @@ def verify_tree(draft, target, parent, tokens, u_accept, u_correct, T, workspace
     lay = layout(B, V=V, N=N, parent=parent)
     dev = draft.device
     ws = _ws(workspace, lay, dev)
-    f = dict(device=dev)
-    o = dict(alpha=torch.empty(B, N, dtype=torch.float32, **f),
-             accept=torch.empty(B, N, dtype=torch.uint8, **f),
-             path_accept=torch.empty(B, N, dtype=torch.uint8, **f),
-             logkappa=torch.empty(B, N, dtype=torch.float32, **f),
-             corr_tokens=torch.empty(B, N, dtype=torch.int32, **f),
-             deepest=torch.empty(B, dtype=torch.int32, **f),
-             accept_len=torch.empty(B, dtype=torch.int32, **f),
-             bonus=torch.empty(B, dtype=torch.int32, **f),
-             row_stats=torch.empty(B * N, 4, dtype=torch.float32, **f))
+    o = out if out is not None else tree_outputs(B, N, dev)
     st = TreeOutputs(*[o[n].data_ptr() for n in TREE_FIELDS])
     _check(_lib().vsd_verify_paths(_ptr(draft), _ptr(target), _dtype_code(draft), lay, float(T),
                                    _ptr(tokens), _ptr(u_accept), _ptr(u_correct), None, None,
@@ -406,34 +411,147 @@ def device_status(workspace):
     return code, bits.value
 
 
+class _Feeder:
+    """Two device copies of a step's inputs.  Each step queues the
+    host-to-device copies of its inputs on a copy stream, into the copy the
+    step before last used (after that step's kernels were queued), and the
+    caller's stream waits for them; so the copies of one step run while the
+    kernels of the step before it do."""
+
+    def __init__(self, shapes, device):
+        self.dev = torch.device(device)
+        self.stream = torch.cuda.Stream(device=self.dev)
+        self.bufs = []
+        for _ in range(2):
+            b = {k: torch.empty(sh, dtype=dt, device=self.dev) for k, (sh, dt) in shapes.items()}
+            for t in b.values():
+                t.record_stream(self.stream)
+            self.bufs.append(b)
+        self.copied = [torch.cuda.Event() for _ in range(2)]
+        self.released = [None, None]
+        self.n = 0
+
+    def nbytes(self):
+        return sum(t.numel() * t.element_size() for t in self.bufs[0].values())
+
+    def feed(self, host):
+        """Queue the copies of host (pinned tensors by name); returns the slot
+        and its device tensors, ready on the caller's stream."""
+        s = self.n % 2
+        self.n += 1
+        with torch.cuda.stream(self.stream):
+            if self.released[s] is not None:
+                self.stream.wait_event(self.released[s])
+            for k, h in host.items():
+                self.bufs[s][k].copy_(h, non_blocking=True)
+            self.copied[s].record(self.stream)
+        torch.cuda.current_stream(self.dev).wait_event(self.copied[s])
+        return s, self.bufs[s]
+
+    def release(self, s):
+        """The kernels reading slot s have been queued on the caller's stream."""
+        ev = torch.cuda.Event()
+        ev.record(torch.cuda.current_stream(self.dev))
+        self.released[s] = ev
+
+
 class HostStep:
-    """End-to-end E-step + M-step from pinned host tensors: per call, copy the
-    inputs to the device, run the fused kernel, read the loss back."""
+    """End-to-end E-step + M-step from pinned host tensors: each call copies
+    its inputs to the device (double-buffered, overlapping the previous call's
+    kernel), runs the fused kernel and queues the read-back of the loss.  The
+    returned pinned loss tensor is valid after a synchronise and until the
+    call after next."""
 
     def __init__(self, B, K, D, V, dtype, device, prm=None, full=False):
         self.B, self.K, self.D, self.V = B, K, D, V
         R = B * K * D
         self.dev = torch.device(device)
-        self.draft = torch.empty(R, V, dtype=dtype, device=self.dev)
-        self.target = torch.empty(R, V, dtype=dtype, device=self.dev)
-        self.u = torch.empty(3, R, dtype=torch.float32, device=self.dev)
-        self.prm = prm or params(like=self.draft)
+        self.feed = _Feeder(dict(draft=((R, V), dtype), target=((R, V), dtype),
+                                 u=((3, R), torch.float32)), self.dev)
+        self.prm = prm or params(like=self.feed.bufs[0]["draft"])
         gdt = torch.bfloat16 if self.prm.grad_dtype == VSD_BF16 else torch.float32
         self.out = linear_outputs(B, K, D, V, self.dev, grad_dtype=gdt, full=full)
         self.ws = new_workspace(layout(B, K, D, V), self.dev)
-        self.loss_host = torch.empty(B + 1, dtype=torch.float32).pin_memory()
+        self.loss_host = [torch.empty(B + 1, dtype=torch.float32).pin_memory() for _ in range(2)]
 
     def h2d_bytes(self):
-        return (self.draft.numel() * self.draft.element_size() * 2 + self.u.numel() * 4)
+        return self.feed.nbytes()
 
     def d2h_bytes(self):
-        return self.loss_host.numel() * 4
+        return self.loss_host[0].numel() * 4
 
     def __call__(self, h_draft, h_target, h_u, T):
-        self.draft.copy_(h_draft, non_blocking=True)
-        self.target.copy_(h_target, non_blocking=True)
-        self.u.copy_(h_u, non_blocking=True)
-        estep_mstep(self.draft, self.target, self.u[0], self.u[1], self.u[2], self.K, self.D, T,
+        s, d = self.feed.feed(dict(draft=h_draft, target=h_target, u=h_u))
+        estep_mstep(d["draft"], d["target"], d["u"][0], d["u"][1], d["u"][2], self.K, self.D, T,
                     prm=self.prm, workspace=self.ws, out=self.out)
-        self.loss_host.copy_(self.out["loss"], non_blocking=True)
-        return self.loss_host
+        self.feed.release(s)
+        self.loss_host[s].copy_(self.out["loss"], non_blocking=True)
+        return self.loss_host[s]
+
+
+class HostLMHeadStep:
+    """HostStep for the LM head fused with the E-step + M-step: per call the
+    hidden states, target logits and uniforms come from pinned host tensors
+    (double-buffered); the LM-head weight stays on the device."""
+
+    def __init__(self, weight, B, K, D, V, prm=None, full=True):
+        self.B, self.K, self.D, self.V = B, K, D, V
+        R, H = B * K * D, weight.shape[1]
+        self.dev = weight.device
+        self.weight = weight
+        self.feed = _Feeder(dict(hidden=((R, H), torch.bfloat16), target=((R, V), torch.bfloat16),
+                                 u=((3, R), torch.float32)), self.dev)
+        self.prm = prm or params(grad_dtype=torch.bfloat16)
+        gdt = torch.bfloat16 if self.prm.grad_dtype == VSD_BF16 else torch.float32
+        self.out = linear_outputs(B, K, D, V, self.dev, grad_dtype=gdt, full=full)
+        self.ws = new_workspace(layout(B, K, D, V), self.dev)
+        self.logits = torch.empty(R, V, dtype=torch.bfloat16, device=self.dev)
+        self.loss_host = [torch.empty(B + 1, dtype=torch.float32).pin_memory() for _ in range(2)]
+
+    def h2d_bytes(self):
+        return self.feed.nbytes()
+
+    def d2h_bytes(self):
+        return self.loss_host[0].numel() * 4
+
+    def __call__(self, h_hidden, h_target, h_u, T):
+        s, d = self.feed.feed(dict(hidden=h_hidden, target=h_target, u=h_u))
+        lmhead_estep_mstep(d["hidden"], self.weight, d["target"], d["u"][0], d["u"][1],
+                           d["u"][2], self.K, self.D, T, prm=self.prm, workspace=self.ws,
+                           out=self.out, draft_logits=self.logits)
+        self.feed.release(s)
+        self.loss_host[s].copy_(self.out["loss"], non_blocking=True)
+        return self.loss_host[s]
+
+
+class HostTreeStep:
+    """HostStep for tree verification: per call the logits, the tree and the
+    uniforms come from pinned host tensors (double-buffered); the accepted
+    lengths are read back."""
+
+    def __init__(self, B, N, V, dtype, device):
+        self.B, self.N, self.V = B, N, V
+        self.dev = torch.device(device)
+        i32, f32 = torch.int32, torch.float32
+        self.feed = _Feeder(dict(draft=((B * N, V), dtype), target=((B * N, V), dtype),
+                                 parent=((B, N), i32), tokens=((B, N), i32),
+                                 u_accept=((B, N), f32), u_correct=((B, N), f32)), self.dev)
+        self.ws = new_workspace(layout(B, V=V, N=N, parent=self.feed.bufs[0]["parent"]), self.dev)
+        self.out = tree_outputs(B, N, self.dev)
+        self.len_host = [torch.empty(B, dtype=i32).pin_memory() for _ in range(2)]
+
+    def h2d_bytes(self):
+        return self.feed.nbytes()
+
+    def d2h_bytes(self):
+        return self.len_host[0].numel() * 4
+
+    def __call__(self, host, T):
+        """host: pinned tensors draft, target, parent, tokens, u_accept, u_correct."""
+        s, d = self.feed.feed(host)
+        verify_tree(d["draft"], d["target"], d["parent"], d["tokens"], d["u_accept"],
+                    d["u_correct"], T, workspace=self.ws, out=self.out)
+        self.feed.release(s)
+        self.len_host[s].copy_(self.out["accept_len"], non_blocking=True)
+        return self.len_host[s]
+
