@@ -577,10 +577,13 @@ def run_tree(args):
     R = B * N
     T = 1.0
     ws = vsd.new_workspace(vsd.layout(B, V=V, N=N, parent=prob["parent"]), dev)
+    # the verification outputs; no per-row statistics, so leaf rows are read
+    # only where a bonus token needs one
+    tout = vsd.tree_outputs(B, N, dev, row_stats=False)
 
     def step(i):
         return vsd.verify_tree(prob["draft"], prob["target"], prob["parent"], prob["tokens"],
-                               prob["u_accept"], prob["u_correct"], T, workspace=ws)
+                               prob["u_accept"], prob["u_correct"], T, workspace=ws, out=tout)
 
     def barrier():
         multirank.barrier(world, dev)
@@ -640,7 +643,18 @@ def run_tree(args):
         return
     peak, peak_kind = peaks()
     elem = prob["draft"].element_size()
-    alg = 2 * R * V * elem + R * 16  # both logit rows once; token, parent, two uniforms
+    # rows the outputs need: both logit rows of every node with children, and
+    # of the deepest accepted node when it is a leaf (its bonus token)
+    par = prob["parent"].cpu()
+    has_kids = torch.zeros(B, N, dtype=torch.bool)
+    for b in range(B):
+        kids = par[b, 1:]
+        has_kids[b, kids[kids >= 0].long()] = True
+    deepest = tout["deepest"].cpu()
+    leaf_bonus = sum(1 for b in range(B)
+                     if deepest[b] >= 0 and not bool(has_kids[b, int(deepest[b])]))
+    rows_read = int(has_kids.sum()) + leaf_bonus
+    alg = 2 * rows_read * V * elem + R * 16  # those rows once; token, parent, two uniforms
     achieved = alg / (launch_ms / 1e3) / 1e9
     line = {
         "metric": METRIC, "value": multirank.job_rate(R, world, ms), "unit": "rows/s", "n_gpus": world,
@@ -650,7 +664,8 @@ def run_tree(args):
         "data": "synthetic (seeded; EAGLE-2-style trees, spiked logits)",
         "config": {"workload": "tree60", "B": B, "N": N, "V": V, "logits": "bf16",
                    "temperatures": [T], "l2": "inputs larger than L2 (no flush)",
-                   "rows_per_gpu": R},
+                   "rows_per_gpu": R, "row_stats": "not requested",
+                   "rows_read": rows_read},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
                      "kernel": "k_tree_fused",

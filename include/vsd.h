@@ -126,7 +126,11 @@ typedef struct {
     int32_t* accept_len;    /* [B] depth of that node                                    */
     int32_t* bonus;         /* [B] token after the accepted path: the residual of the
                                deepest node's first child, or a p-sample at its row      */
-    float* row_stats;       /* optional [B*N][4] as in vsd_linear_outputs                */
+    float* row_stats;       /* optional [B*N][4] as in vsd_linear_outputs; when NULL
+                               the rows of leaves are not read (a leaf's row enters
+                               the results only through the bonus token, for which
+                               the deepest accepted leaf's row is read), and a leaf
+                               row's invalid values then set no status bit        */
 } vsd_tree_outputs;
 
 /* Bytes of device workspace the calls below need for `layout` (0 if invalid). */

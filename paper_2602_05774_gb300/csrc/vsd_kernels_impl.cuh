@@ -465,7 +465,8 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
 // ------------------------------------------------------------ fused tree kernel
 // Tree verification in one launch of plain 128-thread blocks, R + tail
 // blocks.  Each block first takes a ticket: a ticket below R is a node row
-// (its tables and p-draw, then its children's acceptance); the block completing a
+// (its tables and p-draw, then its children's acceptance; a leaf's row is
+// skipped unless row statistics are requested); the block completing a
 // tree's last row runs the per-node pass for that tree (its shared memory is
 // the idle ring) and queues the tree's residual rows.  After its row a block
 // takes queued residual rows (the rejected children's draws) while any are
@@ -498,11 +499,33 @@ __device__ int claim_residual(const Problem<T>& P, bool wait) {
     }
 }
 
+// The bonus token of tree b (block).  When the deepest accepted node is a
+// leaf and the leaf rows were not read (no row statistics requested), its
+// row's pass runs now: the bonus is that row's p-draw.
+template <typename T, bool VEC>
+__device__ void tree_bonus_block(const Problem<T>& P, int b, Ring* rg, float4* tab,
+                                 RowShared& sh, int* s_row) {
+    const int N = P.N, n0 = b * N;
+    if (threadIdx.x == 0) {
+        const int best = ld_cg(P.tout.deepest + b);
+        const int child = best >= 0 ? ld_cg(P.tlist + n0 + N - 1) : 0;
+        *s_row = (best >= 0 && child < 0 && !P.tout.row_stats) ? n0 + best : -1;
+    }
+    __syncthreads();
+    const int r = *s_row;
+    if (r >= 0) {
+        row_pass<T, VEC, true, kNoToken, false>(P, r, rg, tab, sh);
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) tree_bonus<T>(P, b);
+    __syncthreads();
+}
+
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ RowShared sh;
-    __shared__ int s_t, s_last, s_tok;
+    __shared__ int s_t, s_last, s_tok, s_row;
     Ring* rg;
     float4* tab;
     smem_views<VEC>(dsm, rg, tab);
@@ -517,11 +540,18 @@ __global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
     __syncthreads();
     const int t = s_t;
     if (t < P.R) {
-        const int b = t / N;
-        row_pass<T, VEC, true, kNoToken, false>(P, t, rg, tab, sh);
-        __syncthreads();
-        tree_children<T>(P, b, t - b * N);
-        __syncthreads();
+        const int b = t / N, u = t - b * N;
+        // A leaf's row is needed only for the bonus token (taken later if at
+        // all) and for the row statistics output.
+        int need = P.tout.row_stats != nullptr;
+        for (int n = u + 1 + threadIdx.x; n < N && !need; n += kThreads)
+            need = __ldg(P.parent + (int64_t)b * N + n) == u;
+        if (__syncthreads_or(need)) {
+            row_pass<T, VEC, true, kNoToken, false>(P, t, rg, tab, sh);
+            __syncthreads();
+            tree_children<T>(P, b, u);
+            __syncthreads();
+        }
         if (threadIdx.x == 0) {
             __threadfence();
             s_last = atomicAdd(P.path_cnt + b, 1) == N - 1;
@@ -531,16 +561,19 @@ __global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
         if (s_last) {
             tree_nodes<T>(P, b, *tsh);
             __syncthreads();
-            if (threadIdx.x == 0) {
-                const int cnt = ld_cg(P.tcount + b);
-                if (cnt == 0) {
-                    tree_bonus<T>(P, b);
+            if (threadIdx.x == 0) s_row = ld_cg(P.tcount + b);
+            __syncthreads();
+            const int cnt = s_row;
+            __syncthreads();
+            if (cnt == 0) {
+                tree_bonus_block<T, VEC>(P, b, rg, tab, sh, &s_row);
+                if (threadIdx.x == 0) {
                     __threadfence();
                     atomicAdd(P.prefix_done, 1);
-                } else {  // queue the tree's residual rows (list positions)
-                    publish_residuals(P.resq_tail, P.resq_avail, P.resq_flag, P.resq, b * N,
-                                      cnt, true);
                 }
+            } else if (threadIdx.x == 0) {  // queue the tree's residual rows (list positions)
+                publish_residuals(P.resq_tail, P.resq_avail, P.resq_flag, P.resq, b * N, cnt,
+                                  true);
             }
             __syncthreads();
         }
@@ -555,9 +588,13 @@ __global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
         tree_residual_row<T, VEC>(P, b, ld_cg(P.tlist + item), rg, tab, &s_tok);
         if (threadIdx.x == 0) {
             __threadfence();
-            if (atomicAdd(P.res_seg_cnt + b, 1) == ld_cg(P.tcount + b) - 1) {
-                __threadfence();
-                tree_bonus<T>(P, b);
+            s_last = atomicAdd(P.res_seg_cnt + b, 1) == ld_cg(P.tcount + b) - 1;
+            if (s_last) __threadfence();
+        }
+        __syncthreads();
+        if (s_last) {
+            tree_bonus_block<T, VEC>(P, b, rg, tab, sh, &s_row);
+            if (threadIdx.x == 0) {
                 __threadfence();
                 atomicAdd(P.prefix_done, 1);
             }

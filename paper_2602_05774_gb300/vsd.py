@@ -254,18 +254,22 @@ def verify_paths(draft, target, tokens, u_accept, u_correct, K, D, T, ref_logkap
     return o
 
 
-def tree_outputs(B, N, device):
-    """Output tensors of verify_tree, to pass as out= and reuse across calls."""
+def tree_outputs(B, N, device, row_stats=True):
+    """Output tensors of verify_tree, to pass as out= and reuse across calls.
+    Without row_stats the kernel reads no leaf row but the one a bonus token
+    may need."""
     f = dict(device=device)
-    return dict(alpha=torch.empty(B, N, dtype=torch.float32, **f),
-                accept=torch.empty(B, N, dtype=torch.uint8, **f),
-                path_accept=torch.empty(B, N, dtype=torch.uint8, **f),
-                logkappa=torch.empty(B, N, dtype=torch.float32, **f),
-                corr_tokens=torch.empty(B, N, dtype=torch.int32, **f),
-                deepest=torch.empty(B, dtype=torch.int32, **f),
-                accept_len=torch.empty(B, dtype=torch.int32, **f),
-                bonus=torch.empty(B, dtype=torch.int32, **f),
-                row_stats=torch.empty(B * N, 4, dtype=torch.float32, **f))
+    o = dict(alpha=torch.empty(B, N, dtype=torch.float32, **f),
+             accept=torch.empty(B, N, dtype=torch.uint8, **f),
+             path_accept=torch.empty(B, N, dtype=torch.uint8, **f),
+             logkappa=torch.empty(B, N, dtype=torch.float32, **f),
+             corr_tokens=torch.empty(B, N, dtype=torch.int32, **f),
+             deepest=torch.empty(B, dtype=torch.int32, **f),
+             accept_len=torch.empty(B, dtype=torch.int32, **f),
+             bonus=torch.empty(B, dtype=torch.int32, **f))
+    if row_stats:
+        o["row_stats"] = torch.empty(B * N, 4, dtype=torch.float32, **f)
+    return o
 
 
 def verify_tree(draft, target, parent, tokens, u_accept, u_correct, T, workspace=None, out=None):
@@ -277,7 +281,7 @@ def verify_tree(draft, target, parent, tokens, u_accept, u_correct, T, workspace
     dev = draft.device
     ws = _ws(workspace, lay, dev)
     o = out if out is not None else tree_outputs(B, N, dev)
-    st = TreeOutputs(*[o[n].data_ptr() for n in TREE_FIELDS])
+    st = TreeOutputs(*[o[n].data_ptr() if o.get(n) is not None else None for n in TREE_FIELDS])
     _check(_lib().vsd_verify_paths(_ptr(draft), _ptr(target), _dtype_code(draft), lay, float(T),
                                    _ptr(tokens), _ptr(u_accept), _ptr(u_correct), None, None,
                                    C.byref(st), _ptr(ws), ws.numel(), _stream(dev)),
@@ -537,7 +541,7 @@ class HostTreeStep:
                                  parent=((B, N), i32), tokens=((B, N), i32),
                                  u_accept=((B, N), f32), u_correct=((B, N), f32)), self.dev)
         self.ws = new_workspace(layout(B, V=V, N=N, parent=self.feed.bufs[0]["parent"]), self.dev)
-        self.out = tree_outputs(B, N, self.dev)
+        self.out = tree_outputs(B, N, self.dev, row_stats=False)
         self.len_host = [torch.empty(B, dtype=i32).pin_memory() for _ in range(2)]
 
     def h2d_bytes(self):

@@ -179,10 +179,11 @@ def test_tree60_matches_oracle(vsd, oracle):
     orc = oracle.tree(_np32(prob["draft"]), _np32(prob["target"]), 1.0, prob["parent"].numpy(),
                       prob["tokens"].numpy(), _np32(prob["u_accept"]), _np32(prob["u_correct"]))
     p = to_cuda(prob)
-    g = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"], p["u_accept"],
-                        p["u_correct"], 1.0)
-    torch.cuda.synchronize()
-    compare_tree(g, orc)
+    for stats in (True, False):  # without row statistics leaf rows are not read
+        g = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"], p["u_accept"],
+                            p["u_correct"], 1.0, out=vsd.tree_outputs(B, N, "cuda", stats))
+        torch.cuda.synchronize()
+        compare_tree(g, orc)
 
 
 def test_small_trees_matches_oracle(vsd, oracle):
@@ -194,10 +195,12 @@ def test_small_trees_matches_oracle(vsd, oracle):
                           prob["parent"].numpy(), prob["tokens"].numpy(),
                           _np32(prob["u_accept"]), _np32(prob["u_correct"]))
         p = to_cuda(prob)
-        g = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"], p["u_accept"],
-                            p["u_correct"], 0.9)
-        torch.cuda.synchronize()
-        compare_tree(g, orc)
+        for stats in (True, False):
+            g = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"],
+                                p["u_accept"], p["u_correct"], 0.9,
+                                out=vsd.tree_outputs(B, N, "cuda", stats))
+            torch.cuda.synchronize()
+            compare_tree(g, orc)
 
 
 
@@ -232,12 +235,15 @@ def test_tree_edge_shapes(vsd, oracle):
                           prob["parent"].numpy(), prob["tokens"].numpy(),
                           _np32(prob["u_accept"]), _np32(prob["u_correct"]))
         p = to_cuda(prob)
-        g = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"], p["u_accept"],
-                            p["u_correct"], 1.0)
-        torch.cuda.synchronize()
-        compare_tree(g, orc)
-        if i == 2:  # the chain: every node accepted, so the accepted length is N - 1
-            assert (g["accept_len"].cpu() == 7).all()
+        B, N = prob["parent"].shape
+        for stats in (True, False):  # without row statistics leaf rows are not read
+            g = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"],
+                                p["u_accept"], p["u_correct"], 1.0,
+                                out=vsd.tree_outputs(B, N, "cuda", stats))
+            torch.cuda.synchronize()
+            compare_tree(g, orc)
+            if i == 2:  # the chain: every node accepted, so the accepted length is N - 1
+                assert (g["accept_len"].cpu() == 7).all()
 
 
 @pytest.mark.parametrize("T", [1.0, 0.7])
