@@ -499,33 +499,11 @@ __device__ int claim_residual(const Problem<T>& P, bool wait) {
     }
 }
 
-// The bonus token of tree b (block).  When the deepest accepted node is a
-// leaf and the leaf rows were not read (no row statistics requested), its
-// row's pass runs now: the bonus is that row's p-draw.
-template <typename T, bool VEC>
-__device__ void tree_bonus_block(const Problem<T>& P, int b, Ring* rg, float4* tab,
-                                 RowShared& sh, int* s_row) {
-    const int N = P.N, n0 = b * N;
-    if (threadIdx.x == 0) {
-        const int best = ld_cg(P.tout.deepest + b);
-        const int child = best >= 0 ? ld_cg(P.tlist + n0 + N - 1) : 0;
-        *s_row = (best >= 0 && child < 0 && !P.tout.row_stats) ? n0 + best : -1;
-    }
-    __syncthreads();
-    const int r = *s_row;
-    if (r >= 0) {
-        row_pass<T, VEC, true, kNoToken, false>(P, r, rg, tab, sh);
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) tree_bonus<T>(P, b);
-    __syncthreads();
-}
-
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ RowShared sh;
-    __shared__ int s_t, s_last, s_tok, s_row;
+    __shared__ int s_t, s_last, s_tok, s_cnt, s_leaf;
     Ring* rg;
     float4* tab;
     smem_views<VEC>(dsm, rg, tab);
@@ -561,19 +539,39 @@ __global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
         if (s_last) {
             tree_nodes<T>(P, b, *tsh);
             __syncthreads();
-            if (threadIdx.x == 0) s_row = ld_cg(P.tcount + b);
+            if (threadIdx.x == 0) {
+                const int cnt = ld_cg(P.tcount + b);
+                const int best = ld_cg(P.tout.deepest + b);
+                const int child = best >= 0 ? ld_cg(P.tlist + b * N + N - 1) : 0;
+                // a leaf's row not read yet that the bonus token needs
+                const int leaf = (best >= 0 && child < 0 && !P.tout.row_stats) ? b * N + best : -1;
+                s_cnt = cnt;
+                s_leaf = leaf;
+                if (cnt > 0) {  // queue the tree's residual rows (list positions)
+                    // the leaf's row pass here counts as one more of the tree's items
+                    if (leaf >= 0) atomicSub(P.res_seg_cnt + b, 1);
+                    publish_residuals(P.resq_tail, P.resq_avail, P.resq_flag, P.resq, b * N,
+                                      cnt, true);
+                }
+            }
             __syncthreads();
-            const int cnt = s_row;
-            __syncthreads();
-            if (cnt == 0) {
-                tree_bonus_block<T, VEC>(P, b, rg, tab, sh, &s_row);
-                if (threadIdx.x == 0) {
+            const int cnt = s_cnt, leaf = s_leaf;
+            if (leaf >= 0) {  // while other blocks take the residual rows
+                row_pass<T, VEC, true, kNoToken, false>(P, leaf, rg, tab, sh);
+                __syncthreads();
+            }
+            if (threadIdx.x == 0) {
+                bool done = cnt == 0;
+                if (!done && leaf >= 0) {
+                    __threadfence();
+                    done = atomicAdd(P.res_seg_cnt + b, 1) == cnt - 1;
+                }
+                if (done) {
+                    __threadfence();
+                    tree_bonus<T>(P, b);
                     __threadfence();
                     atomicAdd(P.prefix_done, 1);
                 }
-            } else if (threadIdx.x == 0) {  // queue the tree's residual rows (list positions)
-                publish_residuals(P.resq_tail, P.resq_avail, P.resq_flag, P.resq, b * N, cnt,
-                                  true);
             }
             __syncthreads();
         }
@@ -588,13 +586,9 @@ __global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
         tree_residual_row<T, VEC>(P, b, ld_cg(P.tlist + item), rg, tab, &s_tok);
         if (threadIdx.x == 0) {
             __threadfence();
-            s_last = atomicAdd(P.res_seg_cnt + b, 1) == ld_cg(P.tcount + b) - 1;
-            if (s_last) __threadfence();
-        }
-        __syncthreads();
-        if (s_last) {
-            tree_bonus_block<T, VEC>(P, b, rg, tab, sh, &s_row);
-            if (threadIdx.x == 0) {
+            if (atomicAdd(P.res_seg_cnt + b, 1) == ld_cg(P.tcount + b) - 1) {
+                __threadfence();
+                tree_bonus<T>(P, b);
                 __threadfence();
                 atomicAdd(P.prefix_done, 1);
             }
