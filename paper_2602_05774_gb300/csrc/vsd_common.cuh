@@ -311,11 +311,6 @@ __device__ __forceinline__ double warp_sum(double v) {
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     return v;
 }
-__device__ __forceinline__ int warp_min(int v) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
-    return v;
-}
 // Inclusive prefix sum over the lanes of a warp.
 __device__ __forceinline__ float warp_incl_scan(float v, int lane) {
 #pragma unroll
