@@ -1,0 +1,52 @@
+"""bench.py's output contract, on CPU: the reference arm (the oracle timed on
+the host cores) prints one JSON line with the keys the driver reads, for every
+workload; under torchrun with two ranks only rank 0 prints it and both ranks
+exit 0."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+KEYS = ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+        "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config")
+
+
+def _run(args, timeout=240):
+    r = subprocess.run([sys.executable] + args, cwd=ROOT, capture_output=True, text=True,
+                       timeout=timeout)
+    assert r.returncode == 0, r.stderr[-2000:]
+    return [l for l in r.stdout.splitlines() if l.startswith("{")]
+
+
+@pytest.mark.parametrize("config", ["vocab128k", "tree60", "lmhead"])
+def test_reference_arm_json_line(config):
+    lines = _run(["bench.py", "--impl", "reference", "--config", config, "--steps", "1",
+                  "--warmup", "1"])
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for k in KEYS:
+        assert k in d, k
+    assert d["impl"] == "reference" and d["n_gpus"] == 1 and d["steps"] == 1
+    assert d["higher_is_better"] is True and d["value"] > 0
+    assert d["config"]["workload"] == config
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
+    assert isinstance(cb["sample"], str) and cb["sample"]
+    e = d["e2e"]
+    assert e["value"] == d["value"] and e["unit"] == d["unit"]
+    assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+
+
+def test_reference_arm_under_torchrun_prints_once():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    lines = _run(["-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+                  "--master-addr", "127.0.0.1", "--master-port", str(port), "bench.py",
+                  "--impl", "reference", "--steps", "1", "--warmup", "1"])
+    assert len(lines) == 1
+    assert json.loads(lines[0])["impl"] == "reference"
