@@ -14,6 +14,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -72,12 +73,20 @@ def tensor_peak():
         return 1900.0, "fallback"
 
 
+def _code_only(text):
+    """Source text without comments and with whitespace collapsed: the hash
+    below follows the code, not its comments."""
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
 def kernel_source_hash():
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2602_05774_gb300", "csrc")
     for f in sorted(os.listdir(csrc)):
-        h.update(open(os.path.join(csrc, f), "rb").read())
-    h.update(open(os.path.join(ROOT, "include", "vsd.h"), "rb").read())
+        h.update(_code_only(open(os.path.join(csrc, f)).read()).encode())
+    h.update(_code_only(open(os.path.join(ROOT, "include", "vsd.h")).read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -468,10 +468,12 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
 // (its tables and p-draw, then its children's acceptance; a leaf's row is
 // skipped unless row statistics are requested); the block completing a
 // tree's last row runs the per-node pass for that tree (its shared memory is
-// the idle ring) and queues the tree's residual rows.  After its row a block
-// takes queued residual rows (the rejected children's draws) while any are
-// ready; the block completing a tree's last residual row writes its bonus
-// token.  A block whose ticket is R or more was started after every row had
+// the idle ring), queues the tree's residual rows and, when the bonus token
+// needs the row of a leaf that was skipped, runs that row's pass itself as
+// one more of the tree's items.  After its row a block takes queued residual
+// rows (the rejected children's draws) while any are ready; the block
+// completing a tree's last item writes its bonus token.  A block whose
+// ticket is R or more was started after every row had
 // been claimed, so every job it may wait for is held by a running block: it
 // waits for residual rows (bounded, status bit on expiry) until every tree is
 // done.
