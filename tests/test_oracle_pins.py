@@ -398,6 +398,41 @@ def test_tree_acceptance_lattice(oracle):
     assert np.all(tr["deepest"][d == 1] == np.where(tr["path_accept"][d == 1, 1] == 1, 1, 2))
 
 
+def test_tree_residual_and_bonus_distributions(oracle):
+    """Root with two leaf children, dyadic rows, a lattice over the uniforms:
+    child 1 (token 0 at the root row, alpha = 1/2) is accepted half the time;
+    when it is rejected its correction token follows norm(max(0, p - q)) of
+    the root row; child 2 (alpha = 1) is always accepted; the bonus is the
+    p-draw at the deepest accepted node's row (a leaf here: child 1 if
+    accepted, else child 2), so it follows (P_B + P_UNI) / 2 (Sec. 3, App. E)."""
+    parent = np.array([-1, 0, 0], np.int32)
+    tok = np.array([0, 0, 2], np.int32)
+    rq = [Q4, Q4, Q4]
+    rp = [P_UNI, P_B, P_UNI]
+    M = 8
+    g = np.meshgrid(lattice(M), lattice(M), lattice(M), indexing="ij")
+    B = M ** 3
+    ua = np.zeros((B, 3), np.float32)
+    uc = np.zeros((B, 3), np.float32)
+    ua[:, 1] = g[0].ravel()
+    ua[:, 2] = 0.999
+    uc[:, 1] = g[1].ravel()
+    uc[:, 2] = g[2].ravel()
+    draft = np.tile(np.stack([logits(r) for r in rq]), (B, 1))
+    target = np.tile(np.stack([logits(r) for r in rp]), (B, 1))
+    tr = oracle.tree(draft, target, 1.0, np.tile(parent, (B, 1)), np.tile(tok, (B, 1)), ua, uc)
+    acc1 = tr["path_accept"][:, 1] == 1
+    assert acc1.mean() == 1 / 2 and (tr["path_accept"][:, 2] == 1).all()
+    assert (tr["accept_len"] == 1).all()
+    assert np.array_equal(tr["deepest"], np.where(acc1, 1, 2))
+    # residual of the root row: max(0, P_UNI - Q4) = (0, 0, 1/8, 1/8), normalised
+    c1 = tr["corr_tokens"][~acc1, 1]
+    assert np.array_equal(np.bincount(c1, minlength=4) / c1.size, [0, 0, 1 / 2, 1 / 2])
+    assert (tr["corr_tokens"][acc1, 1] == -1).all() and (tr["corr_tokens"][:, 2] == -1).all()
+    bonus = np.bincount(tr["bonus"], minlength=4) / B
+    assert np.array_equal(bonus, (P_B + P_UNI) / 2)
+
+
 # --------------------------------------------------------------------------
 # Sec. 4.4 theorems by brute force on a tabulated autoregressive toy model
 
