@@ -246,6 +246,40 @@ def test_tree_edge_shapes(vsd, oracle):
                 assert (g["accept_len"].cpu() == 7).all()
 
 
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_tree_lattice_residual_and_bonus(vsd, oracle, dtype):
+    """512 three-node trees (a root and two leaves) with dyadic rows and a
+    lattice of uniforms: every bonus token is a draw at a leaf's row (the leaf
+    row skipped without row statistics is read for it), and half the trees
+    draw a residual token at the root row."""
+    q4, uni, pb = [0.5, 0.25, 0.125, 0.125], [0.25] * 4, [0.125, 0.375, 0.25, 0.25]
+    rows_q = np.log(np.array([q4, q4, q4]))
+    rows_p = np.log(np.array([uni, pb, uni]))
+    M, N, V = 8, 3, 4
+    lat = (np.arange(M) + 0.5) / M
+    g = np.meshgrid(lat, lat, lat, indexing="ij")
+    B = M ** 3
+    ua = np.zeros((B, N), np.float32)
+    uc = np.zeros((B, N), np.float32)
+    ua[:, 1], ua[:, 2] = g[0].ravel(), 0.999
+    uc[:, 1], uc[:, 2] = g[1].ravel(), g[2].ravel()
+    prob = dict(B=B, N=N, V=V,
+                draft=torch.tensor(np.tile(rows_q, (B, 1)), dtype=torch.float32).to(dtype),
+                target=torch.tensor(np.tile(rows_p, (B, 1)), dtype=torch.float32).to(dtype),
+                parent=torch.tensor([[-1, 0, 0]] * B, dtype=torch.int32),
+                tokens=torch.tensor([[0, 0, 2]] * B, dtype=torch.int32),
+                u_accept=torch.from_numpy(ua), u_correct=torch.from_numpy(uc))
+    orc = oracle.tree(_np32(prob["draft"]), _np32(prob["target"]), 1.0, prob["parent"].numpy(),
+                      prob["tokens"].numpy(), ua, uc)
+    p = to_cuda(prob)
+    for stats in (True, False):
+        g_ = vsd.verify_tree(p["draft"], p["target"], p["parent"], p["tokens"], p["u_accept"],
+                             p["u_correct"], 1.0, out=vsd.tree_outputs(B, N, "cuda", stats))
+        torch.cuda.synchronize()
+        compare_tree(g_, orc)
+
+
 @pytest.mark.parametrize("T", [1.0, 0.7])
 def test_vocab128k_full_size_sampled_prefixes(vsd, oracle, T):
     """The benchmark's workload and launch; the oracle checks two sampled prefixes."""
