@@ -173,10 +173,19 @@ vsd_status vsd_weighted_loss_fwd_bwd(const void* draft, vsd_dtype dtype, vsd_lay
                                      const vsd_params* params, float* loss, void* grad,
                                      float* weights, void* ws, size_t ws_bytes, void* stream);
 
-/* The fused E-step + M-step: one persistent kernel runs sampling, verification,
- * utilities, weights, loss and gradient over all prefixes.  Required members
- * of `out`: tokens, accept_len, corr_tokens, logkappa, loss, grad; the rest are
- * optional.  Linear layout only. */
+/* The fused E-step + M-step (Algorithm 1, both steps, for all prefixes at
+ * once; Algorithm 2 as the oracle; Eqs. 1, 2, 11, beta, zeta, advance): one
+ * persistent kernel runs sampling, verification, utilities, weights, loss and
+ * gradient over all prefixes, with the results of vsd_sample_paths,
+ * vsd_verify_paths and vsd_weighted_loss_fwd_bwd.  Arguments as for those
+ * calls: draft, target [R][V] of `dtype`; u_draft, u_accept, u_correct [R];
+ * ref_logkappa optional [B][D]; params NULL for the defaults (App. F:
+ * w(l) = 1.05^l, tau = 0.2).  Required members of `out`: tokens, accept_len,
+ * corr_tokens, logkappa, loss, grad; the rest are optional.  Linear layout
+ * only.  Errors: VSD_ERR_INVALID_ARG for a bad shape, pointer, dtype or
+ * parameter, VSD_ERR_UNSUPPORTED for T = 0, VSD_ERR_WORKSPACE for a missing
+ * or small workspace, VSD_ERR_CUDA if a launch fails; data errors on the
+ * device go to the status word (vsd_device_status). */
 vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtype,
                            vsd_layout layout, float T, const float* u_draft,
                            const float* u_accept, const float* u_correct,
@@ -203,14 +212,23 @@ vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtyp
  *     contents (each call clears the part that must start at zero).  Calls that
  *     overlap on the GPU -- on different streams, or from different host
  *     threads -- race on it; order them on one stream.
- *   - The device status word of these calls lives in that array and is not
- *     exposed; argument and launch errors are returned as usual. */
+ *   - The address is looked up again when the device's context has changed
+ *     (after a cudaDeviceReset, for example).
+ *   - The device status word of these calls (timeouts, invalid rows) lives in
+ *     that array: read it with vsd_noalloc_device_status(); argument and
+ *     launch errors are returned as usual. */
 #define VSD_NOALLOC_SCRATCH_BYTES (32u << 20)
 vsd_status vsd_estep_mstep_noalloc(const void* draft, const void* target, vsd_dtype dtype,
                                    vsd_layout layout, float T, const float* u_draft,
                                    const float* u_accept, const float* u_correct,
                                    const float* ref_logkappa, const vsd_params* params,
                                    vsd_linear_outputs* out, void* stream);
+
+/* vsd_device_status() for the calls of vsd_estep_mstep_noalloc on the current
+ * device: waits for `stream`, then reads and clears the status word kept in
+ * the library's array into *status_bits (host).  Allocates nothing.  Same
+ * return codes as vsd_device_status(). */
+vsd_status vsd_noalloc_device_status(void* stream, int32_t* status_bits);
 
 /* The draft model's LM head, the layer that produces the draft logits q is
  * computed from (paper Sec. 5, implementation details: the draft head's output

@@ -47,27 +47,55 @@ class _TreeOut(C.Structure):
         "accept_len", "bonus", "margins")]
 
 
+def _bind(path):
+    """Load an oracle shared library and declare its entry points."""
+    lib_ = C.CDLL(path)
+    lib_.vso_linear.argtypes = [C.POINTER(_LinearIn), C.POINTER(_LinearOut)]
+    lib_.vso_linear.restype = C.c_int
+    lib_.vso_tree.argtypes = [C.POINTER(_TreeIn), C.POINTER(_TreeOut)]
+    lib_.vso_tree.restype = C.c_int
+    lib_.vso_log_softmax.argtypes = [C.c_void_p, C.c_int64, C.c_double, C.c_void_p]
+    lib_.vso_log_softmax.restype = C.c_double
+    lib_.vso_sample.argtypes = [C.c_void_p, C.c_int64, C.c_double, C.c_void_p]
+    lib_.vso_sample.restype = C.c_int64
+    lib_.vso_prefix_weights.argtypes = [
+        C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+        C.c_double, C.c_double, C.c_int, C.c_void_p]
+    lib_.vso_prefix_weights.restype = C.c_double
+    lib_.vso_prefix_objective.argtypes = [
+        C.c_void_p, C.c_int, C.c_int, C.c_int64, C.c_double, C.c_void_p, C.c_void_p,
+        C.c_void_p, C.c_double, C.c_int, C.c_void_p]
+    lib_.vso_prefix_objective.restype = C.c_double
+    lib_.vso_decision_margin.argtypes = [C.c_double, C.c_double, C.c_int, C.c_void_p,
+                                         C.c_void_p, C.c_void_p, C.c_void_p]
+    lib_.vso_decision_margin.restype = C.c_double
+    return lib_
+
+
 def lib():
     global _lib
     if _lib is None:
-        _lib = C.CDLL(build_oracle())
-        _lib.vso_linear.argtypes = [C.POINTER(_LinearIn), C.POINTER(_LinearOut)]
-        _lib.vso_linear.restype = C.c_int
-        _lib.vso_tree.argtypes = [C.POINTER(_TreeIn), C.POINTER(_TreeOut)]
-        _lib.vso_tree.restype = C.c_int
-        _lib.vso_log_softmax.argtypes = [C.c_void_p, C.c_int64, C.c_double, C.c_void_p]
-        _lib.vso_log_softmax.restype = C.c_double
-        _lib.vso_sample.argtypes = [C.c_void_p, C.c_int64, C.c_double, C.c_void_p]
-        _lib.vso_sample.restype = C.c_int64
-        _lib.vso_prefix_weights.argtypes = [
-            C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
-            C.c_double, C.c_double, C.c_int, C.c_void_p]
-        _lib.vso_prefix_weights.restype = C.c_double
-        _lib.vso_prefix_objective.argtypes = [
-            C.c_void_p, C.c_int, C.c_int, C.c_int64, C.c_double, C.c_void_p, C.c_void_p,
-            C.c_void_p, C.c_double, C.c_int, C.c_void_p]
-        _lib.vso_prefix_objective.restype = C.c_double
+        _lib = _bind(build_oracle())
     return _lib
+
+
+class using_library:
+    """Context manager that routes this module's functions to another build of
+    the oracle (the mutation test compiles deliberately broken copies of
+    vsd_oracle.c and checks that the pins reject each of them)."""
+
+    def __init__(self, path):
+        self.path = path
+
+    def __enter__(self):
+        global _lib
+        self.saved = lib()
+        _lib = _bind(self.path)
+        return self
+
+    def __exit__(self, *exc):
+        global _lib
+        _lib = self.saved
 
 
 def _f32(a):
@@ -157,6 +185,24 @@ def tree(draft, target, T, parent, tokens, u_accept, u_correct):
     if rc != 0:
         raise ValueError("oracle rejected the tree (code %d)" % rc)
     return o
+
+
+def decision_margin(a, b, ra, ta, rb=None, tb=None):
+    """Margin of the comparison log k(z_a) >= log k(z_b) of Algorithm 2, as the
+    parity protocol uses it: |a - b| for unequal sums; for equal sums the
+    smallest log-ratio log(p/q) at the positions where the two paths hold
+    different tokens if every one of them is >= 0 (so min(0, .) clips it and
+    the equality is exact), else 0; 0 for an equality with an input reference
+    other than 0 (rb = None).  ra, rb: log(p/q) per position."""
+    ra = np.ascontiguousarray(ra, dtype=np.float64).reshape(-1)
+    ta = _i32(ta).reshape(-1)
+    n = ra.size
+    if rb is not None:
+        rb = np.ascontiguousarray(rb, dtype=np.float64).reshape(-1)
+        tb = _i32(tb).reshape(-1)
+        assert rb.size == n and tb.size == n
+    return lib().vso_decision_margin(float(a), float(b), n, _ptr(ra), _ptr(ta), _ptr(rb),
+                                     _ptr(tb))
 
 
 def prefix_weights(logkappa, logkappa_corr, logkappa_ref, logq_path, w_base=1.05,

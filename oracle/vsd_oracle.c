@@ -587,3 +587,11 @@ int64_t vso_sample(const double* prob, int64_t V, double u, double* margin)
 {
     return sample_inverse_cdf(prob, V, u, margin);
 }
+
+/* The margin of one Algorithm 2 comparison (see decision_margin); rb and tb
+ * may be NULL (an input reference). */
+double vso_decision_margin(double a, double b, int n, const double* ra, const int32_t* ta,
+                           const double* rb, const int32_t* tb)
+{
+    return decision_margin(a, b, n, ra, ta, rb, tb);
+}

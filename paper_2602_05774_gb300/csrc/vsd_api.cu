@@ -5,6 +5,9 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <mutex>
+#include <vector>
+
 #include <cuda_runtime.h>
 
 #include "vsd.h"
@@ -118,12 +121,7 @@ template <typename U> U* at(void* ws, size_t off) {
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
-int num_sms() {
-    int dev = 0, n = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 1;
-    return n > 0 ? n : 1;
-}
+int num_sms() { return device_sm_count(); }
 
 vsd_status check_temperature(float T) {
     if (T == 0.f) return VSD_ERR_UNSUPPORTED;  // greedy decoding is not served here
@@ -260,6 +258,68 @@ bool vec_ok(const void* a, const void* b, const void* g, int V, size_t elem, siz
     return true;
 }
 
+
+// ------------------------------------------------------------ per-device caches
+std::mutex g_cache_mu;
+struct SmemEntry { const void* kernel; int dev; size_t smem; };
+struct OccEntry { const void* kernel; int dev; int threads; size_t smem; int blocks; };
+std::vector<SmemEntry> g_smem;
+std::vector<OccEntry> g_occ;
+int g_sms[256];
+
+}  // namespace
+
+int device_sm_count() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return 1;
+    std::lock_guard<std::mutex> lock(g_cache_mu);
+    if (g_sms[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+            return 1;
+        g_sms[dev] = n;
+    }
+    return g_sms[dev];
+}
+
+cudaError_t ensure_dyn_smem(const void* kernel, size_t smem) {
+    if (smem == 0) return cudaSuccess;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(g_cache_mu);
+    for (SmemEntry& x : g_smem)
+        if (x.kernel == kernel && x.dev == dev) {
+            if (x.smem >= smem) return cudaSuccess;
+            e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e == cudaSuccess) x.smem = smem;
+            return e;
+        }
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess) g_smem.push_back(SmemEntry{kernel, dev, smem});
+    return e;
+}
+
+int blocks_per_sm(const void* kernel, int threads, size_t smem) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    {
+        std::lock_guard<std::mutex> lock(g_cache_mu);
+        for (const OccEntry& x : g_occ)
+            if (x.kernel == kernel && x.dev == dev && x.threads == threads && x.smem == smem)
+                return x.blocks;
+    }
+    if (ensure_dyn_smem(kernel, smem) != cudaSuccess) return 0;
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, threads, smem) != cudaSuccess)
+        return 0;
+    std::lock_guard<std::mutex> lock(g_cache_mu);
+    g_occ.push_back(OccEntry{kernel, dev, threads, smem, n});
+    return n;
+}
+
+namespace {
+
 // ------------------------------------------------------------ entry bodies
 template <typename T>
 vsd_status sample_impl(const void* draft, vsd_layout L, float T_, const float* u_draft,
@@ -346,8 +406,6 @@ vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float
     const int64_t tickets = (int64_t)P.R * (P.nseg + P.gnseg);
     int ctas = per_sm * num_sms();
     if ((int64_t)ctas > tickets) ctas = (int)tickets;
-    const char* env_ctas = getenv("VSD_FUSED_CTAS");
-    if (env_ctas && atoi(env_ctas) > 0 && atoi(env_ctas) < ctas) ctas = atoi(env_ctas);
     cudaError_t e = clear ? clear_counters(ws, L, s) : cudaSuccess;
     if (e == cudaSuccess) e = Launch<T>::fused(P, vec, out->grad, P.grad_bf16, ctas, s);
     return from_cuda(e);
@@ -463,7 +521,8 @@ vsd_status vsd_lmhead_logits(const void* hidden, const void* weight, int32_t M, 
     if (!ws || ws_bytes < 256 || ((uintptr_t)ws & 255)) return VSD_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int32_t), s);
-    if (e == cudaSuccess) e = lmhead_gemm(hidden, weight, M, N, K, logits, static_cast<int*>(ws), s);
+    if (e == cudaSuccess)
+        e = lmhead_gemm(hidden, weight, M, N, K, logits, static_cast<int*>(ws), kDefaultTimeoutNs, s);
     return from_cuda(e);
 }
 
@@ -491,7 +550,8 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
     // the counters and the status word are cleared once, before both steps
     cudaError_t e = clear_counters(ws, layout, s);
     if (e == cudaSuccess)
-        e = lmhead_gemm(hidden, weight, (int)R, layout.V, H, draft_logits, static_cast<int*>(ws), s);
+        e = lmhead_gemm(hidden, weight, (int)R, layout.V, H, draft_logits, static_cast<int*>(ws),
+                        p.wait_timeout_ns ? p.wait_timeout_ns : kDefaultTimeoutNs, s);
     if (e != cudaSuccess) return from_cuda(e);
     return fused_impl<__nv_bfloat16>(draft_logits, target, layout, T, u_draft, u_accept,
                                      u_correct, ref_logkappa, p, out, ws, s, false);

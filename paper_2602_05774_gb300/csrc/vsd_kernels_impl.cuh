@@ -8,11 +8,12 @@ namespace vsd {
 
 // Dynamic shared memory: [Ring (vector rows)] [chunk table].
 template <bool VEC>
-__device__ __forceinline__ void smem_views(unsigned char* dsm, Ring*& rg, float4*& tab) {
+__device__ __forceinline__ void smem_views(unsigned char* dsm, Ring*& rg, float4*& tab,
+                                           uint64_t timeout_ns) {
     if (VEC) {
         rg = reinterpret_cast<Ring*>(dsm);
         tab = reinterpret_cast<float4*>(dsm + sizeof(Ring));
-        ring_init(rg);
+        ring_init(rg, timeout_ns);
     } else {
         rg = nullptr;
         tab = reinterpret_cast<float4*>(dsm);
@@ -26,7 +27,7 @@ __global__ void __launch_bounds__(kThreads) k_sample(Problem<T> P) {
     __shared__ RowShared sh;
     Ring* rg;
     float4* tab;
-    smem_views<VEC>(dsm, rg, tab);
+    smem_views<VEC>(dsm, rg, tab, P.timeout_ns);
     const int r = blockIdx.x;
     row_pass<T, VEC, false, kSampleToken, false>(P, r, rg, tab, sh);
     if (threadIdx.x == 0) {
@@ -45,7 +46,7 @@ __global__ void __launch_bounds__(kThreads) k_rows_verify(Problem<T> P) {
     __shared__ RowShared sh;
     Ring* rg;
     float4* tab;
-    smem_views<VEC>(dsm, rg, tab);
+    smem_views<VEC>(dsm, rg, tab, P.timeout_ns);
     row_pass<T, VEC, true, kGivenToken, true>(P, blockIdx.x, rg, tab, sh);
 }
 
@@ -55,7 +56,7 @@ __global__ void __launch_bounds__(kThreads) k_paths(Problem<T> P) {
     __shared__ PathShared sh;
     Ring* rg;
     float4* tab;
-    smem_views<VEC>(dsm, rg, tab);
+    smem_views<VEC>(dsm, rg, tab, P.timeout_ns);
     path_pass<T, VEC>(P, blockIdx.x, rg, tab, sh);
 }
 
@@ -390,7 +391,7 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
     __shared__ RowShared rsh;
     Ring* rg;
     float4* tab;
-    smem_views<VEC>(dsm, rg, tab);
+    smem_views<VEC>(dsm, rg, tab, P.timeout_ns);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (warp < kWarps) {  // ------------------------------- streaming warps
         for (int i = 0;; ++i) {
@@ -508,7 +509,7 @@ __global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
     __shared__ int s_t, s_last, s_tok, s_cnt, s_leaf;
     Ring* rg;
     float4* tab;
-    smem_views<VEC>(dsm, rg, tab);
+    smem_views<VEC>(dsm, rg, tab, P.timeout_ns);
     // The per-node pass runs between streams: on the vector path its shared
     // memory is the ring's data (no copy is in flight then), else it follows
     // the chunk table.
@@ -600,11 +601,11 @@ __global__ void __launch_bounds__(kThreads) k_tree_fused(Problem<T> P) {
 }
 
 // ------------------------------------------------------------ launchers
-// Static plus dynamic shared memory above 48 KB needs the kernel's opt-in.
+// Static plus dynamic shared memory above 48 KB needs the kernel's opt-in
+// (made once per kernel and device).
 template <typename K>
 static cudaError_t prep(K kernel, size_t smem) {
-    if (smem == 0) return cudaSuccess;
-    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    return ensure_dyn_smem(reinterpret_cast<const void*>(kernel), smem);
 }
 
 template <>
@@ -658,12 +659,7 @@ cudaError_t Launch<VSD_T>::tree(const Problem<VSD_T>& P, bool vec, cudaStream_t 
     auto kern = vec ? k_tree_fused<VSD_T, true> : k_tree_fused<VSD_T, false>;
     cudaError_t e = prep(kern, smem);
     if (e) return e;
-    int dev = 0, sms = 0;
-    e = cudaGetDevice(&dev);
-    if (e) return e;
-    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e) return e;
-    long long tail = (long long)sms * VSD_TREE_TAIL_PER_SM;
+    long long tail = (long long)device_sm_count() * VSD_TREE_TAIL_PER_SM;
     const long long most = (long long)P.B * (P.N - 1);  // residual rows at most
     if (tail > most) tail = most;
     if (tail < 1) tail = 1;
@@ -712,23 +708,12 @@ cudaError_t Launch<VSD_T>::fused(const Problem<VSD_T>& P, bool vec, void* grad, 
 template <>
 int Launch<VSD_T>::fused_blocks_per_sm(const Problem<VSD_T>& P, bool vec, bool grad_bf16) {
     const size_t smem = stream_smem_bytes(P.nch, vec);
-    // the attribute must allow this much before the occupancy query counts it
-    if (vec && grad_bf16) prep(k_fused<VSD_T, true, __nv_bfloat16>, smem);
-    else if (vec) prep(k_fused<VSD_T, true, float>, smem);
-    else if (grad_bf16) prep(k_fused<VSD_T, false, __nv_bfloat16>, smem);
-    else prep(k_fused<VSD_T, false, float>, smem);
-    int n = 0;
-    cudaError_t e;
-    if (vec && grad_bf16)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, true, __nv_bfloat16>, kFusedThreads, smem);
-    else if (vec)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, true, float>, kFusedThreads, smem);
-    else if (grad_bf16)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, false, __nv_bfloat16>, kFusedThreads, smem);
-    else
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_fused<VSD_T, false, float>, kFusedThreads, smem);
-    if (e != cudaSuccess || n < 1) return 1;
-    return n;
+    const void* k = vec ? (grad_bf16 ? reinterpret_cast<const void*>(k_fused<VSD_T, true, __nv_bfloat16>)
+                                     : reinterpret_cast<const void*>(k_fused<VSD_T, true, float>))
+                        : (grad_bf16 ? reinterpret_cast<const void*>(k_fused<VSD_T, false, __nv_bfloat16>)
+                                     : reinterpret_cast<const void*>(k_fused<VSD_T, false, float>));
+    const int n = blocks_per_sm(k, kFusedThreads, smem);
+    return n < 1 ? 1 : n;
 }
 
 template struct Launch<VSD_T>;

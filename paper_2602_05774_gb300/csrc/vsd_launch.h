@@ -31,6 +31,17 @@ template <typename T> struct Launch {
     static int fused_blocks_per_sm(const Problem<T>& P, bool vec, bool grad_bf16);
 };
 
+// Host-side per-device caches, so that a call makes no attribute or
+// occupancy query once a kernel has been set up on its device (vsd_api.cu).
+// The SM count of the current device.
+int device_sm_count();
+// Lets `kernel` use `smem` bytes of dynamic shared memory on the current
+// device (cudaFuncSetAttribute only when a larger size than before is asked).
+cudaError_t ensure_dyn_smem(const void* kernel, size_t smem);
+// Resident blocks per SM of `kernel` with `threads` threads and `smem` bytes
+// of dynamic shared memory on the current device (0 on error).
+int blocks_per_sm(const void* kernel, int threads, size_t smem);
+
 inline size_t table_smem_bytes(int nch) { return (size_t)nch * sizeof(float4); }
 // Dynamic shared memory of a streaming kernel: the TMA ring (vector rows
 // only) followed by the chunk table.
@@ -43,6 +54,6 @@ inline size_t stream_smem_bytes(int nch, bool vec) {
 bool lmhead_shape_ok(const void* hidden, const void* weight, const void* logits, int M, int N,
                      int K);
 cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, int K, void* logits,
-                        int* status, cudaStream_t s);
+                        int* status, uint64_t timeout_ns, cudaStream_t s);
 
 }  // namespace vsd

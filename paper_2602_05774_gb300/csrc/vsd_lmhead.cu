@@ -49,7 +49,6 @@ constexpr int kABytes = BM * BK * 2;  // 16 KB
 constexpr int kBBytes = BN * BK * 2;  // 32 KB
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kTmemCols = 2 * BN;  // two fp32 accumulators of 128 lanes x BN columns
-constexpr uint64_t kWaitNs = 2000000000ull;
 
 struct Bars {
     uint64_t full[kStages];   // TMA bytes landed in stage s
@@ -57,6 +56,7 @@ struct Bars {
     uint64_t acc_full[2];     // accumulator b holds a finished tile
     uint64_t acc_empty[2];    // the epilogue has read accumulator b (4 arrivals)
     uint64_t drain;           // the MMA warp's final commit
+    uint64_t timeout_ns;      // bound of every wait (the call's wait timeout)
     uint32_t tmem_base;
     int err;
 };
@@ -148,7 +148,7 @@ __device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity, Bars*
     for (;;) {
         if (mbar_try_wait(bar, parity)) return true;
         if (*(volatile int*)&sb->err) return false;
-        if (global_timer_ns() - t0 > kWaitNs) {
+        if (global_timer_ns() - t0 > sb->timeout_ns) {
             sb->err = 1;
             atomicOr(status, VSD_STATUS_TIMEOUT);
             return false;
@@ -158,10 +158,11 @@ __device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity, Bars*
 
 // Bounded wait that ignores the error flag (winding down after an error: the
 // copies and MMAs already issued must finish before the CTA exits).
-__device__ __forceinline__ void wait_phase_drain(uint64_t* bar, uint32_t parity) {
+__device__ __forceinline__ void wait_phase_drain(uint64_t* bar, uint32_t parity,
+                                                 uint64_t timeout_ns) {
     const uint64_t t0 = global_timer_ns();
     while (!mbar_try_wait(bar, parity))
-        if (global_timer_ns() - t0 > kWaitNs) return;
+        if (global_timer_ns() - t0 > timeout_ns) return;
 }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
@@ -178,7 +179,8 @@ __device__ __forceinline__ uint32_t pack_bf16(uint32_t lo, uint32_t hi) {
 // the hidden states stay in L2 throughout.
 __global__ void __launch_bounds__(kThreads, 1)
     k_lmhead(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-             __nv_bfloat16* __restrict__ out, int M, int N, int K, int* status) {
+             __nv_bfloat16* __restrict__ out, int M, int N, int K, int* status,
+             uint64_t timeout_ns) {
     extern __shared__ unsigned char dsm_raw[];
     unsigned char* dsm = dsm_raw + ((1024u - (smem_u32(dsm_raw) & 1023u)) & 1023u);
     Bars* sb = reinterpret_cast<Bars*>(dsm + kStages * kStageBytes);
@@ -196,6 +198,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_init(&sb->drain, 1);
         sb->err = 0;
+        sb->timeout_ns = timeout_ns;
         mbar_init_fence();
     }
     if (warp == 1) {  // the whole warp allocates the two accumulators
@@ -232,7 +235,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // the last copies issued have landed before the CTA may exit
             for (uint32_t j = it > (uint32_t)kStages ? it - kStages : 0; j < it; ++j)
-                wait_phase_drain(&sb->full[j % kStages], (j / kStages) & 1u);
+                wait_phase_drain(&sb->full[j % kStages], (j / kStages) & 1u, timeout_ns);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------ MMA issuer
@@ -267,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // every MMA this thread issued is complete once this arrives
             mma_commit(&sb->drain);
-            wait_phase_drain(&sb->drain, 0);
+            wait_phase_drain(&sb->drain, 0, timeout_ns);
         }
     } else {
         // ------------------------------------------------------ epilogue
@@ -364,7 +367,7 @@ bool lmhead_shape_ok(const void* hidden, const void* weight, const void* logits,
 }
 
 cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, int K, void* logits,
-                        int* status, cudaStream_t s) {
+                        int* status, uint64_t timeout_ns, cudaStream_t s) {
     using vsd_lm::k_lmhead;
     using vsd_lm::make_map;
     CUtensorMap ta, tb;
@@ -395,7 +398,7 @@ cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, in
     const int grid = (int)(ntiles < slots ? ntiles : slots);
     // (qualified: the enclosing namespace has a kThreads of its own)
     k_lmhead<<<grid, vsd_lm::kThreads, vsd_lm::kSmemBytes, s>>>(
-        ta, tb, static_cast<__nv_bfloat16*>(logits), M, N, K, status);
+        ta, tb, static_cast<__nv_bfloat16*>(logits), M, N, K, status, timeout_ns);
     return cudaGetLastError();
 }
 

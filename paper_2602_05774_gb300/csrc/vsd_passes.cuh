@@ -202,11 +202,13 @@ struct Ring {
     int pos2[kWarps];
     int pos1[kWarps];
     int broken[kWarps];  // a wait ran out: no further waits or copies in this block
+    uint64_t timeout_ns; // bound of every slot wait (the call's wait timeout)
 };
 
 // Every thread of the block calls it; warps beyond the streaming warps (the
 // fused kernel's control warp) own no ring slots.
-__device__ __forceinline__ void ring_init(Ring* rg) {
+__device__ __forceinline__ void ring_init(Ring* rg, uint64_t timeout_ns) {
+    if (threadIdx.x == 0) rg->timeout_ns = timeout_ns;
     if ((threadIdx.x & 31) == 0 && (threadIdx.x >> 5) < kWarps) {
         const int w = threadIdx.x >> 5;
         for (int st = 0; st < kStages; ++st) mbar_init(&rg->bar2[w][st], 1);
@@ -220,12 +222,13 @@ __device__ __forceinline__ void ring_init(Ring* rg) {
 }
 
 // Bounded wait on a slot; false (and the timeout status bit) if it ran out.
-__device__ __forceinline__ bool ring_wait(uint64_t* bar, uint32_t parity, int* status) {
+__device__ __forceinline__ bool ring_wait(uint64_t* bar, uint32_t parity, int* status,
+                                          uint64_t timeout_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     for (;;) {
         if (mbar_try_wait(bar, parity)) return true;
-        if (global_timer_ns() - t0 > 2000000000ull) {
+        if (global_timer_ns() - t0 > timeout_ns) {
             atomicOr(status, VSD_STATUS_TIMEOUT);
             return false;
         }
@@ -273,7 +276,7 @@ __device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, in
     for (int j = 0; j < nj; ++j) {
         const int slot = (pos + j) % NS;
         const uint32_t parity = (uint32_t)((pos + j) / NS) & 1u;
-        bool ok = broken ? false : ring_wait(&bars[slot], parity, status);
+        bool ok = broken ? false : ring_wait(&bars[slot], parity, status, rg->timeout_ns);
         broken = __any_sync(0xffffffffu, !ok);
         const int ch = cfirst + j * cstride;
         const int64_t e0 = (int64_t)ch * CE;

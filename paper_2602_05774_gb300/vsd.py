@@ -23,7 +23,7 @@ _STATUS_NAMES = {0: "VSD_OK", 1: "VSD_ERR_INVALID_ARG", 2: "VSD_ERR_UNSUPPORTED"
 SYMBOLS = ("vsd_workspace_bytes", "vsd_sample_paths", "vsd_verify_paths",
            "vsd_weighted_loss_fwd_bwd", "vsd_estep_mstep", "vsd_device_status",
            "vsd_status_string", "vsd_version", "vsd_estep_mstep_noalloc",
-           "vsd_lmhead_logits", "vsd_lmhead_estep_mstep")
+           "vsd_noalloc_device_status", "vsd_lmhead_logits", "vsd_lmhead_estep_mstep")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -97,11 +97,13 @@ def _lib():
                                                vp, vp, C.POINTER(Params), vp,
                                                C.POINTER(LinearOutputs), vp, C.c_size_t, vp]
         lib.vsd_device_status.argtypes = [vp, vp, C.POINTER(C.c_int32)]
+        lib.vsd_noalloc_device_status.argtypes = [vp, C.POINTER(C.c_int32)]
         lib.vsd_status_string.argtypes = [C.c_int]
         lib.vsd_status_string.restype = C.c_char_p
         lib.vsd_version.restype = C.c_char_p
         for name in ("vsd_sample_paths", "vsd_verify_paths", "vsd_weighted_loss_fwd_bwd",
                      "vsd_estep_mstep", "vsd_device_status", "vsd_estep_mstep_noalloc",
+                     "vsd_noalloc_device_status",
                      "vsd_lmhead_logits", "vsd_lmhead_estep_mstep"):
             getattr(lib, name).restype = C.c_int
         _LIB = lib
@@ -406,6 +408,15 @@ def estep_mstep_noalloc(draft, target, u_draft, u_accept, u_correct, K, D, T,
                                           _ptr(u_correct), _ptr(ref_logkappa), C.byref(prm),
                                           C.byref(st), _stream(dev)), "vsd_estep_mstep_noalloc")
     return out
+
+
+def noalloc_device_status(device=None):
+    """(status code, status bits) of the vsd_estep_mstep_noalloc calls on the
+    current device; synchronises the current stream."""
+    bits = C.c_int32(0)
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else device
+    code = _lib().vsd_noalloc_device_status(_stream(dev), C.byref(bits))
+    return code, bits.value
 
 
 def device_status(workspace):

@@ -17,3 +17,17 @@ def oracle():
     from oracle import oracle as o
     o.lib()
     return o
+
+
+def pytest_terminal_summary(terminalreporter):
+    """Report what the parity protocol excused in this run: decisions that
+    fell within the margin of their boundary, and prefixes (trees) excluded
+    because such a decision went the other way on the GPU."""
+    from tests.parity import SESSION
+    if SESSION["calls"] == 0 and SESSION["trees"] == 0:
+        return
+    terminalreporter.write_line(
+        "parity protocol: %d linear calls, %d prefixes compared, %d near-boundary decisions, "
+        "%d prefixes excluded; %d trees compared, %d trees excluded" % (
+            SESSION["calls"], SESSION["prefixes"], SESSION["near_boundary_decisions"],
+            SESSION["excluded_prefixes"], SESSION["trees"], SESSION["excluded_trees"]))

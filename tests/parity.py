@@ -20,6 +20,26 @@ LOGK_MARGIN = 1e-5
 LOSS_RTOL = 1e-5
 ALPHA_ATOL = 2e-6
 
+# Session-wide record of what the protocol excused, printed at the end of the
+# run (tests/conftest.py): near-boundary decisions seen and prefixes excluded.
+SESSION = {"calls": 0, "prefixes": 0, "near_boundary_decisions": 0, "excluded_prefixes": 0,
+           "trees": 0, "excluded_trees": 0}
+
+
+def exclusion_budget(B):
+    """How many prefixes (or trees) of one call may be excluded.
+
+    A prefix is excluded only when one of its decisions lies within the
+    margin of its boundary and the two sides took it differently.  With the
+    margins below, a decision falls inside one with probability of order
+    1e-5 on these inputs, so an exclusion is rare; the budget allows one per
+    ten prefixes (at least one for B >= 3) and none at all for B <= 2, so
+    that every call compares at least one prefix in full and a call whose
+    only prefixes are excluded fails."""
+    if B <= 2:
+        return 0
+    return max(1, B // 10)
+
 
 def to_np(t):
     if hasattr(t, "detach"):
@@ -84,12 +104,18 @@ def compare_linear(gpu, orc, B, K, D, V, T, grad_dtype="f32", check_grad=True, r
     rows_ok = np.repeat(ok, K * D)
     paths_ok = np.repeat(ok, K)
     nbad = int(div.sum())
+    m = orc["margins"]
+    near = int((np.minimum(np.minimum(m[:, 0], m[:, 1]), m[:, 2]) < PROB_MARGIN).sum()
+               + (np.minimum(m[:, 3], m[:, 4]) < LOGK_MARGIN).sum())
+    SESSION["calls"] += 1
+    SESSION["prefixes"] += B
+    SESSION["near_boundary_decisions"] += near
+    SESSION["excluded_prefixes"] += nbad
     if report is not None:
         report["excluded_prefixes"] = nbad
-        m = orc["margins"]
-        report["near_boundary_decisions"] = int((np.minimum(np.minimum(m[:, 0], m[:, 1]), m[:, 2])
-                                                 < PROB_MARGIN).sum())
-    assert nbad <= max(1, B // 8), "too many diverged prefixes: %d of %d" % (nbad, B)
+        report["near_boundary_decisions"] = near
+    assert nbad <= exclusion_budget(B) and nbad < B, \
+        "too many diverged prefixes: %d of %d" % (nbad, B)
 
     def eq(name, mask=rows_ok):
         g = to_np(gpu[name]).reshape(-1)
@@ -102,9 +128,12 @@ def compare_linear(gpu, orc, B, K, D, V, T, grad_dtype="f32", check_grad=True, r
         g = to_np(gpu[name]).reshape(-1).astype(np.float64)
         o = np.asarray(orc[name], dtype=np.float64).reshape(-1)
         both_inf = np.isinf(g) & np.isinf(o) & (np.sign(g) == np.sign(o))
-        err = np.where(both_inf, 0.0, np.abs(g - o))
-        lim = atol + rtol * np.abs(np.where(np.isinf(o), 0, o))
-        badi = np.nonzero((err > lim) & mask)[0]
+        both_nan = np.isnan(g) & np.isnan(o)
+        with np.errstate(invalid="ignore"):
+            err = np.where(both_inf | both_nan, 0.0, np.abs(g - o))
+        lim = atol + rtol * np.abs(np.where(np.isfinite(o), o, 0))
+        # written as "not within": a NaN or a lone infinity on either side fails
+        badi = np.nonzero(~(err <= lim) & mask)[0]
         assert badi.size == 0, "%s off at %s: gpu %s oracle %s" % (
             name, badi[:8], g[badi[:8]], o[badi[:8]])
 
@@ -154,7 +183,7 @@ def compare_linear(gpu, orc, B, K, D, V, T, grad_dtype="f32", check_grad=True, r
         else:
             lim = 1e-5 * np.abs(o) + 1e-6 * scale + 1e-30
         err = np.abs(g - o)
-        badr = np.nonzero(((err > lim).any(axis=1)) & rows_ok)[0]
+        badr = np.nonzero((~(err <= lim)).any(axis=1) & rows_ok)[0]
         assert badr.size == 0, "grad rows off: %s, max err %g (scale %g)" % (
             badr[:8], err[badr].max(), scale)
         emax = float(err[rows_ok].max()) if rows_ok.any() else 0.0
@@ -183,9 +212,12 @@ def compare_tree(gpu, orc, report=None):
             assert (m[b, bad, 1] < PROB_MARGIN).all(), "residual differs outside the margin"
             div[b] = True
     ok = ~div
+    SESSION["trees"] += B
+    SESSION["excluded_trees"] += int(div.sum())
     if report is not None:
         report["excluded_trees"] = int(div.sum())
-    assert div.sum() <= max(1, B // 8)
+    assert div.sum() <= exclusion_budget(B) and div.sum() < B, \
+        "too many diverged trees: %d of %d" % (int(div.sum()), B)
     for name in ("accept", "path_accept", "corr_tokens"):
         assert np.array_equal(to_np(gpu[name])[ok], orc[name][ok]), name
     for name in ("deepest", "accept_len", "bonus"):
@@ -196,4 +228,7 @@ def compare_tree(gpu, orc, report=None):
     ol = orc["logkappa"]
     sel = ok[:, None] & np.isfinite(ol)
     assert np.allclose(gl[sel], ol[sel], atol=LOGK_MARGIN, rtol=1e-6)
+    # a path the oracle gives zero validity (log kappa = -inf) must be -inf too
+    neg = ok[:, None] & np.isneginf(ol)
+    assert np.all(np.isneginf(gl[neg])), "log kappa finite where the oracle has -inf"
     return int(div.sum())

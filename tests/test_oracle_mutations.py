@@ -1,0 +1,127 @@
+"""Mutation check of the oracle's pins.
+
+Each case below plants one plausible mistake in a copy of oracle/vsd_oracle.c
+(a tie rule, a sign, an index, a dropped term, a swapped operand), compiles
+that copy, and runs every pin of tests/test_oracle_pins.py against it: at
+least one pin must fail.  A mutation no pin notices would mean that part of
+the oracle is checked only against itself.  CPU only; gcc builds each copy in
+well under a second.
+"""
+import inspect
+import itertools
+import os
+import subprocess
+
+import pytest
+
+from oracle import oracle as oracle_mod
+from oracle.build import SRC
+from tests import test_oracle_pins as pins
+
+# (name, text in vsd_oracle.c, replacement); the text must occur exactly once.
+MUTATIONS = [
+    ("accept tie goes to reject",
+     "double u = (double)in->u_accept[r];\n                uint8_t a = (u <= alpha)",
+     "double u = (double)in->u_accept[r];\n                uint8_t a = (u < alpha)"),
+    ("inverse CDF takes the boundary", "        if (u < F) {", "        if (u <= F) {"),
+    ("residual direction reversed",
+     "                    for (int64_t v = 0; v < V; ++v) {\n"
+     "                        double dv = p[v] - q[v];",
+     "                    for (int64_t v = 0; v < V; ++v) {\n"
+     "                        double dv = q[v] - p[v];"),
+    ("w(l) off by one", "pow(w_base, (double)l)", "pow(w_base, (double)(l - 1))"),
+    ("beta not leave-one-out", "        if (j == s) continue;\n", ""),
+    ("beta denominator counts proposals", "den += op[j];", "den += 1.0;"),
+    ("zeta modes swapped", "(mode == 0 ? exp(logq_path[j]) : logq_path[j])",
+     "(mode == 1 ? exp(logq_path[j]) : logq_path[j])"),
+    ("zeta multiplies by tau", "logq_path[j]) / tau;", "logq_path[j]) * tau;"),
+    ("control-variate sign", "J += op * (logq_z - beta * zeta * logq_zt);",
+     "J += op * (logq_z + beta * zeta * logq_zt);"),
+    ("gradient of the correction term", "double c_neg = op * beta * zeta /",
+     "double c_neg = -op * beta * zeta /"),
+    ("o' of a substitute path dropped",
+     "op[s] = oracle_utility(logkappa_corr[s * D + d], lkr, l, w_base);", "op[s] = 0.0;"),
+    ("o' of a kept proposal is binary", "                op[s] = o_tilde; /* z = z~, o' = o(z~) */",
+     "                op[s] = 1.0;"),
+    ("greedy reference ties to the highest index", "if (xp[v] > xp[vb]) vb = v;",
+     "if (xp[v] >= xp[vb]) vb = v;"),
+    ("expected length skips S_1", "for (int d = 0; d < D; ++d) EA += exp(lk[s * D + d]);",
+     "for (int d = 1; d < D; ++d) EA += exp(lk[s * D + d]);"),
+    ("after the first rejection draws from q",
+     "                } else {\n                    zc = sample_inverse_cdf(p, V, "
+     "(double)in->u_correct[r], &mg);\n                }",
+     "                } else {\n                    zc = sample_inverse_cdf(q, V, "
+     "(double)in->u_correct[r], &mg);\n                }"),
+    ("log kappa of z' uses z~'s alpha", "lkc[s * D + d] = prev + log(ac);",
+     "lkc[s * D + d] = prev + log(out->alpha[r]);"),
+    ("loss not normalised by N", "double lb = N > 0.0 ? -J / N : 0.0;",
+     "double lb = N > 0.0 ? -J : 0.0;"),
+    ("tree acceptance not an AND-scan",
+     "out->path_accept[n0 + n] = (uint8_t)(a && out->path_accept[rp]);",
+     "out->path_accept[n0 + n] = (uint8_t)a;"),
+    ("tree residual direction reversed",
+     "                for (int64_t v = 0; v < V; ++v) {\n"
+     "                    double dv = p[v] - q[v];",
+     "                for (int64_t v = 0; v < V; ++v) {\n"
+     "                    double dv = q[v] - p[v];"),
+    ("tree bonus ignores the residual", "if (par[n] == best) { bonus = out->corr_tokens[n0 + n]; break; }",
+     "if (par[n] == best) { break; }"),
+    ("margin: unequal sums given no margin", "if (a != b) return fabs(a - b);",
+     "if (a != b) return 0.0;"),
+    ("margin: a clipped tie given no margin", "        if (ra[i] < m) m = ra[i];\n", ""),
+    ("margin: identical tokens not cancelled",
+     "        if (rb && ta[i] == tb[i]) continue; /* identical terms cancel exactly */\n", ""),
+]
+
+
+def _pin_calls():
+    """Every pin of test_oracle_pins as (name, zero-argument callable)."""
+    calls = []
+    for name, fn in inspect.getmembers(pins, inspect.isfunction):
+        if not name.startswith("test_") or fn.__module__ != pins.__name__:
+            continue
+        marks = [m for m in getattr(fn, "pytestmark", []) if m.name == "parametrize"]
+        grids = []
+        for m in marks:
+            names = [n.strip() for n in m.args[0].split(",")] if isinstance(m.args[0], str) \
+                else list(m.args[0])
+            vals = [v if len(names) > 1 else (v,) for v in m.args[1]]
+            grids.append([dict(zip(names, v)) for v in vals])
+        for combo in itertools.product(*grids) if grids else [()]:
+            kw = {}
+            for d in combo:
+                kw.update(d)
+            calls.append((name, lambda fn=fn, kw=kw: fn(oracle_mod, **kw)))
+    return calls
+
+
+def _build(text, path):
+    with open(path + ".c", "w") as f:
+        f.write(text)
+    subprocess.run(["gcc", "-O1", "-std=c99", "-fPIC", "-shared", "-fno-fast-math",
+                    "-ffp-contract=off", path + ".c", "-o", path, "-lm"], check=True)
+
+
+def test_unmutated_copy_passes_every_pin(tmp_path, oracle):
+    path = str(tmp_path / "orig.so")
+    _build(open(SRC).read(), path)
+    with oracle_mod.using_library(path):
+        for name, call in _pin_calls():
+            call()
+
+
+@pytest.mark.parametrize("name,old,new", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_each_mutation_fails_a_pin(tmp_path, oracle, name, old, new):
+    src = open(SRC).read()
+    assert src.count(old) == 1, "mutation anchor must occur once: %r" % old
+    path = str(tmp_path / "mut.so")
+    _build(src.replace(old, new), path)
+    caught = []
+    with oracle_mod.using_library(path):
+        for pin, call in _pin_calls():
+            try:
+                call()
+            except (AssertionError, ValueError, IndexError, OverflowError, ZeroDivisionError):
+                caught.append(pin)
+                break
+    assert caught, "no pin fails with the mutation %r" % name

@@ -93,9 +93,13 @@ def test_mixture_reproduces_target_exactly(oracle, T):
     assert np.array_equal(hist, P_UNI)
     # acceptance rate sum_v min(p, q)
     assert o["accept"].mean() == np.minimum(P_UNI, Q4).sum()
-    # a residual token always has p > q, so its alpha is 1
+    # a residual token always has p > q, so its alpha is 1 and the corrected
+    # path's log kappa is 0; an accepted token keeps its own alpha
     rej = o["accept"] == 0
     assert np.all(o["alpha_corr"][rej] == 1.0)
+    assert np.all(o["logkappa_corr"][rej] == 0.0)
+    assert np.array_equal(o["alpha_corr"][~rej], o["alpha"][~rej])
+    assert np.allclose(o["logkappa_corr"], np.log(o["alpha_corr"]), rtol=0, atol=1e-15)
     assert set(np.unique(out[rej])) <= {2, 3}
 
 
@@ -517,3 +521,68 @@ def test_round_bf16_ties_to_even_and_matches_torch(oracle):
     f = np.random.default_rng(3).standard_normal(20000).astype(np.float32) * 40
     want = torch.from_numpy(f).to(torch.bfloat16).float().numpy()
     assert np.array_equal(oracle.round_bf16(f.astype(np.float64)), want)
+
+
+# --------------------------------------------------------------------------
+# Algorithm 2's comparison log k(z) >= log k(z-bar): the margin the parity
+# protocol uses to decide which disagreements it may excuse.  Each case is
+# built by hand so that the answer is known without the oracle.
+
+
+def test_decision_margin_unequal_sums_is_the_gap(oracle):
+    assert oracle.decision_margin(-1.0, -1.5, [-1.0], [3], [-1.5], [4]) == 0.5
+    assert oracle.decision_margin(-2.25, -0.25, [-2.25], [3]) == 2.0
+
+
+def test_decision_margin_clipped_tie_is_smallest_ratio(oracle):
+    # both sums 0: every ratio at a position where the tokens differ is >= 0,
+    # so min(0, r) clips it; position 0 holds the same token on both paths and
+    # cancels exactly (its ratios do not count)
+    ra, ta = [-0.4, 0.7, 0.3], [5, 1, 2]
+    rb, tb = [-0.4, 0.2, 0.9], [5, 7, 8]
+    assert oracle.decision_margin(-0.4, -0.4, ra, ta, rb, tb) == 0.2
+    # an input reference of 0 (rb = None): every ratio of the path counts
+    assert oracle.decision_margin(0.0, 0.0, [0.6, 0.25], [1, 2]) == 0.25
+
+
+def test_decision_margin_coincidental_tie_is_zero(oracle):
+    # equal sums reached through an unclipped ratio at a differing position:
+    # a rounding difference could flip the comparison, so the margin is 0
+    ra, ta = [-0.3, 0.5], [1, 2]
+    rb, tb = [-0.3, 0.5], [4, 2]
+    assert oracle.decision_margin(-0.3, -0.3, ra, ta, rb, tb) == 0.0
+    # the same when only the reference's ratio is unclipped
+    assert oracle.decision_margin(-0.1, -0.1, [0.4, -0.1], [1, 2], [0.4, -0.1],
+                                  [1, 3]) == 0.0
+
+
+def test_decision_margin_input_reference_tie_is_zero(oracle):
+    # an input reference b != 0 equal to the path's sum is a coincidence
+    assert oracle.decision_margin(-0.75, -0.75, [0.5, -0.75], [1, 2]) == 0.0
+    assert oracle.decision_margin(-0.75, -0.75, [-0.5, -0.25], [1, 2]) == 0.0
+
+
+def test_margins_of_a_worked_prefix(oracle):
+    """The margins the oracle reports for a prefix built by hand: path 0
+    accepts both tokens with ratios >= 1 (log k = 0 = the greedy reference,
+    every differing ratio clipped), so its o~ margin is the smaller ratio."""
+    q = [0.5, 0.25, 0.125, 0.125]
+    p = [0.125, 0.5, 0.25, 0.125]
+    D = 2
+    draft = np.stack([logits(q)] * D)
+    target = np.stack([logits(p)] * D)
+    # z~ = 1 at both positions (ratio 2), greedy reference = 1 as well -> the
+    # paths are equal: every term cancels, the comparison is exact
+    ud = np.array([midpoint(q, 1)] * D, np.float32)
+    o = oracle.linear(draft, target, 1.0, ud, np.full(D, 0.5, np.float32),
+                      np.full(D, 0.5, np.float32), K=1, D=D, want_grad=False)
+    assert list(o["tokens"]) == [1, 1] and list(o["ref_tokens"]) == [1, 1]
+    assert np.all(np.isinf(o["margins"][:, 3]))
+    # z~ = 2 at both positions (ratio 2, clipped): log k = 0 = reference, and
+    # the differing positions hold ratios log 2 on both sides
+    ud = np.array([midpoint(q, 2)] * D, np.float32)
+    o = oracle.linear(draft, target, 1.0, ud, np.full(D, 0.5, np.float32),
+                      np.full(D, 0.5, np.float32), K=1, D=D, want_grad=False)
+    assert list(o["tokens"]) == [2, 2]
+    # (the logits hold log q, log p rounded to float32: ratios within 1e-7 of 2)
+    assert np.allclose(o["margins"][:, 3], math.log(2), rtol=0, atol=1e-7)

@@ -25,19 +25,22 @@ def vsd():
 
 
 def test_rejects_layouts_beyond_the_scratch(vsd):
-    """Host-side check, before any CUDA call: too large -> VSD_ERR_TOO_LARGE."""
+    """Host-side check, before any CUDA call: too large -> VSD_ERR_TOO_LARGE.
+    Every pointer is NULL, so a call that got past the size check would be
+    refused as an invalid argument before anything is launched."""
     lib = vsd.load()
     lay = vsd.layout(64, 64, 64, 1024)  # needs ~49 MB of scratch
     assert vsd.workspace_bytes(lay) > vsd.NOALLOC_SCRATCH_BYTES
-    fake = C.c_void_p(0x1000)  # never dereferenced: the size check fails first
-    outs = vsd.LinearOutputs(*([0x1000] * len(vsd.LINEAR_FIELDS)))
-    code = lib.vsd_estep_mstep_noalloc(fake, fake, 1, lay, 1.0, fake, fake, fake, None, None,
+    null = None
+    outs = vsd.LinearOutputs(*([None] * len(vsd.LINEAR_FIELDS)))
+    code = lib.vsd_estep_mstep_noalloc(null, null, 1, lay, 1.0, null, null, null, None, None,
                                        C.byref(outs), None)
     assert code == 7
     assert b"scratch" in lib.vsd_status_string(code)
     bad = vsd.layout(0, 1, 1, 8)
-    assert lib.vsd_estep_mstep_noalloc(fake, fake, 1, bad, 1.0, fake, fake, fake, None, None,
+    assert lib.vsd_estep_mstep_noalloc(null, null, 1, bad, 1.0, null, null, null, None, None,
                                        C.byref(outs), None) == 1
+    assert lib.vsd_noalloc_device_status(None, None) == 1
 
 
 def _problem(kind):
@@ -65,3 +68,22 @@ def test_noalloc_matches_workspace_entry_point(vsd):
             # the same kernel on the same inputs is deterministic: equal bits
             assert torch.equal(ref[name], got[name]), (kind, T, name)
         assert torch.isfinite(got["loss"]).all()
+        assert vsd.noalloc_device_status() == (0, 0)
+
+
+@pytest.mark.gpu
+def test_noalloc_status_word_reports_a_timeout(vsd):
+    """The status word of the built-in array is readable: a call whose
+    gradient waits are made to run out (the test hook, with a 2 ms bound)
+    reports the timeout bit, and the next ordinary call reports none."""
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    p = _problem("ragged")
+    K, D = p["K"], p["D"]
+    prm = vsd.params(like=p["draft"], wait_timeout_ns=2_000_000, test_never_publish=1)
+    vsd.estep_mstep_noalloc(p["draft"], p["target"], p["u_draft"], p["u_accept"],
+                            p["u_correct"], K, D, 1.0, prm=prm)
+    code, bits = vsd.noalloc_device_status()
+    assert code == 4 and bits & vsd.STATUS_TIMEOUT
+    vsd.estep_mstep_noalloc(p["draft"], p["target"], p["u_draft"], p["u_accept"],
+                            p["u_correct"], K, D, 1.0)
+    assert vsd.noalloc_device_status() == (0, 0)
