@@ -27,7 +27,9 @@ def pytest_terminal_summary(terminalreporter):
     if SESSION["calls"] == 0 and SESSION["trees"] == 0:
         return
     terminalreporter.write_line(
-        "parity protocol: %d linear calls, %d prefixes compared, %d near-boundary decisions, "
-        "%d prefixes excluded; %d trees compared, %d trees excluded" % (
+        "parity protocol: %d linear calls, %d prefixes, %d near-boundary decisions, "
+        "%d paths with a flipped decision, %d prefixes checked conditionally, %d excluded; "
+        "%d trees, %d trees excluded" % (
             SESSION["calls"], SESSION["prefixes"], SESSION["near_boundary_decisions"],
+            SESSION["diverged_paths"], SESSION["conditional_prefixes"],
             SESSION["excluded_prefixes"], SESSION["trees"], SESSION["excluded_trees"]))

@@ -14,7 +14,7 @@ import numpy as np
 import pytest
 import torch
 
-from tests.parity import compare_linear
+from tests.parity import compare_linear, mstep_inputs
 
 pytestmark = pytest.mark.gpu
 
@@ -107,4 +107,37 @@ def test_lmhead_estep_mstep_matches_oracle(vsd, oracle, B, K, D, V, H, T):
     orc = oracle.linear(draft, p["target"].float().cpu().numpy(), T,
                         p["u_draft"].cpu().numpy(), p["u_accept"].cpu().numpy(),
                         p["u_correct"].cpu().numpy(), K, D)
-    compare_linear(g, orc, B, K, D, V, T, grad_dtype="bf16")
+    compare_linear(g, orc, B, K, D, V, T, grad_dtype="bf16",
+                   mstep_inputs=mstep_inputs(dict(B=B, K=K, D=D, draft=draft)))
+
+
+def test_lmhead_estep_mstep_full_size(vsd, oracle):
+    """The lmhead workload's shape (R = 64*8*8 = 4096 rows, H = 4096, V =
+    32000) through vsd_lmhead_estep_mstep, on inputs whose float32 partial
+    sums are exact (so the oracle's logits are the GPU's bit for bit): the
+    draft logits of three sampled prefixes (first, middle, last) are checked
+    bit for bit, and those prefixes' E-step/M-step results against the oracle
+    run on the oracle's own logits."""
+    from paper_2602_05774_gb300 import inputs
+    from tests.parity import sub_batch
+    c = inputs.CONFIGS["lmhead"]
+    B, K, D, V, H = c["B"], c["K"], c["D"], c["V"], c["H"]
+    p = inputs.lmhead_exact_problem(B, K, D, V, H, device="cuda", seed=4242)
+    ws = vsd.new_workspace(vsd.layout(B, K, D, V), "cuda")
+    g = vsd.lmhead_estep_mstep(p["hidden"], p["weight"], p["target"], p["u_draft"],
+                               p["u_accept"], p["u_correct"], K, D, 1.0, workspace=ws)
+    assert vsd.device_status(ws) == (0, 0)
+    assert torch.isfinite(g["loss"]).all()
+    W = _np(p["weight"])
+    P = K * D
+    for b in (0, B // 2, B - 1):
+        rows = slice(b * P, (b + 1) * P)
+        draft = oracle.round_bf16(oracle.lmhead_logits(_np(p["hidden"][rows]), W))
+        assert np.array_equal(g["draft_logits"][rows].float().cpu().numpy(), draft), b
+        orc = oracle.linear(draft, p["target"][rows].float().cpu().numpy(), 1.0,
+                            p["u_draft"][rows].cpu().numpy(), p["u_accept"][rows].cpu().numpy(),
+                            p["u_correct"][rows].cpu().numpy(), K, D)
+        orc["grad"] = orc["grad"] / B
+        compare_linear(sub_batch(g, b, b + 1, B, K, D), orc, 1, K, D, V, 1.0,
+                       grad_dtype="bf16", check_mean=False,
+                       mstep_inputs=mstep_inputs(dict(B=1, K=K, D=D, draft=draft), B_total=B))

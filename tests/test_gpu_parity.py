@@ -8,7 +8,7 @@ import numpy as np
 import pytest
 import torch
 
-from tests.parity import compare_linear, compare_tree, to_np
+from tests.parity import compare_linear, compare_tree, mstep_inputs, to_np
 
 pytestmark = pytest.mark.gpu
 
@@ -49,7 +49,8 @@ def test_tiny_fused_matches_oracle(vsd, oracle, T):
     prob = inputs.config("tiny")
     orc = run_oracle(oracle, prob, T)
     g = fused(vsd, to_cuda(prob), T)
-    compare_linear(g, orc, prob["B"], prob["K"], prob["D"], prob["V"], T, grad_dtype="f32")
+    compare_linear(g, orc, prob["B"], prob["K"], prob["D"], prob["V"], T, grad_dtype="f32",
+                   mstep_inputs=mstep_inputs(prob))
 
 
 def test_vocab32k_fused_matches_oracle(vsd, oracle):
@@ -59,7 +60,7 @@ def test_vocab32k_fused_matches_oracle(vsd, oracle):
     g = fused(vsd, to_cuda(prob), 1.0)
     rep = {}
     compare_linear(g, orc, prob["B"], prob["K"], prob["D"], prob["V"], 1.0, grad_dtype="bf16",
-                   report=rep)
+                   report=rep, mstep_inputs=mstep_inputs(prob))
 
 
 SHAPES = [
@@ -90,7 +91,7 @@ def test_random_shapes_fused(vsd, oracle, B, K, D, V, dtype, kind, T):
     prob = inputs.linear_problem(B, K, D, V, dtype, kind, seed=1000 + V + 7 * K + D)
     orc = run_oracle(oracle, prob, T)
     g = fused(vsd, to_cuda(prob), T)
-    compare_linear(g, orc, B, K, D, V, T, grad_dtype=dtype)
+    compare_linear(g, orc, B, K, D, V, T, grad_dtype=dtype, mstep_inputs=mstep_inputs(prob))
 
 
 @pytest.mark.parametrize("zeta_mode,ref", [(1, False), (0, True)])
@@ -105,7 +106,8 @@ def test_params_and_reference_input(vsd, oracle, zeta_mode, ref):
     p = to_cuda(prob)
     prm = vsd.params(w_base=1.2, tau_car=0.5, zeta_mode=zeta_mode, grad_dtype=torch.float32)
     g = fused(vsd, p, 1.0, prm=prm, ref_logkappa=None if refk is None else refk.cuda())
-    compare_linear(g, orc, 3, 4, 3, 3000, 1.0, grad_dtype="f32")
+    compare_linear(g, orc, 3, 4, 3, 3000, 1.0, grad_dtype="f32",
+                   mstep_inputs=mstep_inputs(prob, w_base=1.2, tau_car=0.5, zeta_mode=zeta_mode))
 
 
 def test_draft_equals_target(vsd, oracle):
@@ -116,7 +118,7 @@ def test_draft_equals_target(vsd, oracle):
     g = fused(vsd, to_cuda(prob), 1.0)
     assert np.all(to_np(g["alpha"]) == 1.0)
     assert np.all(to_np(g["accept_len"]) == 4)
-    compare_linear(g, orc, 2, 4, 4, 2500, 1.0, grad_dtype="bf16")
+    compare_linear(g, orc, 2, 4, 4, 2500, 1.0, grad_dtype="bf16", mstep_inputs=mstep_inputs(prob))
 
 
 def test_one_token_rows(vsd, oracle):
@@ -137,7 +139,7 @@ def test_one_token_rows(vsd, oracle):
                 u_correct=torch.rand(R, generator=gen))
     orc = run_oracle(oracle, prob, 1.0)
     g = fused(vsd, to_cuda(prob), 1.0, prm=vsd.params(grad_dtype=torch.float32))
-    compare_linear(g, orc, B, K, D, V, 1.0, grad_dtype="f32")
+    compare_linear(g, orc, B, K, D, V, 1.0, grad_dtype="f32", mstep_inputs=mstep_inputs(prob))
 
 
 def test_separate_entry_points(vsd, oracle):
@@ -280,37 +282,42 @@ def test_tree_lattice_residual_and_bonus(vsd, oracle, dtype):
         compare_tree(g_, orc)
 
 
-@pytest.mark.parametrize("T", [1.0, 0.7])
-def test_vocab128k_full_size_sampled_prefixes(vsd, oracle, T):
-    """The benchmark's workload and launch; the oracle checks two sampled prefixes."""
+def test_vocab128k_full_size_all_prefixes(vsd, oracle):
+    """The benchmark's workload (B=32, K=16, D=8, V=128256, bf16) in the launch
+    the benchmark times, T = 1: every prefix against the oracle over the whole
+    batch (the oracle's own gradient scale 1/B matches the call's)."""
     from paper_2602_05774_gb300 import inputs
     prob = inputs.config("vocab128k", device="cuda")
     B, K, D, V = prob["B"], prob["K"], prob["D"], prob["V"]
+    g = fused(vsd, prob, 1.0)
+    rs = g["grad"].float().sum(dim=1)  # each gradient row sums to ~0
+    assert torch.isfinite(g["loss"]).all() and rs.abs().max().item() < 1e-3
+    orc = run_oracle(oracle, prob, 1.0)
+    rep = {}
+    compare_linear(g, orc, B, K, D, V, 1.0, grad_dtype="bf16", report=rep,
+                   mstep_inputs=mstep_inputs(prob))
+    print("vocab128k T=1: %s" % rep)
+
+
+def test_vocab128k_last_published_prefixes(vsd, oracle):
+    """T = 0.7, the four prefixes the fused kernel publishes last (their
+    gradient segments are scheduled after every other prefix's), compared as
+    a sub-batch of the full call."""
+    from paper_2602_05774_gb300 import inputs
+    from tests.parity import sub_batch
+    prob = inputs.config("vocab128k", device="cuda")
+    B, K, D, V = prob["B"], prob["K"], prob["D"], prob["V"]
+    T = 0.7
     g = fused(vsd, prob, T)
+    b0 = B - 4
     P = K * D
-    # properties at full size: gradient rows sum to ~0, loss finite
-    grad = g["grad"]
-    rs = grad.float().sum(dim=1)
-    assert torch.isfinite(g["loss"]).all()
-    assert rs.abs().max().item() < 1e-3
-    for b in (0, B - 1) if T == 1.0 else (B // 2,):
-        rows = slice(b * P, (b + 1) * P)
-        sub = dict(B=1, K=K, D=D, V=V, draft=prob["draft"][rows], target=prob["target"][rows],
-                   u_draft=prob["u_draft"][rows], u_accept=prob["u_accept"][rows],
-                   u_correct=prob["u_correct"][rows])
-        orc = run_oracle(oracle, sub, T)
-        # the oracle's loss normalises over its own batch of 1: rescale the grad
-        orc["grad"] = orc["grad"] / B
-        gsub = {}
-        for n, t in g.items():
-            if t is None:
-                continue
-            if n in ("accept_len", "expected_len"):
-                gsub[n] = t[b * K:(b + 1) * K]
-            elif n == "weights":
-                gsub[n] = t[b:b + 1]
-            elif n == "loss":
-                gsub[n] = torch.stack([t[b], t[b]])
-            elif t.shape[0] == B * P:
-                gsub[n] = t[rows]
-        compare_linear(gsub, orc, 1, K, D, V, T, grad_dtype="bf16")
+    rows = slice(b0 * P, B * P)
+    sub = dict(B=4, K=K, D=D, V=V, draft=prob["draft"][rows], target=prob["target"][rows],
+               u_draft=prob["u_draft"][rows], u_accept=prob["u_accept"][rows],
+               u_correct=prob["u_correct"][rows])
+    orc = run_oracle(oracle, sub, T)
+    orc["grad"] = orc["grad"] * (4.0 / B)  # the call normalises over its B prefixes
+    rep = {}
+    compare_linear(sub_batch(g, b0, B, B, K, D), orc, 4, K, D, V, T, grad_dtype="bf16",
+                   report=rep, check_mean=False, mstep_inputs=mstep_inputs(sub, B_total=B))
+    print("vocab128k T=0.7 last prefixes: %s" % rep)

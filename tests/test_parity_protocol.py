@@ -105,3 +105,58 @@ def test_budget_is_one_in_ten(oracle):
     _fails(gpu, orc, shape)
     assert parity.exclusion_budget(32) == 3 and parity.exclusion_budget(3) == 1
     assert parity.exclusion_budget(2) == 0 and parity.exclusion_budget(1) == 0
+
+
+def _gpu_view(o):
+    gpu = {}
+    for n in ("tokens", "accept_len", "corr_tokens", "ref_tokens"):
+        gpu[n] = o[n].astype(np.int32)
+    gpu["accept"] = o["accept"].astype(np.uint8)
+    for n in ("alpha", "alpha_corr", "logq_tok", "logq_corr", "logkappa", "logkappa_corr",
+              "logkappa_ref", "expected_len", "loss", "grad", "weights"):
+        gpu[n] = o[n].astype(np.float32)
+    return gpu
+
+
+def test_flipped_draw_is_checked_conditionally(oracle):
+    """A consistent result that took one near-boundary draft draw the other
+    way (the oracle itself run with that row's uniform moved across the CDF
+    boundary by one float step) passes: the flipped path is compared up to
+    the flip and the prefix's M-step conditionally; the same result with its
+    loss changed fails."""
+    from paper_2602_05774_gb300 import inputs
+    B, K, D, V = 4, 3, 3, 300
+    p = inputs.linear_problem(B, K, D, V, "f32", "gauss", seed=8)
+    f = {k: p[k].numpy().copy() for k in ("draft", "target", "u_draft", "u_accept", "u_correct")}
+    r = K * D + 1  # prefix 1, path 0, row 1
+    q = np.exp(oracle.log_softmax(f["draft"][r], 1.0))
+    F = float(np.cumsum(q)[10])
+    below = np.float32(F)
+    while float(below) >= F:
+        below = np.nextafter(below, np.float32(0))
+    above = np.nextafter(below, np.float32(1))
+    assert float(below) < F <= float(above)
+    f["u_draft"][r] = below
+    orc = oracle.linear(f["draft"], f["target"], 1.0, f["u_draft"], f["u_accept"],
+                        f["u_correct"], K, D)
+    f2 = dict(f)
+    f2["u_draft"] = f["u_draft"].copy()
+    f2["u_draft"][r] = above
+    o2 = oracle.linear(f2["draft"], f2["target"], 1.0, f2["u_draft"], f2["u_accept"],
+                       f2["u_correct"], K, D)
+    assert o2["tokens"][r] != orc["tokens"][r] and orc["margins"][r, 0] < parity.PROB_MARGIN
+    gpu = _gpu_view(o2)
+    P = K * D
+    mi = dict(draft_rows=lambda b: f["draft"][b * P:(b + 1) * P], B_total=B)
+    rep = {}
+    assert parity.compare_linear(gpu, orc, B, K, D, V, 1.0, grad_dtype="f32", report=rep,
+                                 mstep_inputs=mi) == 1
+    assert rep["diverged_paths"] == 1 and rep["conditional_prefixes"] == 1
+    bad = _gpu_view(o2)
+    bad["loss"][1] += 1e-3
+    with pytest.raises(AssertionError):
+        parity.compare_linear(bad, orc, B, K, D, V, 1.0, grad_dtype="f32", mstep_inputs=mi)
+    bad = _gpu_view(o2)
+    bad["grad"][P + 2, 5] += 1e-3
+    with pytest.raises(AssertionError):
+        parity.compare_linear(bad, orc, B, K, D, V, 1.0, grad_dtype="f32", mstep_inputs=mi)
