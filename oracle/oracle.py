@@ -22,6 +22,7 @@ class _LinearIn(C.Structure):
         ("u_draft", C.c_void_p), ("u_accept", C.c_void_p), ("u_correct", C.c_void_p),
         ("ref_logkappa", C.c_void_p),
         ("w_base", C.c_double), ("tau_car", C.c_double), ("zeta_mode", C.c_int32),
+        ("kl_weight", C.c_double), ("kl_topk", C.c_int32),
     ]
 
 
@@ -29,7 +30,8 @@ class _LinearOut(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in (
         "tokens", "logq_tok", "alpha", "accept", "accept_len", "corr_tokens",
         "logq_corr", "alpha_corr", "logkappa", "logkappa_corr", "logkappa_ref",
-        "ref_tokens", "expected_len", "row_lse", "weights", "loss", "grad", "margins")]
+        "ref_tokens", "expected_len", "row_lse", "weights", "loss", "grad", "margins",
+        "kl_loss")]
 
 
 class _TreeIn(C.Structure):
@@ -69,6 +71,9 @@ def _bind(path):
     lib_.vso_decision_margin.argtypes = [C.c_double, C.c_double, C.c_int, C.c_void_p,
                                          C.c_void_p, C.c_void_p, C.c_void_p]
     lib_.vso_decision_margin.restype = C.c_double
+    lib_.vso_topk_ce.argtypes = [C.c_void_p, C.c_void_p, C.c_int64, C.c_double, C.c_int,
+                                 C.c_void_p, C.c_void_p]
+    lib_.vso_topk_ce.restype = C.c_double
     return lib_
 
 
@@ -127,9 +132,10 @@ def sample(prob, u):
 
 
 def linear(draft, target, T, u_draft, u_accept, u_correct, K, D, ref_logkappa=None,
-           w_base=1.05, tau_car=0.2, zeta_mode=0, want_grad=True):
+           w_base=1.05, tau_car=0.2, zeta_mode=0, want_grad=True, kl_weight=0.0, kl_topk=10):
     """E-step + M-step over linear paths (Algorithm 1, Algorithm 2, Eqs. 1, 2, 11,
-    beta, zeta, advance).
+    beta, zeta, advance); with kl_weight != 0 the VSD (KL) variant adds
+    kl_weight times the prefix's top-kl_topk term of Eq. klv (reading R11).
 
     draft, target: [B*K*D, V] (any float dtype; widened to f32 exactly).
     Returns a dict of numpy arrays named as the C-ABI outputs.
@@ -152,9 +158,11 @@ def linear(draft, target, T, u_draft, u_accept, u_correct, K, D, ref_logkappa=No
         logkappa=np.zeros(R), logkappa_corr=np.zeros(R), logkappa_ref=np.zeros(R),
         ref_tokens=np.zeros(R, np.int32), expected_len=np.zeros(B * K),
         row_lse=np.zeros((R, 2)), weights=np.zeros((B, D, K, 4)), loss=np.zeros(B + 1),
-        grad=np.zeros((R, V)) if want_grad else None, margins=np.zeros((R, 6)))
+        grad=np.zeros((R, V)) if want_grad else None, margins=np.zeros((R, 6)),
+        kl_loss=np.zeros(R))
     li = _LinearIn(_ptr(draft), _ptr(target), B, K, D, V, float(T), _ptr(ud), _ptr(ua),
-                   _ptr(uc), _ptr(ref), float(w_base), float(tau_car), int(zeta_mode))
+                   _ptr(uc), _ptr(ref), float(w_base), float(tau_car), int(zeta_mode),
+                   float(kl_weight), int(kl_topk))
     lo = _LinearOut(*[_ptr(o[n]) for n, _ in _LinearOut._fields_])
     rc = lib().vso_linear(C.byref(li), C.byref(lo))
     if rc != 0:
@@ -185,6 +193,17 @@ def tree(draft, target, T, parent, tokens, u_accept, u_correct):
     if rc != 0:
         raise ValueError("oracle rejected the tree (code %d)" % rc)
     return o
+
+
+def topk_ce(draft_row, target_row, T=1.0, k=10):
+    """Eq. klv for one row: (L, Omega [k] in selection order, dL/dx at Omega)."""
+    xq = _f32(draft_row).reshape(-1)
+    xp = _f32(target_row).reshape(-1)
+    kk = min(k, xq.size)
+    tok = np.zeros(max(kk, 1), np.int32)
+    dl = np.zeros(max(kk, 1))
+    L = lib().vso_topk_ce(_ptr(xq), _ptr(xp), xq.size, float(T), int(k), _ptr(tok), _ptr(dl))
+    return L, tok[:kk], dl[:kk]
 
 
 def decision_margin(a, b, ra, ta, rb=None, tb=None):

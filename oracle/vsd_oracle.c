@@ -41,6 +41,13 @@
  *   R9  Ties: accept on u <= alpha (Eq. 1 text "r <= alpha"); sample = smallest
  *       v with u < F(v); argmax lowest index; ">=" passes in Algorithm 2.
  *   R10 If the residual mass sum_v max(0,p-q) is 0 the correction samples p.
+ *   R11 VSD (KL): the KL term of the ELBO (Eq. elbo_vi) is replaced by the
+ *       top-K renormalised cross-entropy of Eq. klv (K = 10) at every row the
+ *       proposals visit; per prefix L_KL = (1/S) sum_{s,d} L_topK(row (s,d)),
+ *       an MC estimate of the path-level KL, which is a sum over positions;
+ *       loss_b = -J_b/N_b + kl_weight L_KL.  The paper gives no weight;
+ *       kl_weight = 0 is VSD without the term.  The rows' contexts are held
+ *       fixed in the gradient (as in R8).
  *   Tree (App. E verification): node n's token was drafted from the row of
  *   parent(n); alpha_n uses that row; A_n = a_n AND A_parent(n); a rejected node
  *   whose parent is accepted gets a residual token drawn at the parent's row.
@@ -105,6 +112,8 @@ typedef struct {
     double w_base;             /* w(l) = w_base^l                            */
     double tau_car;            /* CAR temperature tau                        */
     int32_t zeta_mode;         /* 0: q(path) (literal), 1: log q(path)       */
+    double kl_weight;          /* weight of the top-K term (R11), 0 = none   */
+    int32_t kl_topk;           /* K of Eq. klv (the paper's 10)              */
 } vso_linear_in;
 
 typedef struct {
@@ -126,6 +135,7 @@ typedef struct {
     double*  loss;          /* [B+1]: loss_b, then the mean over b      */
     double*  grad;          /* optional [R][V] d loss / d draft logits  */
     double*  margins;       /* optional [R][6] decision margins (below) */
+    double*  kl_loss;       /* optional [R] L_topK of the row (Eq. klv) */
 } vso_linear_out;
 /* margins[r][0]: draft sample, |u - nearest CDF boundary| of q
  * margins[r][1]: accept, |u_accept - alpha|
@@ -295,6 +305,49 @@ static double decision_margin(double a, double b, int n, const double* ra, const
 }
 
 /* ------------------------------------------------------------------ */
+/* VSD (KL), Eq. klv: the top-K renormalised cross-entropy of one row.  Omega
+ * = the Kt tokens of highest target probability (lowest index on ties);
+ * p^(x) = p(x) / sum_{y in Omega} p(y), q^ likewise;
+ * L = -sum_{x in Omega} p^(x) log q^(x) (a term with p^(x) = 0 is 0).
+ * tok[k] receives Omega in order of selection, dl[k] = dL/dx_{tok[k]} =
+ * (q^ - p^)/T: log q^(x) = x_x/T - log sum_{Omega} exp(x_y/T), so the full
+ * vocabulary's partition cancels and every other logit has derivative 0. */
+static double topk_ce_row(const float* xq, const float* xp, int64_t V, double T, int Kt,
+                          int32_t* tok, double* dl)
+{
+    if (Kt > V) Kt = (int)V;
+    for (int k = 0; k < Kt; ++k) {
+        int64_t best = -1;
+        for (int64_t v = 0; v < V; ++v) {
+            int taken = 0;
+            for (int j = 0; j < k; ++j) taken |= tok[j] == v;
+            if (taken) continue;
+            if (best < 0 || xp[v] > xp[best]) best = v; /* strict: lowest index wins ties */
+        }
+        tok[k] = (int32_t)best;
+    }
+    double mp = -INFINITY, mq = -INFINITY;
+    for (int k = 0; k < Kt; ++k) {
+        double a = (double)xp[tok[k]] / T, b = (double)xq[tok[k]] / T;
+        if (a > mp) mp = a;
+        if (b > mq) mq = b;
+    }
+    double Sp = 0.0, Sq = 0.0;
+    for (int k = 0; k < Kt; ++k) {
+        Sp += exp((double)xp[tok[k]] / T - mp);
+        Sq += exp((double)xq[tok[k]] / T - mq);
+    }
+    double L = 0.0;
+    for (int k = 0; k < Kt; ++k) {
+        double ph = exp((double)xp[tok[k]] / T - mp) / Sp;
+        double lqh = (double)xq[tok[k]] / T - mq - log(Sq);
+        if (ph > 0.0) L -= ph * lqh;
+        dl[k] = (exp(lqh) - ph) / T;
+    }
+    return L;
+}
+
+/* ------------------------------------------------------------------ */
 /* Public: the whole E-step + M-step for linear paths.  Returns 0 on success,
  * nonzero on an invalid argument. */
 int vso_linear(const vso_linear_in* in, vso_linear_out* out)
@@ -451,6 +504,24 @@ int vso_linear(const vso_linear_in* in, vso_linear_out* out)
                                         out->tokens + rb, out->corr_tokens + rb, wb, N, B,
                                         out->grad ? out->grad + rb * V : NULL);
         double lb = N > 0.0 ? -J / N : 0.0;
+        if (in->kl_weight != 0.0) {
+            /* R11: + kl_weight (1/S) sum over the prefix's rows of Eq. klv */
+            int32_t tok[64];
+            double dl[64];
+            int Kt = in->kl_topk < 1 ? 1 : (in->kl_topk > 64 ? 64 : in->kl_topk);
+            double kl = 0.0;
+            for (size_t r = rb; r < rb + (size_t)K * D; ++r) {
+                double L = topk_ce_row(in->draft + r * V, in->target + r * V, V, T, Kt, tok, dl);
+                if (out->kl_loss) out->kl_loss[r] = L;
+                kl += L;
+                if (out->grad) {
+                    int kk = Kt > V ? (int)V : Kt;
+                    for (int k = 0; k < kk; ++k)
+                        out->grad[r * V + tok[k]] += in->kl_weight / ((double)B * K) * dl[k];
+                }
+            }
+            lb += in->kl_weight * kl / (double)K;
+        }
         out->loss[b] = lb;
         loss_sum += lb;
     }
@@ -586,6 +657,13 @@ double vso_log_softmax(const float* x, int64_t V, double T, double* lp)
 int64_t vso_sample(const double* prob, int64_t V, double u, double* margin)
 {
     return sample_inverse_cdf(prob, V, u, margin);
+}
+
+/* Eq. klv for one row (see topk_ce_row). */
+double vso_topk_ce(const float* xq, const float* xp, int64_t V, double T, int Kt, int32_t* tok,
+                   double* dl)
+{
+    return topk_ce_row(xq, xp, V, T, Kt, tok, dl);
 }
 
 /* The margin of one Algorithm 2 comparison (see decision_margin); rb and tb

@@ -66,6 +66,13 @@ MUTATIONS = [
      "                    double dv = q[v] - p[v];"),
     ("tree bonus ignores the residual", "if (par[n] == best) { bonus = out->corr_tokens[n0 + n]; break; }",
      "if (par[n] == best) { break; }"),
+    ("top-K ties to the highest index", "if (best < 0 || xp[v] > xp[best]) best = v;",
+     "if (best < 0 || xp[v] >= xp[best]) best = v;"),
+    ("top-K gradient sign", "dl[k] = (exp(lqh) - ph) / T;", "dl[k] = (ph - exp(lqh)) / T;"),
+    ("top-K term not averaged over proposals", "lb += in->kl_weight * kl / (double)K;",
+     "lb += in->kl_weight * kl;"),
+    ("top-K gradient scale", "in->kl_weight / ((double)B * K) * dl[k];",
+     "in->kl_weight / (double)B * dl[k];"),
     ("margin: unequal sums given no margin", "if (a != b) return fabs(a - b);",
      "if (a != b) return 0.0;"),
     ("margin: a clipped tie given no margin", "        if (ra[i] < m) m = ra[i];\n", ""),

@@ -586,3 +586,115 @@ def test_margins_of_a_worked_prefix(oracle):
     assert list(o["tokens"]) == [2, 2]
     # (the logits hold log q, log p rounded to float32: ratios within 1e-7 of 2)
     assert np.allclose(o["margins"][:, 3], math.log(2), rtol=0, atol=1e-7)
+
+
+# --------------------------------------------------------------------------
+# VSD (KL): the top-10 renormalised term of Eq. klv (reading R11), pinned to
+# torch's cross-entropy with probability targets and its autograd.
+
+
+def _torch_topk_ce(xq, xp, T, k=10):
+    """L and dL/dxq of Eq. klv by torch: top-k of the target (distinct values),
+    renormalised softmaxes on them, cross-entropy with soft targets."""
+    import torch
+    q = torch.tensor(np.asarray(xq, np.float64), requires_grad=True)
+    p = torch.tensor(np.asarray(xp, np.float64))
+    idx = torch.topk(p, min(k, p.numel())).indices
+    phat = torch.softmax(p[idx] / T, dim=0)
+    L = torch.nn.functional.cross_entropy((q[idx] / T)[None], phat[None])
+    L.backward()
+    return float(L.detach()), set(idx.tolist()), q.grad.numpy()
+
+
+@pytest.mark.parametrize("T", [1.0, 0.7])
+def test_topk_ce_matches_torch(oracle, T):
+    rng = np.random.default_rng(11)
+    for V in (10, 37, 300):
+        xq = rng.normal(0, 2, V).astype(np.float32)
+        xp = (xq + rng.normal(0, 1, V)).astype(np.float32)
+        L, tok, dl = oracle.topk_ce(xq, xp, T, 10)
+        Lt, it, gt = _torch_topk_ce(xq, xp, T)
+        assert set(tok.tolist()) == it
+        assert abs(L - Lt) < 1e-12 * max(1.0, abs(Lt))
+        full = np.zeros(V)
+        full[tok] = dl
+        assert np.allclose(full, gt, rtol=1e-10, atol=1e-14)  # zero outside the top 10
+        # cross-entropy = KL(p^ || q^) + H(p^) >= H(p^)
+        import torch
+        ph = torch.softmax(torch.tensor(xp[tok].astype(np.float64)) / T, 0)
+        lqh = torch.log_softmax(torch.tensor(xq[tok].astype(np.float64)) / T, 0)
+        kl = float(torch.nn.functional.kl_div(lqh, ph, reduction="sum"))
+        H = float(-(ph * torch.log(ph)).sum())
+        assert abs(L - (kl + H)) < 1e-12 * max(1.0, abs(L)) and kl >= 0
+
+
+def test_topk_ce_finite_differences(oracle):
+    rng = np.random.default_rng(12)
+    xq = rng.normal(0, 1, 40)
+    xp = rng.normal(0, 1, 40).astype(np.float32)
+    T = 0.8
+    L, tok, dl = oracle.topk_ce(xq.astype(np.float32), xp, T, 10)
+    # central differences in float64 on logits exactly representable in float32
+    for k in (0, 4, 9):
+        v = tok[k]
+        h = 2.0 ** -10
+        xa, xb = xq.astype(np.float32).copy(), xq.astype(np.float32).copy()
+        xa[v] += np.float32(h)
+        xb[v] -= np.float32(h)
+        fd = (oracle.topk_ce(xa, xp, T, 10)[0] - oracle.topk_ce(xb, xp, T, 10)[0]) / (2 * h)
+        assert abs(fd - dl[k]) < 1e-6
+    other = [v for v in range(40) if v not in set(tok.tolist())][0]
+    xa = xq.astype(np.float32).copy()
+    xa[other] += np.float32(0.5)
+    assert oracle.topk_ce(xa, xp, T, 10)[0] == L  # a logit outside the top 10 does not enter
+
+
+def test_topk_ce_ties_and_degenerate_rows(oracle):
+    # ties at the cut: the lowest indices are kept
+    xp = np.zeros(20, np.float32)
+    xq = np.arange(20, dtype=np.float32) / 10
+    L, tok, dl = oracle.topk_ce(xq, xp, 1.0, 10)
+    assert sorted(tok.tolist()) == list(range(10))
+    xp = np.array([5, 1, 1, 1, 3, 1, 1, 1, 1, 1, 1, 1, 2], np.float32)
+    tok = oracle.topk_ce(np.zeros(13, np.float32), xp, 1.0, 10)[1]
+    assert sorted(tok.tolist()) == [0, 1, 2, 3, 4, 5, 6, 7, 8, 12]
+    # draft = target: q^ = p^, so the gradient is 0 and L is the entropy of p^
+    x = np.array([3.0, 1.0, 0.5, -1.0, 2.0, 0.0, -2.0, 1.5, 0.25, -0.5, -3.0, -4.0], np.float32)
+    L, tok, dl = oracle.topk_ce(x, x, 1.0, 10)
+    assert np.allclose(dl, 0.0, atol=1e-15)
+    import torch
+    ph = torch.softmax(torch.tensor(x[tok].astype(np.float64)), 0)
+    assert abs(L - float(-(ph * torch.log(ph)).sum())) < 1e-12
+    # fewer than 10 tokens: the whole vocabulary, i.e. the ordinary soft-target
+    # cross-entropy of the full softmaxes
+    xq = np.array([0.3, -1.2, 2.0, 0.7, -0.1, 1.1], np.float32)
+    xp = np.array([1.0, 0.2, -0.4, 0.9, 2.2, -1.0], np.float32)
+    L, tok, dl = oracle.topk_ce(xq, xp, 1.0, 10)
+    full = torch.nn.functional.cross_entropy(torch.tensor(xq.astype(np.float64))[None],
+                                             torch.softmax(torch.tensor(xp.astype(np.float64)), 0)[None])
+    assert abs(L - float(full)) < 1e-12
+
+
+def test_kl_term_enters_loss_and_gradient(oracle):
+    """kl_weight lam adds lam/K sum_rows L_topk to each prefix's loss and
+    lam/(B K) dL/dx to the gradient rows (R11), here with torch computing
+    the added terms; the rest of the result is unchanged."""
+    from paper_2602_05774_gb300 import inputs
+    B, K, D, V, T, lam = 2, 3, 2, 64, 0.9, 0.37
+    p = inputs.linear_problem(B, K, D, V, "f32", "gauss", seed=21)
+    f = {k: p[k].numpy() for k in ("draft", "target", "u_draft", "u_accept", "u_correct")}
+    args = (f["draft"], f["target"], T, f["u_draft"], f["u_accept"], f["u_correct"], K, D)
+    o0 = oracle.linear(*args)
+    o1 = oracle.linear(*args, kl_weight=lam)
+    for n in ("tokens", "corr_tokens", "weights", "logkappa"):
+        assert np.array_equal(o0[n], o1[n])
+    dg = np.zeros_like(o0["grad"])
+    add = np.zeros(B)
+    for r in range(B * K * D):
+        Lt, _, gt = _torch_topk_ce(f["draft"][r], f["target"][r], T)
+        add[r // (K * D)] += lam / K * Lt
+        dg[r] = lam / (B * K) * gt
+        assert abs(o1["kl_loss"][r] - Lt) < 1e-12 * max(1.0, Lt)
+    assert np.allclose(o1["loss"][:B], o0["loss"][:B] + add, rtol=1e-12, atol=1e-12)
+    assert abs(o1["loss"][B] - o1["loss"][:B].mean()) < 1e-12
+    assert np.allclose(o1["grad"], o0["grad"] + dg, rtol=1e-10, atol=1e-15)
