@@ -87,6 +87,11 @@ typedef struct {
                                  never publishes a prefix's M-step, so every gradient
                                  wait runs out after wait_timeout_ns, no gradient row
                                  is written and VSD_STATUS_TIMEOUT is set            */
+    double kl_weight;  /* VSD (KL) (App., Eq. klv): 0 = none; else loss_b gains
+                          kl_weight (1/K) sum over the prefix's rows of the top-K
+                          renormalised cross-entropy -sum_{x in top-K of p}
+                          p^(x) log q^(x) (the paper gives no weight)       */
+    int32_t kl_topk;   /* K of that term (the paper's 10), 1 <= kl_topk <= 16  */
 } vsd_params;
 
 /* Output arrays of the linear E-step / M-step (all device, caller-owned).
@@ -112,6 +117,7 @@ typedef struct {
     float* weights;         /* [B][D][K][4] o~, o', beta, zeta (Alg. 1, Eq. beta/zeta)*/
     float* loss;            /* [B+1] loss_b = -J_b/N_b, then mean over b (Eq. advance)*/
     void* grad;             /* [R][V] d loss / d draft logits, params.grad_dtype      */
+    float* kl_loss;         /* [R] the row's top-K term of Eq. klv (with kl_weight)   */
 } vsd_linear_outputs;
 
 /* Output arrays of tree verification (device, caller-owned), [B][N] unless noted. */
@@ -161,7 +167,8 @@ vsd_status vsd_verify_paths(const void* draft, const void* target, vsd_dtype dty
                             vsd_tree_outputs* tree_out, void* ws, size_t ws_bytes,
                             void* stream);
 
-/* M-step (Algorithm 1 M-step, Algorithm 2 utility, Eqs. beta, zeta, advance):
+/* M-step (Algorithm 1 M-step, Algorithm 2 utility, Eqs. beta, zeta, advance;
+ * params->kl_weight must be 0 here, VSD_ERR_UNSUPPORTED otherwise):
  * from the E-step results in `estep` (tokens, corr_tokens, logq_tok, logq_corr,
  * logkappa, logkappa_corr, logkappa_ref, row_stats: all required) computes
  * o~, o', beta, zeta, loss_b = -J_b/N_b, their mean, and the gradient of the

@@ -29,7 +29,7 @@ struct WsLayout {
     size_t status, ticket, prefix_done, grad_head, resq_head, resq_tail, resq_avail;
     size_t path_cnt, prefix_cnt, ready, grad_cnt, row_seg_cnt, res_seg_cnt, resq_flag, zero_end;
     size_t rows, rstats, es_tok, es_corr, es_lq_tok, es_lq_corr, es_lk, es_lkc, es_lkr;
-    size_t coef, wscr, path_A, resq, gtab, total;
+    size_t coef, wscr, path_A, resq, klr, gtab, total;
     int nch_ws, nseg_ws;
 };
 
@@ -110,6 +110,7 @@ WsLayout ws_layout(const vsd_layout& L) {
     w.wscr = o; o = align256(o + sizeof(double2) * R);
     w.path_A = o; o = align256(o + 4 * npath);
     w.resq = o; o = align256(o + 4 * nq);
+    w.klr = o; o = align256(o + sizeof(KlRec) * R);
     w.gtab = o; o = align256(o + sizeof(float4) * R * (size_t)w.nch_ws);
     w.total = o;
     return w;
@@ -146,6 +147,8 @@ vsd_params default_params(vsd_dtype dtype) {
     p.grad_dtype = dtype;
     p.wait_timeout_ns = kDefaultTimeoutNs;
     p.test_never_publish = 0;
+    p.kl_weight = 0.0;
+    p.kl_topk = 10;
     return p;
 }
 
@@ -154,6 +157,8 @@ vsd_status check_params(const vsd_params& p) {
     if (!(p.tau_car > 0.0)) return VSD_ERR_INVALID_ARG;  // +inf allowed: zeta = 1/K
     if (p.zeta_mode != 0 && p.zeta_mode != 1) return VSD_ERR_INVALID_ARG;
     if (p.grad_dtype != VSD_F32 && p.grad_dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
+    if (!isfinite(p.kl_weight) || p.kl_weight < 0.0) return VSD_ERR_INVALID_ARG;
+    if (p.kl_weight != 0.0 && (p.kl_topk < 1 || p.kl_topk > kMaxKlTop)) return VSD_ERR_INVALID_ARG;
     return VSD_OK;
 }
 
@@ -211,6 +216,7 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.es.lkc = at<float>(ws, w.es_lkc);
     P.es.lkr = at<float>(ws, w.es_lkr);
     P.coef = at<Coef>(ws, w.coef);
+    P.klr = at<KlRec>(ws, w.klr);
     P.wscr = at<double2>(ws, w.wscr);
     P.segc = kSegChunks;
     P.nseg = (P.nch + kSegChunks - 1) / kSegChunks;
@@ -244,6 +250,9 @@ void set_params(Problem<T>& P, const vsd_params& p) {
     P.grad_bf16 = p.grad_dtype == VSD_BF16;
     P.timeout_ns = p.wait_timeout_ns ? p.wait_timeout_ns : kDefaultTimeoutNs;
     P.inject_wait_fault = p.test_never_publish;
+    P.kl_weight = p.kl_weight;
+    P.kl_topk = p.kl_weight != 0.0 ? p.kl_topk : 0;
+    P.kl_scale = p.kl_weight / ((double)P.B * (double)P.K * P.ts.Td);
     fill_wl(P);
 }
 
@@ -483,6 +492,7 @@ vsd_status vsd_weighted_loss_fwd_bwd(const void* draft, vsd_dtype dtype, vsd_lay
     if (st) return st;
     const vsd_params p = params ? *params : default_params(dtype);
     if ((st = check_params(p))) return st;
+    if (p.kl_weight != 0.0) return VSD_ERR_UNSUPPORTED;  // the top-K term needs the target rows
     if ((st = check_ws(layout, ws, ws_bytes))) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (dtype == VSD_F32)
@@ -586,6 +596,6 @@ const char* vsd_status_string(vsd_status status) {
     return "unknown status";
 }
 
-const char* vsd_version(void) { return "0.1.0"; }
+const char* vsd_version(void) { return "0.2.0"; }
 
 }  // extern "C"

@@ -294,14 +294,14 @@ __device__ void finish_path_warp(const Problem<T>& P, const EStepView& E, int pa
 }
 
 // What the control warp does after the streaming warps finished job j.
-template <typename T, bool VEC>
+template <typename T, bool VEC, bool KL>
 __device__ void post_job(const Problem<T>& P, const EStepView& E, const Job& j, float4* tab,
                          CtlShared& cs, int lane) {
     const int D = P.D, nseg = P.nseg, nch = P.nch;
     if (j.kind == kJobRow) {
         const int r = j.r;
         if (!warp_count_last(P.row_seg_cnt + r, nseg, lane)) return;
-        if (!P.stream_tails) row_tail_warp<T, VEC>(P, r, tab, cs.rb, lane);
+        if (!P.stream_tails) row_tail_warp<T, VEC, KL>(P, r, tab, cs.rb, lane);
         __syncwarp();
         const int path = r / D;
         if (!warp_count_last(P.path_cnt + path, D, lane)) return;
@@ -382,12 +382,15 @@ __device__ void post_job(const Problem<T>& P, const EStepView& E, const Job& j, 
 #ifndef VSD_FUSED_MIN_BLOCKS
 #define VSD_FUSED_MIN_BLOCKS 4
 #endif
-template <typename T, bool VEC, typename G>
+// KL: VSD (KL), the rows' top-K terms (a separate instantiation, so that the
+// plain kernel's code is unchanged by them).
+template <typename T, bool VEC, typename G, bool KL>
 __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
     k_fused(Problem<T> P, G* grad) {
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ CtlShared cs;
     __shared__ Job slots[kSlots];
+    __shared__ KlRec kslot[kSlots];  // VSD (KL): the top-K terms of a gradient job's row
     __shared__ RowShared rsh;
     Ring* rg;
     float4* tab;
@@ -409,14 +412,15 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
                                             policy_evict_first(), P.status);
                 if (P.stream_tails) {  // short rows: the tail here, three draws at once
                     asm volatile("bar.sync %0, %1;" ::"r"(kStreamBar), "r"(kThreads) : "memory");
-                    row_tail<T, VEC, true, kSampleToken, true, kStreamBar>(P, j.r, rtab, rsh);
+                    row_tail<T, VEC, true, kSampleToken, true, kStreamBar, KL>(
+                        P, j.r, rtab, rsh, VEC ? &rg->data[kWarps - 1][0][0][0] : nullptr);
                 }
             } else if (j.kind == kJobResidual) {
                 // row A's table was consumed by its row tail: reuse it
                 stream_residual<T, VEC>(rg, x, P.target + (int64_t)j.r * V, V, j.c0, j.c1,
                                         P.gtab + (int64_t)j.r * P.nch_ws, j.mr, P.status);
             } else {
-                stream_grad<T, VEC, G>(rg, P, j.r, j.c0, j.c1, grad);
+                stream_grad<T, VEC, G, KL>(rg, P, j.r, j.c0, j.c1, grad, KL ? &kslot[s] : nullptr);
             }
             __syncwarp();
             named_arrive(bar_done(s));
@@ -440,6 +444,12 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
             if (!got) break;
             __syncwarp();
             const int kind = slots[tail % kSlots].kind;
+            if (KL && kind == kJobGrad) {  // the row's top-K terms for the streaming warps
+                const int4* src = reinterpret_cast<const int4*>(P.klr + slots[tail % kSlots].r);
+                if (lane < (int)(sizeof(KlRec) / 16))
+                    reinterpret_cast<int4*>(&kslot[tail % kSlots])[lane] = __ldcg(src + lane);
+                __syncwarp();
+            }
             named_arrive(bar_full(tail % kSlots));
             ++tail;
             if (kind == kJobEnd) {
@@ -458,7 +468,7 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
         __syncwarp();
         ++head;
         --inflight;
-        if (cur.kind != kJobGrad) post_job<T, VEC>(P, E, cur, tab, cs, lane);
+        if (cur.kind != kJobGrad) post_job<T, VEC, KL>(P, E, cur, tab, cs, lane);
         __syncwarp();
     }
 }
@@ -691,16 +701,24 @@ template <>
 cudaError_t Launch<VSD_T>::fused(const Problem<VSD_T>& P, bool vec, void* grad, bool grad_bf16,
                                  int ctas, cudaStream_t s) {
     const size_t smem = stream_smem_bytes(P.nch, vec);
-#define VSD_FUSED(V_, G_)                                                              \
+    const bool kl = P.kl_topk != 0;
+#define VSD_FUSED(V_, G_, KL_)                                                         \
     do {                                                                               \
-        cudaError_t e = prep(k_fused<VSD_T, V_, G_>, smem);                            \
+        cudaError_t e = prep(k_fused<VSD_T, V_, G_, KL_>, smem);                       \
         if (e) return e;                                                               \
-        k_fused<VSD_T, V_, G_><<<ctas, kFusedThreads, smem, s>>>(P, reinterpret_cast<G_*>(grad)); \
+        k_fused<VSD_T, V_, G_, KL_><<<ctas, kFusedThreads, smem, s>>>(                 \
+            P, reinterpret_cast<G_*>(grad));                                           \
     } while (0)
-    if (vec && grad_bf16) VSD_FUSED(true, __nv_bfloat16);
-    else if (vec) VSD_FUSED(true, float);
-    else if (grad_bf16) VSD_FUSED(false, __nv_bfloat16);
-    else VSD_FUSED(false, float);
+#define VSD_FUSED_KL(V_, G_)                 \
+    do {                                     \
+        if (kl) VSD_FUSED(V_, G_, true);     \
+        else VSD_FUSED(V_, G_, false);       \
+    } while (0)
+    if (vec && grad_bf16) VSD_FUSED_KL(true, __nv_bfloat16);
+    else if (vec) VSD_FUSED_KL(true, float);
+    else if (grad_bf16) VSD_FUSED_KL(false, __nv_bfloat16);
+    else VSD_FUSED_KL(false, float);
+#undef VSD_FUSED_KL
 #undef VSD_FUSED
     return cudaGetLastError();
 }
@@ -708,10 +726,12 @@ cudaError_t Launch<VSD_T>::fused(const Problem<VSD_T>& P, bool vec, void* grad, 
 template <>
 int Launch<VSD_T>::fused_blocks_per_sm(const Problem<VSD_T>& P, bool vec, bool grad_bf16) {
     const size_t smem = stream_smem_bytes(P.nch, vec);
-    const void* k = vec ? (grad_bf16 ? reinterpret_cast<const void*>(k_fused<VSD_T, true, __nv_bfloat16>)
-                                     : reinterpret_cast<const void*>(k_fused<VSD_T, true, float>))
-                        : (grad_bf16 ? reinterpret_cast<const void*>(k_fused<VSD_T, false, __nv_bfloat16>)
-                                     : reinterpret_cast<const void*>(k_fused<VSD_T, false, float>));
+    const bool kl = P.kl_topk != 0;
+#define VSD_K(V_, G_) (kl ? reinterpret_cast<const void*>(k_fused<VSD_T, V_, G_, true>) \
+                          : reinterpret_cast<const void*>(k_fused<VSD_T, V_, G_, false>))
+    const void* k = vec ? (grad_bf16 ? VSD_K(true, __nv_bfloat16) : VSD_K(true, float))
+                        : (grad_bf16 ? VSD_K(false, __nv_bfloat16) : VSD_K(false, float));
+#undef VSD_K
     const int n = blocks_per_sm(k, kFusedThreads, smem);
     return n < 1 ? 1 : n;
 }

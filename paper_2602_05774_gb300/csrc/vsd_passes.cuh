@@ -56,6 +56,18 @@ struct __align__(16) Coef {     // grad[v] = g q(v) - c0 [v == t0] - c1 [v == t1
 };
 static_assert(sizeof(Coef) == 32, "Coef layout");
 
+// VSD (KL), Eq. klv: the top-K renormalised cross-entropy of one row and its
+// gradient, which touches only the K selected tokens.
+constexpr int kMaxKlTop = 16;
+struct __align__(16) KlRec {
+    int tok[kMaxKlTop];     // the K tokens of highest target probability (lowest index on ties)
+    float coef[kMaxKlTop];  // their gradient terms, kl_weight / (B K T) (q^ - p^)
+    float loss;             // L_topK of the row
+    int n;                  // entries used (0: the row has no term)
+    int pad[2];
+};
+static_assert(sizeof(KlRec) == 144, "KlRec layout");
+
 // Coherent loads of records written by other blocks of the same grid.
 template <typename U>
 __device__ __forceinline__ U ld_cg_rec(const U* p) {
@@ -68,6 +80,7 @@ __device__ __forceinline__ U ld_cg_rec(const U* p) {
     return r;
 }
 __device__ __forceinline__ RowRec ld_cg(const RowRec* p) { return ld_cg_rec(p); }
+__device__ __forceinline__ KlRec ld_cg(const KlRec* p) { return ld_cg_rec(p); }
 __device__ __forceinline__ Coef ld_cg(const Coef* p) { return ld_cg_rec(p); }
 
 // E-step results the M-step reads (structure of arrays, [R] each).
@@ -112,6 +125,10 @@ struct Problem {
     double inv_tau;  // 1 / tau_car
     float inv_tau_f;
     int zeta_mode;
+    int kl_topk;                  // VSD (KL): K of Eq. klv, 0 = no top-K term
+    double kl_weight;             // its weight in the loss
+    double kl_scale;              // kl_weight / (B K T), the gradient factor
+    KlRec* klr;                   // [R] the rows' terms
     int grad_bf16;
     int inject_wait_fault;
     uint64_t timeout_ns;
@@ -259,6 +276,7 @@ __device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, in
     const int cfirst = ch0 + warp, cstride = kWarps;
     const int pos = *posp;
     bool broken = rg->broken[warp] != 0;
+    const uint64_t timeout_ns = rg->timeout_ns;
     auto issue = [&](int j) {
         const int ch = cfirst + j * cstride;
         const int slot = (pos + j) % NS;
@@ -276,7 +294,7 @@ __device__ __forceinline__ void ring_stream(Ring* rg, const T* x, const T* y, in
     for (int j = 0; j < nj; ++j) {
         const int slot = (pos + j) % NS;
         const uint32_t parity = (uint32_t)((pos + j) / NS) & 1u;
-        bool ok = broken ? false : ring_wait(&bars[slot], parity, status, rg->timeout_ns);
+        bool ok = broken ? false : ring_wait(&bars[slot], parity, status, timeout_ns);
         broken = __any_sync(0xffffffffu, !ok);
         const int ch = cfirst + j * cstride;
         const int64_t e0 = (int64_t)ch * CE;
@@ -796,6 +814,11 @@ __device__ __forceinline__ void row_finish(const Problem<T>& P, int r, const Row
         rec.pad[0] = rec.pad[1] = rec.pad[2] = 0;
         rec.flags = ok ? 0 : 1;
         if (!ok) atomicOr(P.status, VSD_STATUS_BAD_ROW);
+        if (!ok && P.kl_topk) {  // an invalid row has no top-K term
+            P.klr[r].n = 0;
+            P.klr[r].loss = 0.f;
+            if (P.out.kl_loss) P.out.kl_loss[r] = 0.f;
+        }
         int t = tok;
         if (XMODE == kGivenToken && !tok_ok) {
             atomicOr(P.status, VSD_STATUS_BAD_TOKEN);
@@ -819,16 +842,26 @@ struct RowShared {
     RowTask t[3];
 };
 
+// VSD (KL): the row's top-K term of Eq. klv (defined below).
+template <typename T, bool VEC>
+__device__ void kl_select(const Problem<T>& P, int r, const float4* tab, int nch, uint4* buf,
+                          int npair, bool ok, int lane);
+
 // The per-row work once the row's chunk table tab[0..nch) is complete
 // (block, or with BAR > 0 the kThreads threads 0 .. kThreads-1 that meet at
 // named barrier BAR): warps 0, 1 and 2 take the three tasks at once, warp 0
 // then writes the record.
-template <typename T, bool VEC, bool HAS_Y, int XMODE, bool ARGMAX, int BAR = 0>
-__device__ void row_tail(const Problem<T>& P, int r, const float4* tab, RowShared& sh) {
+template <typename T, bool VEC, bool HAS_Y, int XMODE, bool ARGMAX, int BAR = 0, bool KL = false>
+__device__ void row_tail(const Problem<T>& P, int r, const float4* tab, RowShared& sh,
+                         uint4* klbuf = nullptr) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (warp == 0 || (HAS_Y && (warp == 1 || (ARGMAX && warp == 2)))) {
         const RowTask t = row_task<T, VEC, XMODE>(P, r, tab, warp, lane);
         if (lane == 0) sh.t[warp] = t;
+    } else if (KL && HAS_Y && warp == 3) {
+        // VSD (KL): the top-K term on the fourth warp (an invalid row's term
+        // is cleared by row_finish)
+        kl_select<T, VEC>(P, r, tab, P.nch, klbuf, 2, true, lane);
     }
     if (BAR == 0)
         __syncthreads();
@@ -884,6 +917,179 @@ __device__ __forceinline__ float smem_elem(const uint4* buf, int ch, int v, cons
         reinterpret_cast<const __nv_bfloat16*>(buf)[v - ch * chunk_elems<__nv_bfloat16>()]);
 }
 
+// --------------------------------------------------------------- VSD (KL)
+// The top-Kt tokens of the target row r (largest logit, lowest index on ties:
+// p's order at any T > 0) and the terms of Eq. klv on them (warp): p^ and q^
+// renormalised on those tokens, L = -sum p^ log q^, and the gradient
+// kl_scale (q^ - p^) of each token (log q^ = x/T - log sum over the tokens, so
+// the vocabulary's partition cancels and no other logit has a gradient).
+//
+// Only a chunk whose target maximum reaches the Kt-th largest chunk maximum
+// can hold a selected token (Kt chunk maxima are that large, so the Kt-th
+// largest logit is too).  The warp reads those chunks of both rows in
+// increasing order, skipping a chunk whose maximum cannot beat the current
+// Kt-th entry, and keeps the running list sorted by (logit desc, index asc)
+// in lanes 0 .. Kt-1.  buf stages npair chunk pairs in shared memory (null:
+// loads into registers, one pair at a time).  ok = false (an invalid row)
+// writes an empty term.
+template <typename T, bool VEC>
+__device__ void kl_select(const Problem<T>& P, int r, const float4* tab, int nch, uint4* buf,
+                          int npair, bool ok, int lane) {
+    constexpr int PV = Traits<T>::kPerVec;
+    constexpr int CE = chunk_elems<T>();
+    constexpr unsigned FULL = 0xffffffffu;
+    const int64_t V = P.V;
+    const T* x = P.draft + (int64_t)r * V;
+    const T* y = P.target + (int64_t)r * V;
+    KlRec* dst = P.klr + r;
+    const int Kt = (int)min((int64_t)P.kl_topk, V);
+    if (!ok) {
+        if (lane == 0) {
+            dst->n = 0;
+            dst->loss = 0.f;
+            if (P.out.kl_loss) P.out.kl_loss[r] = 0.f;
+        }
+        return;
+    }
+    // the Kt-th largest chunk maximum (order: value desc, chunk asc)
+    float tv = INFINITY, tk = -INFINITY;
+    int tch = -1;
+    for (int k = 0; k < Kt; ++k) {
+        float bv = -INFINITY;
+        int bc = 0x7fffffff;
+        for (int ch = lane; ch < nch; ch += 32) {
+            const float v = tab[ch].z;
+            const bool after = v < tv || (v == tv && ch > tch);
+            if (after && (v > bv || (v == bv && ch < bc))) {
+                bv = v;
+                bc = ch;
+            }
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+            const float ov = __shfl_xor_sync(FULL, bv, o);
+            const int oc = __shfl_xor_sync(FULL, bc, o);
+            if (ov > bv || (ov == bv && oc < bc)) {
+                bv = ov;
+                bc = oc;
+            }
+        }
+        if (bc == 0x7fffffff) {  // fewer chunks than Kt: every chunk is a candidate
+            tk = -INFINITY;
+            break;
+        }
+        tv = bv;
+        tch = bc;
+        tk = bv;
+    }
+    float lv = -INFINITY, lx = 0.f;  // lane i < Kt: entry i (target logit, draft logit, index)
+    int li = 0x7fffffff;
+    int cnt = 0;
+    float thv = -INFINITY;
+    int thi = 0x7fffffff;
+    auto insert = [&](float v, int idx, float xv) {
+        const bool above = lane < cnt && (lv > v || (lv == v && li < idx));
+        const int pos = __popc(__ballot_sync(FULL, above));
+        if (pos >= Kt) return;
+        const float pv = __shfl_up_sync(FULL, lv, 1);
+        const int pi = __shfl_up_sync(FULL, li, 1);
+        const float px = __shfl_up_sync(FULL, lx, 1);
+        if (lane > pos) {
+            lv = pv;
+            li = pi;
+            lx = px;
+        }
+        if (lane == pos) {
+            lv = v;
+            li = idx;
+            lx = xv;
+        }
+        cnt = min(cnt + 1, Kt);
+        if (cnt == Kt) {
+            thv = __shfl_sync(FULL, lv, Kt - 1);
+            thi = __shfl_sync(FULL, li, Kt - 1);
+        }
+    };
+    auto scan_chunk = [&](int ch, const uint4 (&bx)[kLoads], const uint4 (&by)[kLoads]) {
+#pragma unroll
+        for (int k = 0; k < kLoads; ++k) {
+            float fx[PV], fy[PV];
+            unpack<T>(bx[k], fx);
+            unpack<T>(by[k], fy);
+#pragma unroll
+            for (int e = 0; e < PV; ++e) {
+                const int idx = ch * CE + k * 32 * PV + lane * PV + e;
+                const bool c = idx < V && (cnt < Kt || fy[e] > thv || (fy[e] == thv && idx < thi));
+                for (unsigned m = __ballot_sync(FULL, c); m; m &= m - 1) {
+                    const int L = __ffs(m) - 1;
+                    insert(__shfl_sync(FULL, fy[e], L), __shfl_sync(FULL, idx, L),
+                           __shfl_sync(FULL, fx[e], L));
+                }
+            }
+        }
+    };
+    const int np = (VEC && buf) ? max(1, min(npair, 3)) : 1;
+    const uint64_t pol = policy_evict_normal();
+    int ch0 = 0;
+    for (;;) {
+        int cand[3] = {-1, -1, -1};
+        int nc = 0;
+        while (nc < np && ch0 < nch) {
+            const int ch = ch0 + lane;
+            const float mxc = ch < nch ? tab[ch].z : -INFINITY;
+            const bool want = ch < nch && mxc >= tk && (cnt < Kt || mxc > thv);
+            unsigned bal = __ballot_sync(FULL, want);
+            while (bal && nc < np) {
+                cand[nc++] = ch0 + __ffs(bal) - 1;
+                bal &= bal - 1;
+            }
+            ch0 = bal ? ch0 + __ffs(bal) - 1 : ch0 + 32;
+        }
+        if (nc == 0) break;
+        if (VEC && buf) {
+            for (int j = 0; j < nc; ++j) {
+                chunk_async<T>(buf + (2 * j) * kLoads * 32, x, V, cand[j], lane);
+                chunk_async<T>(buf + (2 * j + 1) * kLoads * 32, y, V, cand[j], lane);
+            }
+            cp_async_wait_all();
+            __syncwarp();
+            for (int j = 0; j < nc; ++j) {
+                uint4 bx[kLoads], by[kLoads];
+                chunk_from_smem<T>(buf + (2 * j) * kLoads * 32, V, cand[j], lane, bx);
+                chunk_from_smem<T>(buf + (2 * j + 1) * kLoads * 32, V, cand[j], lane, by);
+                scan_chunk(cand[j], bx, by);
+            }
+            __syncwarp();
+        } else {
+            uint4 bx[kLoads], by[kLoads];
+            load_chunk<T, VEC>(x, V, cand[0], lane, pol, bx);
+            load_chunk<T, VEC>(y, V, cand[0], lane, pol, by);
+            scan_chunk(cand[0], bx, by);
+        }
+    }
+    // Eq. klv on the selected tokens (fp64; the list is sorted, lane 0 holds
+    // the largest target logit)
+    const bool mine = lane < Kt;
+    const double invT = P.ts.invTd;
+    const double y0 = (double)__shfl_sync(FULL, lv, 0);
+    const double xm = (double)warp_max(mine ? lx : -INFINITY);
+    const double ep = mine ? exp(((double)lv - y0) * invT) : 0.0;
+    const double eq = mine ? exp(((double)lx - xm) * invT) : 0.0;
+    const double Sp = warp_sum(ep), Sq = warp_sum(eq);
+    const double ph = ep / Sp;
+    const double lqh = ((double)lx - xm) * invT - log(Sq);
+    const double L = warp_sum((mine && ph > 0.0) ? -ph * lqh : 0.0);
+    if (mine) {
+        dst->tok[lane] = li;
+        dst->coef[lane] = (float)(P.kl_scale * (exp(lqh) - ph));
+    }
+    if (lane == 0) {
+        dst->loss = (float)L;
+        dst->n = Kt;
+        if (P.out.kl_loss) P.out.kl_loss[r] = (float)L;
+    }
+}
+
 // Shared memory of the fused kernel's control warp: the six chunks a row tail
 // rescans, or the M-step's scratch (never both at once).
 struct RescanBuf {
@@ -897,7 +1103,7 @@ struct RescanBuf {
 // draws' table work, then one round trip (cp.async) for the draft and target
 // chunks at the three chunks the draws rescan, which also hold the logits of
 // the tokens they return.  Same tokens and record as row_tail.
-template <typename T, bool VEC>
+template <typename T, bool VEC, bool KL = false>
 __device__ void row_tail_warp(const Problem<T>& P, int r, float4* tab, RescanBuf& rb, int lane) {
     const int64_t V = P.V;
     const int nch = P.nch;
@@ -960,6 +1166,11 @@ __device__ void row_tail_warp(const Problem<T>& P, int r, float4* tab, RescanBuf
                                                     yv = elem_value(y, v);
                                                 }
                                             });
+    if (KL) {  // VSD (KL): the row's top-K term, staged through the rescan buffers
+        __syncwarp();
+        kl_select<T, VEC>(P, r, tab, nch, rb.c[0], 3,
+                          row_ok(tx.M, tx.S.Z) && row_ok(ty.M, ty.S.Z), lane);
+    }
 }
 
 // Streams row r of the draft (and, with HAS_Y, of the target) once, then runs
@@ -1459,7 +1670,13 @@ __device__ void weights_warp(const Problem<T>& P, const EStepView& E, int b, flo
             sh.lqc[s] = c1;
         }
     }
-    if (lane == 0) loss_out[b] = N > 0.f ? -J / N : 0.f;
+    float klterm = 0.f;
+    if (P.kl_topk) {  // VSD (KL): + kl_weight (1/K) sum of the prefix's rows' top-K terms
+        double sk = 0.0;
+        for (int i = lane; i < K * D; i += 32) sk += (double)ld_cg(&P.klr[b * K * D + i].loss);
+        klterm = (float)(P.kl_weight / (double)K * warp_sum(sk));
+    }
+    if (lane == 0) loss_out[b] = (N > 0.f ? -J / N : 0.f) + klterm;
 }
 
 // The M-step by a block: warp 0 runs weights_warp (the same bits as the fused
@@ -1507,7 +1724,7 @@ __device__ __forceinline__ void grad_store(G* g, int64_t v0, const float (&o)[PV
 // e1 are multiples of the vector width.
 template <typename T, bool VEC, typename G>
 __device__ void grad_pass_range(const Problem<T>& P, int r, int64_t e0, int64_t e1,
-                                const float4* rstats, G* grad) {
+                                const float4* rstats, G* grad, const KlRec* kl = nullptr) {
     constexpr int PV = Traits<T>::kPerVec;
     constexpr int U = 8;  // vectors per batch per thread (two batches in flight)
     const int64_t V = P.V;
@@ -1566,10 +1783,13 @@ __device__ void grad_pass_range(const Problem<T>& P, int r, int64_t e0, int64_t 
             for (int u = 0; u < U; ++u) cur[u] = nxt[u];
         }
     } else {
+        const int nkl = kl ? min(max(kl->n, 0), kMaxKlTop) : 0;
         for (int64_t v = e0 + threadIdx.x; v < e1; v += kThreads) {
             float val = gq * ex2((elem_value(x, v) - mx) * c);
             if (v == cf.t0) val -= cf.c0;
             if (v == cf.t1) val -= cf.c1;
+            for (int k = 0; k < nkl; ++k)
+                if (v == kl->tok[k]) val += kl->coef[k];
             if constexpr (sizeof(G) == 2)
                 g[v] = __float2bfloat16_rn(val);
             else
@@ -1580,14 +1800,17 @@ __device__ void grad_pass_range(const Problem<T>& P, int r, int64_t e0, int64_t 
 
 // Gradient of chunks [c0, c1) of row r (warp level, through the ring; the
 // streaming warps of the fused kernel).  Same arithmetic as grad_pass_range.
-template <typename T, bool VEC, typename G>
-__device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1, G* grad) {
+// KL: the row has top-K terms (VSD (KL)) in kl; without them the loop is the
+// plain one.
+template <typename T, bool VEC, typename G, bool KL = false>
+__device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1, G* grad,
+                            const KlRec* kl = nullptr) {
     constexpr int PV = Traits<T>::kPerVec;
     constexpr int CE = chunk_elems<T>();
     const int64_t V = P.V;
     if constexpr (!VEC) {
         grad_pass_range<T, VEC, G>(P, r, (int64_t)c0 * CE, min(V, (int64_t)c1 * CE), P.rstats,
-                                   grad);
+                                   grad, kl);
     } else {
         constexpr int NP = PV / 2;
         const int lane = threadIdx.x & 31;
@@ -1599,8 +1822,17 @@ __device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1
         const float gq = cf.g * rec.izx;  // g / Z
         const uint64_t pol = policy_evict_first();
         const uint64_t mx2 = f2(rec.mx, rec.mx), c2 = f2(c, c), gq2 = f2(gq, gq);
-        // the sparse terms touch at most two positions of the row
-        auto emit = [&](int64_t v0, float (&o)[PV]) {
+        const int nkl = KL ? min(max(kl->n, 0), kMaxKlTop) : 0;
+        // VSD (KL): which of the row's top-K terms fall in chunk ch (a
+        // warp-uniform mask; called where the warp is converged)
+        auto kl_mask = [&](int ch) -> unsigned {
+            if (!KL || !nkl) return 0u;
+            const bool in = lane < nkl && (unsigned)(kl->tok[lane] - ch * CE) < (unsigned)CE;
+            return __ballot_sync(0xffffffffu, in);
+        };
+        // the sparse terms touch at most two positions of the row, plus the
+        // top-K terms of the chunk
+        auto emit = [&](int64_t v0, float (&o)[PV], unsigned km) {
             if ((uint64_t)(cf.t0 - v0) < (uint64_t)PV) {
 #pragma unroll
                 for (int e = 0; e < PV; ++e)
@@ -1611,6 +1843,16 @@ __device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1
                 for (int e = 0; e < PV; ++e)
                     if (v0 + e == cf.t1) o[e] -= cf.c1;
             }
+            for (unsigned m = KL ? km : 0u; m; m &= m - 1) {
+                const int k = __ffs(m) - 1;
+                const int t = kl->tok[k];
+                if ((uint64_t)(t - v0) < (uint64_t)PV) {
+                    const float ck = kl->coef[k];
+#pragma unroll
+                    for (int e = 0; e < PV; ++e)
+                        if (v0 + e == t) o[e] += ck;
+                }
+            }
             grad_store<T, G, PV>(g, v0, o, pol);
         };
         if (cf.g == 0.f && isfinite(rec.mx)) {
@@ -1618,6 +1860,7 @@ __device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1
             // draft row is not read (rows no objective term reaches).
             const int warp = threadIdx.x >> 5;
             for (int ch = c0 + warp; ch < c1; ch += kWarps) {
+                const unsigned km = kl_mask(ch);
 #pragma unroll
                 for (int k = 0; k < kLoads; ++k) {
                     const int64_t v0 = (int64_t)ch * CE + (int64_t)k * 32 * PV + lane * PV;
@@ -1625,7 +1868,7 @@ __device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1
                     float o[PV];
 #pragma unroll
                     for (int e = 0; e < PV; ++e) o[e] = 0.f;
-                    emit(v0, o);
+                    emit(v0, o, km);
                 }
             }
             return;
@@ -1633,6 +1876,7 @@ __device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1
         ring_stream<T, false>(
             rg, x, nullptr, V, c0, c1, pol, pol, P.status,
             [&](int ch, const uint4 (&bx)[kLoads], const uint4 (&)[kLoads]) {
+                const unsigned km = kl_mask(ch);
 #pragma unroll
                 for (int k = 0; k < kLoads; ++k) {
                     const int64_t v0 = (int64_t)ch * CE + (int64_t)k * 32 * PV + lane * PV;
@@ -1643,7 +1887,7 @@ __device__ void stream_grad(Ring* rg, const Problem<T>& P, int r, int c0, int c1
 #pragma unroll
                     for (int q = 0; q < NP; ++q)
                         f2split(f2mul(f2_mass(pr[q], mx2, c2), gq2), o[2 * q], o[2 * q + 1]);
-                    emit(v0, o);
+                    emit(v0, o, km);
                 }
             });
     }

@@ -42,12 +42,14 @@ class Layout(C.Structure):
 class Params(C.Structure):
     _fields_ = [("w_base", C.c_double), ("tau_car", C.c_double), ("zeta_mode", C.c_int32),
                 ("grad_dtype", C.c_int32), ("wait_timeout_ns", C.c_uint64),
-                ("test_never_publish", C.c_int32)]
+                ("test_never_publish", C.c_int32), ("kl_weight", C.c_double),
+                ("kl_topk", C.c_int32)]
 
 
 LINEAR_FIELDS = ("tokens", "logq_tok", "alpha", "accept", "accept_len", "corr_tokens",
                  "logq_corr", "alpha_corr", "logkappa", "logkappa_corr", "logkappa_ref",
-                 "ref_tokens", "expected_len", "row_stats", "weights", "loss", "grad")
+                 "ref_tokens", "expected_len", "row_stats", "weights", "loss", "grad",
+                 "kl_loss")
 TREE_FIELDS = ("alpha", "accept", "path_accept", "logkappa", "corr_tokens", "deepest",
                "accept_len", "bonus", "row_stats")
 
@@ -162,13 +164,13 @@ def new_workspace(lay, device):
 
 
 def params(w_base=1.05, tau_car=0.2, zeta_mode=0, grad_dtype=None, wait_timeout_ns=0,
-           test_never_publish=0, like=None):
+           test_never_publish=0, like=None, kl_weight=0.0, kl_topk=10):
     if grad_dtype is None:
         grad_dtype = VSD_BF16 if (like is not None and like.dtype == torch.bfloat16) else VSD_F32
     elif isinstance(grad_dtype, torch.dtype):
         grad_dtype = VSD_BF16 if grad_dtype == torch.bfloat16 else VSD_F32
     return Params(float(w_base), float(tau_car), int(zeta_mode), int(grad_dtype),
-                  int(wait_timeout_ns), int(test_never_publish))
+                  int(wait_timeout_ns), int(test_never_publish), float(kl_weight), int(kl_topk))
 
 
 def _ws(ws, lay, device):
@@ -185,8 +187,9 @@ def _rows(x, V):
     return x.numel() // V
 
 
-def linear_outputs(B, K, D, V, device, grad_dtype=torch.bfloat16, grad=True, full=True):
-    """Allocate the output tensors of the linear E-step / M-step."""
+def linear_outputs(B, K, D, V, device, grad_dtype=torch.bfloat16, grad=True, full=True, kl=False):
+    """Allocate the output tensors of the linear E-step / M-step (kl: the
+    per-row top-K terms of VSD (KL) too)."""
     R = B * K * D
     f = dict(device=device)
     o = dict(tokens=torch.empty(R, dtype=torch.int32, **f),
@@ -206,6 +209,8 @@ def linear_outputs(B, K, D, V, device, grad_dtype=torch.bfloat16, grad=True, ful
                  expected_len=torch.empty(B * K, dtype=torch.float32, **f),
                  row_stats=torch.empty(R, 4, dtype=torch.float32, **f),
                  weights=torch.empty(B, D, K, 4, dtype=torch.float32, **f))
+    if kl:
+        o["kl_loss"] = torch.empty(R, dtype=torch.float32, **f)
     if grad:
         o["grad"] = torch.empty(R, V, dtype=grad_dtype, **f)
     return o
@@ -328,7 +333,7 @@ def estep_mstep(draft, target, u_draft, u_accept, u_correct, K, D, T, ref_logkap
     prm = prm or params(like=draft)
     if out is None:
         gdt = torch.bfloat16 if prm.grad_dtype == VSD_BF16 else torch.float32
-        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full)
+        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full, kl=prm.kl_weight != 0)
     st = _linear_struct(out)
     _check(_lib().vsd_estep_mstep(_ptr(draft), _ptr(target), _dtype_code(draft), lay, float(T),
                                   _ptr(u_draft), _ptr(u_accept), _ptr(u_correct),
@@ -374,7 +379,7 @@ def lmhead_estep_mstep(hidden, weight, target, u_draft, u_accept, u_correct, K, 
         draft_logits = torch.empty(R, V, dtype=torch.bfloat16, device=dev)
     if out is None:
         gdt = torch.bfloat16 if prm.grad_dtype == VSD_BF16 else torch.float32
-        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full)
+        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full, kl=prm.kl_weight != 0)
     st = _linear_struct(out)
     _check(_lib().vsd_lmhead_estep_mstep(_ptr(hidden), _ptr(weight), H, _ptr(target), lay,
                                          float(T), _ptr(u_draft), _ptr(u_accept),
@@ -401,7 +406,7 @@ def estep_mstep_noalloc(draft, target, u_draft, u_accept, u_correct, K, D, T,
     prm = prm or params(like=draft)
     if out is None:
         gdt = torch.bfloat16 if prm.grad_dtype == VSD_BF16 else torch.float32
-        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full)
+        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full, kl=prm.kl_weight != 0)
     st = _linear_struct(out)
     _check(_lib().vsd_estep_mstep_noalloc(_ptr(draft), _ptr(target), _dtype_code(draft), lay,
                                           float(T), _ptr(u_draft), _ptr(u_accept),

@@ -101,7 +101,10 @@ def _grad_rows(name, g_rows, o_rows, grad_dtype, scale):
     assert badr.size == 0, "%s rows off: %s, max err %g (scale %g)" % (
         name, badr[:8], np.nanmax(err[badr]), scale)
     emax = float(err.max()) if err.size else 0.0
-    assert emax <= 1e-3, "%s max-abs error %g" % (name, emax)  # max-abs bar for gradients
+    # the max-abs bar for gradients (fp32); a bf16 gradient adds the rounding
+    # of its largest entry, 2^-8 relative
+    bar = 1e-3 + (2.0 ** -8 * scale if grad_dtype == "bf16" else 0.0)
+    assert emax <= bar, "%s max-abs error %g (bar %g)" % (name, emax, bar)
     return emax
 
 
@@ -164,13 +167,23 @@ def _conditional_mstep(gpu, b, K, D, V, T, grad_dtype, mi, check_grad, scale):
     draft = np.asarray(mi["draft_rows"](b), dtype=np.float32).reshape(K, D, V)
     J, g = orc_mod.prefix_objective(draft, T, tok, corr, w, N, mi["B_total"],
                                     want_grad=check_grad)
+    lam = mi.get("kl_weight", 0.0)
+    kl = 0.0
+    if lam:  # VSD (KL): the rows' top-K terms depend on the logits alone
+        target = np.asarray(mi["target_rows"](b), dtype=np.float32).reshape(K * D, V)
+        dr = draft.reshape(K * D, V)
+        for i in range(K * D):
+            Li, toks, dl = orc_mod.topk_ce(dr[i], target[i], T, mi.get("kl_topk", 10))
+            kl += Li
+            if check_grad:
+                g.reshape(K * D, V)[i, toks] += lam / (mi["B_total"] * K) * dl
     if gpu.get("weights") is not None:
         wg = to_np(gpu["weights"]).reshape(-1, D, K, 4)[b]
         assert np.array_equal(wg[..., 0], w[..., 0]), "o~ (conditional) prefix %d" % b
         assert np.allclose(wg[..., 1], w[..., 1], rtol=1e-6, atol=0), "o' (conditional)"
         assert np.allclose(wg[..., 2], w[..., 2], rtol=1e-5, atol=1e-6), "beta (conditional)"
         assert np.allclose(wg[..., 3], w[..., 3], rtol=1e-5, atol=1e-6), "zeta (conditional)"
-    lo = -J / N if N > 0 else 0.0
+    lo = (-J / N if N > 0 else 0.0) + lam * kl / K
     lg = float(to_np(gpu["loss"])[b])
     assert abs(lg - lo) <= LOSS_RTOL * max(1.0, abs(lo)), \
         "loss[%d] (conditional) gpu %r oracle %r" % (b, lg, lo)
@@ -183,7 +196,7 @@ def _conditional_mstep(gpu, b, K, D, V, T, grad_dtype, mi, check_grad, scale):
 
 
 def compare_linear(gpu, orc, B, K, D, V, T, grad_dtype="f32", check_grad=True, report=None,
-                   check_mean=True, mstep_inputs=None):
+                   check_mean=True, mstep_inputs=None, kl=False):
     """Assert parity of E-step/M-step outputs under the protocol above;
     returns the number of prefixes whose M-step was not compared end to end
     (checked conditionally, or excluded).
@@ -192,7 +205,8 @@ def compare_linear(gpu, orc, B, K, D, V, T, grad_dtype="f32", check_grad=True, r
     draft_rows(b) -> the prefix's draft logits [K*D, V], B_total (the call's
     number of prefixes, which scales the gradient), and the call's w_base,
     tau_car, zeta_mode when not the defaults.  With check_mean=False the mean
-    loss entry is not compared (a sub-batch of a larger call, see sub_batch)."""
+    loss entry is not compared (a sub-batch of a larger call, see sub_batch).
+    kl: the call ran VSD (KL) (the per-row top-K terms are compared too)."""
     f, tmis = _first_divergence(gpu, orc, B, K, D)
     npaths = B * K
     path_div = f < D
@@ -225,6 +239,8 @@ def compare_linear(gpu, orc, B, K, D, V, T, grad_dtype="f32", check_grad=True, r
     close("alpha", ALPHA_ATOL, 0.0, tok_ok)
     close("logq_tok", 2e-5, 1e-6, tok_ok)
     close("logkappa_ref", LOGK_MARGIN, 1e-6, np.ones(B * K * D, bool))
+    if kl:  # VSD (KL): the row's top-K term depends on its logits alone
+        close("kl_loss", 1e-5, 1e-5, np.ones(B * K * D, bool))
     if gpu.get("row_stats") is not None:
         rs = to_np(gpu["row_stats"]).reshape(-1, 4).astype(np.float64)
         _close_mask("row lse q", rs[:, 0] / T + rs[:, 1], orc["row_lse"][:, 0], 2e-5, 1e-6,
@@ -313,18 +329,20 @@ def compare_linear(gpu, orc, B, K, D, V, T, grad_dtype="f32", check_grad=True, r
     return ncond
 
 
-def mstep_inputs(prob, B_total=None, w_base=1.05, tau_car=0.2, zeta_mode=0):
-    """The inputs of the conditional M-step check for a problem dict (draft
-    logits [B*K*D, V] on any device), as compare_linear takes them."""
+def mstep_inputs(prob, B_total=None, w_base=1.05, tau_car=0.2, zeta_mode=0, kl_weight=0.0,
+                 kl_topk=10):
+    """The inputs of the conditional M-step check for a problem dict (draft and
+    target logits [B*K*D, V] on any device), as compare_linear takes them."""
     P = prob["K"] * prob["D"]
-    draft = prob["draft"]
 
-    def rows(b):
-        x = draft[b * P:(b + 1) * P]
-        return to_np(x).astype(np.float32)
+    def rows(name):
+        def get(b):
+            return to_np(prob[name][b * P:(b + 1) * P]).astype(np.float32)
+        return get
 
-    return dict(draft_rows=rows, B_total=B_total or prob["B"], w_base=w_base, tau_car=tau_car,
-                zeta_mode=zeta_mode)
+    return dict(draft_rows=rows("draft"), target_rows=rows("target") if "target" in prob else None,
+                B_total=B_total or prob["B"], w_base=w_base, tau_car=tau_car,
+                zeta_mode=zeta_mode, kl_weight=kl_weight, kl_topk=kl_topk)
 
 
 def sub_batch(gpu, b0, b1, B, K, D):

@@ -118,7 +118,8 @@ def _gpu_view(o):
     return gpu
 
 
-def test_flipped_draw_is_checked_conditionally(oracle):
+@pytest.mark.parametrize("lam", [0.0, 0.4])
+def test_flipped_draw_is_checked_conditionally(oracle, lam):
     """A consistent result that took one near-boundary draft draw the other
     way (the oracle itself run with that row's uniform moved across the CDF
     boundary by one float step) passes: the flipped path is compared up to
@@ -138,19 +139,21 @@ def test_flipped_draw_is_checked_conditionally(oracle):
     assert float(below) < F <= float(above)
     f["u_draft"][r] = below
     orc = oracle.linear(f["draft"], f["target"], 1.0, f["u_draft"], f["u_accept"],
-                        f["u_correct"], K, D)
+                        f["u_correct"], K, D, kl_weight=lam)
     f2 = dict(f)
     f2["u_draft"] = f["u_draft"].copy()
     f2["u_draft"][r] = above
     o2 = oracle.linear(f2["draft"], f2["target"], 1.0, f2["u_draft"], f2["u_accept"],
-                       f2["u_correct"], K, D)
+                       f2["u_correct"], K, D, kl_weight=lam)
     assert o2["tokens"][r] != orc["tokens"][r] and orc["margins"][r, 0] < parity.PROB_MARGIN
     gpu = _gpu_view(o2)
     P = K * D
-    mi = dict(draft_rows=lambda b: f["draft"][b * P:(b + 1) * P], B_total=B)
+    mi = dict(draft_rows=lambda b: f["draft"][b * P:(b + 1) * P],
+              target_rows=lambda b: f["target"][b * P:(b + 1) * P], B_total=B, kl_weight=lam)
+    gpu["kl_loss"] = o2["kl_loss"].astype(np.float32)
     rep = {}
     assert parity.compare_linear(gpu, orc, B, K, D, V, 1.0, grad_dtype="f32", report=rep,
-                                 mstep_inputs=mi) == 1
+                                 mstep_inputs=mi, kl=lam > 0) == 1
     assert rep["diverged_paths"] == 1 and rep["conditional_prefixes"] == 1
     bad = _gpu_view(o2)
     bad["loss"][1] += 1e-3
