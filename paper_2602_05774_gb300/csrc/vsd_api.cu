@@ -391,7 +391,7 @@ vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float
                       const float* u_draft, const float* u_accept, const float* u_correct,
                       const float* ref_logkappa, const vsd_params& p,
                       const vsd_linear_outputs* out, void* ws, cudaStream_t s,
-                      bool clear = true) {
+                      bool clear = true, bool xtab_given = false) {
     Problem<T> P = make_problem<T>(draft, target, L, T_, ws);
     set_params(P, p);
     P.u_draft = u_draft;
@@ -412,6 +412,7 @@ vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float
     // there the claims of the streaming jobs bound it).  Measured on GB300:
     // V=32000 0.107 vs 0.136 ms, V=128256 0.669 vs 0.642 ms.
     P.resq_sem = P.stream_tails;
+    P.xtab_given = xtab_given ? 1 : 0;
     const int64_t tickets = (int64_t)P.R * (P.nseg + P.gnseg);
     int ctas = per_sm * num_sms();
     if ((int64_t)ctas > tickets) ctas = (int)tickets;
@@ -557,14 +558,19 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
     if ((st = check_params(p))) return st;
     if ((st = check_ws(layout, ws, ws_bytes))) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    // the counters and the status word are cleared once, before both steps
+    // the counters and the status word are cleared once, before both steps;
+    // the GEMM's epilogue writes the draft half of every row's chunk table
+    // (a1 for the draft), so the E-step streams only the target rows
+    const WsLayout w = ws_layout(layout);
+    const float c = (float)(kLog2e / (double)T);
     cudaError_t e = clear_counters(ws, layout, s);
     if (e == cudaSuccess)
         e = lmhead_gemm(hidden, weight, (int)R, layout.V, H, draft_logits, static_cast<int*>(ws),
-                        p.wait_timeout_ns ? p.wait_timeout_ns : kDefaultTimeoutNs, s);
+                        p.wait_timeout_ns ? p.wait_timeout_ns : kDefaultTimeoutNs, s,
+                        at<float4>(ws, w.gtab), w.nch_ws, c);
     if (e != cudaSuccess) return from_cuda(e);
     return fused_impl<__nv_bfloat16>(draft_logits, target, layout, T, u_draft, u_accept,
-                                     u_correct, ref_logkappa, p, out, ws, s, false);
+                                     u_correct, ref_logkappa, p, out, ws, s, false, true);
 }
 
 vsd_status vsd_device_status(void* ws, void* stream, int32_t* status_bits) {

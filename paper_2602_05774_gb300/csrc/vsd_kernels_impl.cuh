@@ -407,9 +407,18 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
             if (j.kind == kJobRow) {
                 // The draft row is read again for the gradient: ask L2 to keep it.
                 float4* rtab = P.gtab + (int64_t)j.r * P.nch_ws;
-                stream_tables<T, VEC, true>(rg, x, P.target + (int64_t)j.r * V, V, j.c0, j.c1,
-                                            rtab, P.ts.c, policy_evict_last(),
-                                            policy_evict_first(), P.status);
+                bool both = true;
+                if constexpr (VEC) {
+                    if (P.xtab_given) {  // the LM head wrote the draft's statistics
+                        stream_target_tables<T>(rg, P.target + (int64_t)j.r * V, V, j.c0, j.c1,
+                                                rtab, P.ts.c, policy_evict_first(), P.status);
+                        both = false;
+                    }
+                }
+                if (both)
+                    stream_tables<T, VEC, true>(rg, x, P.target + (int64_t)j.r * V, V, j.c0,
+                                                j.c1, rtab, P.ts.c, policy_evict_last(),
+                                                policy_evict_first(), P.status);
                 if (P.stream_tails) {  // short rows: the tail here, three draws at once
                     asm volatile("bar.sync %0, %1;" ::"r"(kStreamBar), "r"(kThreads) : "memory");
                     row_tail<T, VEC, true, kSampleToken, true, kStreamBar, KL>(

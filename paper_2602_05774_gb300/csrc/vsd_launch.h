@@ -53,7 +53,11 @@ inline size_t stream_smem_bytes(int nch, bool vec) {
 // weight^T, bf16 in, fp32 accumulation, bf16 out; status collects timeouts.
 bool lmhead_shape_ok(const void* hidden, const void* weight, const void* logits, int M, int N,
                      int K);
+// With chunk_tab, the epilogue also writes chunk_tab[r * chunk_stride + ch].xy
+// = (max, sum 2^{(x - max) chunk_c}) of row r's bf16 logits x in columns
+// [1024 ch, 1024 ch + 1024): the draft half of the E-step's chunk table.
 cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, int K, void* logits,
-                        int* status, uint64_t timeout_ns, cudaStream_t s);
+                        int* status, uint64_t timeout_ns, cudaStream_t s,
+                        float4* chunk_tab = nullptr, int chunk_stride = 0, float chunk_c = 0.f);
 
 }  // namespace vsd

@@ -11,7 +11,9 @@
 //            N=256, K=16) into one of two TMEM accumulators (2 x 256 columns);
 //            tcgen05.commit frees a ring stage / hands a finished accumulator on;
 //   warps 2-5 epilogue: tcgen05.ld of the accumulator (each warp its 32 TMEM
-//            lanes = 32 tile rows), rounding to bf16, 16-byte stores.
+//            lanes = 32 tile rows), rounding to bf16, 16-byte stores, and, for
+//            the fused E-step, each row's chunk statistics of the rounded
+//            logits (max, sum 2^{(x - max) c}) over 1024-column chunks.
 // The epilogue of one tile overlaps the main loop of the next.  Every wait is
 // bounded; a wait that runs out sets VSD_STATUS_TIMEOUT in the status word and
 // the CTA winds down (waiting, again bounded, for its copies and MMAs in
@@ -174,19 +176,37 @@ __device__ __forceinline__ uint32_t pack_bf16(uint32_t lo, uint32_t hi) {
     return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// Tiles are numbered with the M tile fastest, so the CTAs working at the same
-// time share the same few weight tiles (read from DRAM once, then from L2) and
-// the hidden states stay in L2 throughout.
+// Work is cut into units of one 128-row M tile by one 1024-column chunk (the
+// E-step's chunk of bf16 logits): kTilesPerChunk consecutive 128 x 256 tiles,
+// computed by one CTA in turn, so that its epilogue threads (one per row) can
+// carry a row's running (max, sum 2^{(x - max) c}) over the chunk.  Units are
+// numbered with the M tile fastest, so the CTAs working at the same time share
+// the same few weight tiles (read from DRAM once, then from L2) and the hidden
+// states stay in L2 throughout.
+constexpr int kChunkCols = 1024;
+constexpr int kTilesPerChunk = kChunkCols / BN;
+static_assert(kChunkCols % BN == 0, "a chunk is a whole number of tiles");
+
+// Chunk statistics of the logits for the E-step (a1 of the hot path): for
+// row r and chunk ch, tab[r * stride + ch].xy = (max, sum 2^{(x - max) c}) of
+// the bf16-rounded logits x of the chunk, c = log2(e) / T.
+struct ChunkStatsOut {
+    float4* tab;   // null: none
+    int stride;    // float4 entries per row
+    float c;
+};
+
 __global__ void __launch_bounds__(kThreads, 1)
     k_lmhead(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
              __nv_bfloat16* __restrict__ out, int M, int N, int K, int* status,
-             uint64_t timeout_ns) {
+             uint64_t timeout_ns, ChunkStatsOut cs) {
     extern __shared__ unsigned char dsm_raw[];
     unsigned char* dsm = dsm_raw + ((1024u - (smem_u32(dsm_raw) & 1023u)) & 1023u);
     Bars* sb = reinterpret_cast<Bars*>(dsm + kStages * kStageBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int mt = (M + BM - 1) / BM, nt = (N + BN - 1) / BN;
-    const int ntiles = mt * nt, nk = (K + BK - 1) / BK;
+    const int mt = (M + BM - 1) / BM, ntn = (N + BN - 1) / BN;
+    const int nchunks = (ntn + kTilesPerChunk - 1) / kTilesPerChunk;
+    const int nunits = mt * nchunks, nk = (K + BK - 1) / BK;
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&sb->full[s], 1);
@@ -215,23 +235,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------ TMA producer
         if (lane == 0) {
             uint32_t it = 0;
-            for (int t = blockIdx.x; t < ntiles && !*(volatile int*)&sb->err; t += gridDim.x) {
-                const int m0 = (t % mt) * BM, n0 = (t / mt) * BN;
-                bool ok = true;
-                for (int kb = 0; kb < nk; ++kb) {
-                    const int s = (int)(it % kStages);
-                    const uint32_t round = it / kStages;
-                    if (round > 0 && !wait_phase(&sb->empty[s], (round - 1) & 1u, sb, status)) {
-                        ok = false;
-                        break;
+            bool ok = true;
+            for (int u = blockIdx.x; ok && u < nunits && !*(volatile int*)&sb->err;
+                 u += gridDim.x) {
+                const int m0 = (u % mt) * BM, nt0 = (u / mt) * kTilesPerChunk;
+                const int nt1 = min(nt0 + kTilesPerChunk, ntn);
+                for (int nt = nt0; ok && nt < nt1; ++nt) {
+                    const int n0 = nt * BN;
+                    for (int kb = 0; kb < nk; ++kb) {
+                        const int s = (int)(it % kStages);
+                        const uint32_t round = it / kStages;
+                        if (round > 0 && !wait_phase(&sb->empty[s], (round - 1) & 1u, sb, status)) {
+                            ok = false;
+                            break;
+                        }
+                        unsigned char* a = dsm + s * kStageBytes;
+                        mbar_expect_tx(&sb->full[s], kStageBytes);
+                        tma_load_2d(a, &tmA, kb * BK, m0, &sb->full[s]);
+                        tma_load_2d(a + kABytes, &tmB, kb * BK, n0, &sb->full[s]);
+                        ++it;
                     }
-                    unsigned char* a = dsm + s * kStageBytes;
-                    mbar_expect_tx(&sb->full[s], kStageBytes);
-                    tma_load_2d(a, &tmA, kb * BK, m0, &sb->full[s]);
-                    tma_load_2d(a + kABytes, &tmB, kb * BK, n0, &sb->full[s]);
-                    ++it;
                 }
-                if (!ok) break;
             }
             // the last copies issued have landed before the CTA may exit
             for (uint32_t j = it > (uint32_t)kStages ? it - kStages : 0; j < it; ++j)
@@ -242,31 +266,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             uint32_t it = 0;
             int lt = 0;
-            for (int t = blockIdx.x; t < ntiles && !*(volatile int*)&sb->err;
-                 t += gridDim.x, ++lt) {
-                const int buf = lt & 1;
-                const uint32_t use = (uint32_t)lt >> 1;
-                if (use > 0 && !wait_phase(&sb->acc_empty[buf], (use - 1) & 1u, sb, status)) break;
-                tc_fence_after();
-                const uint32_t d = tmem + (uint32_t)(buf * BN);
-                bool ok = true;
-                for (int kb = 0; kb < nk; ++kb) {
-                    const int s = (int)(it % kStages);
-                    if (!wait_phase(&sb->full[s], (it / kStages) & 1u, sb, status)) {
+            bool ok = true;
+            for (int u = blockIdx.x; ok && u < nunits && !*(volatile int*)&sb->err;
+                 u += gridDim.x) {
+                const int nt0 = (u / mt) * kTilesPerChunk, nt1 = min(nt0 + kTilesPerChunk, ntn);
+                for (int nt = nt0; ok && nt < nt1; ++nt, ++lt) {
+                    const int buf = lt & 1;
+                    const uint32_t use = (uint32_t)lt >> 1;
+                    if (use > 0 && !wait_phase(&sb->acc_empty[buf], (use - 1) & 1u, sb, status)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a = smem_u32(dsm + s * kStageBytes), b = a + kABytes;
+                    const uint32_t d = tmem + (uint32_t)(buf * BN);
+                    for (int kb = 0; kb < nk; ++kb) {
+                        const int s = (int)(it % kStages);
+                        if (!wait_phase(&sb->full[s], (it / kStages) & 1u, sb, status)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a = smem_u32(dsm + s * kStageBytes), b = a + kABytes;
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k)
-                        mma_bf16(d, sdesc_sw128(a + 32u * k), sdesc_sw128(b + 32u * k),
-                                 (kb | k) != 0 ? 1u : 0u);
-                    mma_commit(&sb->empty[s]);  // frees the stage once these MMAs are done
-                    ++it;
+                        for (int k = 0; k < BK / 16; ++k)
+                            mma_bf16(d, sdesc_sw128(a + 32u * k), sdesc_sw128(b + 32u * k),
+                                     (kb | k) != 0 ? 1u : 0u);
+                        mma_commit(&sb->empty[s]);  // frees the stage once these MMAs are done
+                        ++it;
+                    }
+                    if (!ok) break;
+                    mma_commit(&sb->acc_full[buf]);
                 }
-                if (!ok) break;
-                mma_commit(&sb->acc_full[buf]);
             }
             // every MMA this thread issued is complete once this arrives
             mma_commit(&sb->drain);
@@ -276,34 +306,69 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------ epilogue
         const int q = warp & 3;  // this warp may access TMEM lanes 32q .. 32q + 31
         int lt = 0;
-        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++lt) {
-            const int buf = lt & 1;
-            const uint32_t use = (uint32_t)lt >> 1;
-            if (!wait_phase(&sb->acc_full[buf], use & 1u, sb, status)) break;
-            tc_fence_after();
-            const int m0 = (t % mt) * BM, n0 = (t / mt) * BN;
+        bool ok = true;
+        for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
+            const int m0 = (u % mt) * BM, ch = u / mt;
+            const int nt0 = ch * kTilesPerChunk, nt1 = min(nt0 + kTilesPerChunk, ntn);
             const int row = m0 + 32 * q + lane;
-            const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN);
-#pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                uint32_t r[32];
-                tmem_ld32(taddr + 32u * c, r);
-                const int col = n0 + 32 * c;
-                if (row < M && col < N) {
-                    __nv_bfloat16* o = out + (size_t)row * N + col;
-#pragma unroll
-                    for (int v = 0; v < 4; ++v)
-                        if (col + 8 * v < N)
-                            *reinterpret_cast<uint4*>(o + 8 * v) =
-                                make_uint4(pack_bf16(r[8 * v + 0], r[8 * v + 1]),
-                                           pack_bf16(r[8 * v + 2], r[8 * v + 3]),
-                                           pack_bf16(r[8 * v + 4], r[8 * v + 5]),
-                                           pack_bf16(r[8 * v + 6], r[8 * v + 7]));
+            float rm = -INFINITY, rs = 0.f;  // the row's running chunk statistics
+            for (int nt = nt0; nt < nt1; ++nt, ++lt) {
+                const int buf = lt & 1;
+                const uint32_t use = (uint32_t)lt >> 1;
+                if (!wait_phase(&sb->acc_full[buf], use & 1u, sb, status)) {
+                    ok = false;
+                    break;
                 }
+                tc_fence_after();
+                const int n0 = nt * BN;
+                const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN);
+#pragma unroll 1
+                for (int c = 0; c < BN / 32; ++c) {
+                    uint32_t r[32];
+                    tmem_ld32(taddr + 32u * c, r);
+                    const int col = n0 + 32 * c;
+                    if (row < M && col < N) {
+                        __nv_bfloat16* o = out + (size_t)row * N + col;
+                        uint32_t w[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) w[i] = pack_bf16(r[2 * i], r[2 * i + 1]);
+#pragma unroll
+                        for (int v = 0; v < 4; ++v)
+                            if (col + 8 * v < N)
+                                *reinterpret_cast<uint4*>(o + 8 * v) =
+                                    make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+                        if (cs.tab) {
+                            // the rounded logits of the group, then the running
+                            // (max, sum) rescaled to the new maximum
+                            float f[32];
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                f[2 * i] = __uint_as_float(w[i] << 16);
+                                f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+                            }
+                            float gm = -INFINITY;
+#pragma unroll
+                            for (int i = 0; i < 32; ++i)
+                                if (col + i < N) gm = fmaxf(gm, f[i]);
+                            const float nm = fmaxf(rm, gm);
+                            if (nm > -INFINITY) {
+                                float acc = rs * vsd::ex2((rm - nm) * cs.c);
+#pragma unroll
+                                for (int i = 0; i < 32; ++i)
+                                    if (col + i < N) acc += vsd::ex2((f[i] - nm) * cs.c);
+                                rs = acc;
+                                rm = nm;
+                            }
+                        }
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sb->acc_empty[buf]);
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sb->acc_empty[buf]);
+            if (ok && cs.tab && row < M)
+                reinterpret_cast<float2*>(cs.tab + (size_t)row * cs.stride + ch)[0] =
+                    make_float2(rm, rs);
         }
     }
     tc_fence_before();
@@ -367,7 +432,8 @@ bool lmhead_shape_ok(const void* hidden, const void* weight, const void* logits,
 }
 
 cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, int K, void* logits,
-                        int* status, uint64_t timeout_ns, cudaStream_t s) {
+                        int* status, uint64_t timeout_ns, cudaStream_t s, float4* chunk_tab,
+                        int chunk_stride, float chunk_c) {
     using vsd_lm::k_lmhead;
     using vsd_lm::make_map;
     CUtensorMap ta, tb;
@@ -389,16 +455,18 @@ cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, in
             done[dev] = true;
         }
     }
-    const long long ntiles =
-        (long long)((M + vsd_lm::BM - 1) / vsd_lm::BM) * ((N + vsd_lm::BN - 1) / vsd_lm::BN);
+    const long long ntn = (N + vsd_lm::BN - 1) / vsd_lm::BN;
+    const long long nunits = (long long)((M + vsd_lm::BM - 1) / vsd_lm::BM) *
+                             ((ntn + vsd_lm::kTilesPerChunk - 1) / vsd_lm::kTilesPerChunk);
 #ifndef VSD_LM_CTAS_PER_SM
 #define VSD_LM_CTAS_PER_SM 1
 #endif
     const long long slots = (long long)sms * VSD_LM_CTAS_PER_SM;
-    const int grid = (int)(ntiles < slots ? ntiles : slots);
+    const int grid = (int)(nunits < slots ? nunits : slots);
+    const vsd_lm::ChunkStatsOut cs{chunk_tab, chunk_stride, chunk_c};
     // (qualified: the enclosing namespace has a kThreads of its own)
     k_lmhead<<<grid, vsd_lm::kThreads, vsd_lm::kSmemBytes, s>>>(
-        ta, tb, static_cast<__nv_bfloat16*>(logits), M, N, K, status, timeout_ns);
+        ta, tb, static_cast<__nv_bfloat16*>(logits), M, N, K, status, timeout_ns, cs);
     return cudaGetLastError();
 }
 

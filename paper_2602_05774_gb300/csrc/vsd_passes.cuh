@@ -154,6 +154,8 @@ struct Problem {
     int* row_seg_cnt;             // [R] segments of a row completed
     int* res_seg_cnt;             // [B*K] residual segments of a path completed
     int stream_tails;             // fused kernel: the streaming warps run the row tails
+    int xtab_given;               // fused kernel: gtab[r][ch].xy (the draft's chunk
+                                  // statistics) were written by the LM head's epilogue
     int* path_A;                  // [B*K] accepted length of a path
     int* tlist;                   // tree layout: [R] residual rows of each tree (its rows' slots)
     int* tcount;                  // tree layout: [B] length of each tree's list
@@ -371,6 +373,21 @@ __device__ __forceinline__ void stream_tables(Ring* rg, const T* x, const T* y, 
         }
         ch = cn;
     }
+}
+
+// The target half of a row's chunk table when the draft half is given (the LM
+// head's epilogue wrote it): tab[ch].zw = (max, sum) of target chunk ch, for
+// ch in [ch0, ch1), one streaming read of the target row through the ring.
+template <typename T>
+__device__ __forceinline__ void stream_target_tables(Ring* rg, const T* y, int64_t V, int ch0,
+                                                     int ch1, float4* tab, float c, uint64_t pol,
+                                                     int* status) {
+    const int lane = threadIdx.x & 31;
+    ring_stream<T, false>(rg, y, nullptr, V, ch0, ch1, pol, pol, status,
+                          [&](int ch, const uint4 (&by)[kLoads], const uint4 (&)[kLoads]) {
+                              const float2 sy = chunk_stats<T>(by, c);
+                              if (lane == 0) reinterpret_cast<float2*>(tab + ch)[1] = sy;
+                          });
 }
 
 __device__ __forceinline__ float2 tab_ms(const float4& t, int comp) {
