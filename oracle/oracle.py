@@ -74,6 +74,9 @@ def _bind(path):
     lib_.vso_topk_ce.argtypes = [C.c_void_p, C.c_void_p, C.c_int64, C.c_double, C.c_int,
                                  C.c_void_p, C.c_void_p]
     lib_.vso_topk_ce.restype = C.c_double
+    lib_.vso_reference_logkappa.argtypes = [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32,
+                                            C.c_int64, C.c_double, C.c_void_p]
+    lib_.vso_reference_logkappa.restype = C.c_int
     return lib_
 
 
@@ -136,6 +139,7 @@ def linear(draft, target, T, u_draft, u_accept, u_correct, K, D, ref_logkappa=No
     """E-step + M-step over linear paths (Algorithm 1, Algorithm 2, Eqs. 1, 2, 11,
     beta, zeta, advance); with kl_weight != 0 the VSD (KL) variant adds
     kl_weight times the prefix's top-kl_topk term of Eq. klv (reading R11).
+    T = 0 is greedy decoding (reading R12).
 
     draft, target: [B*K*D, V] (any float dtype; widened to f32 exactly).
     Returns a dict of numpy arrays named as the C-ABI outputs.
@@ -193,6 +197,21 @@ def tree(draft, target, T, parent, tokens, u_accept, u_correct):
     if rc != 0:
         raise ValueError("oracle rejected the tree (code %d)" % rc)
     return o
+
+
+def reference_logkappa(ref_draft, ref_target, T, B, D):
+    """log kappa of supplied greedy reference paths (Algorithm 2, reading R13):
+    rows [B*D, V] along z-bar; returns [B, D] prefix sums of log min(1, p/q)
+    at each row's target argmax (T = 0: the greedy limits)."""
+    xq = _f32(ref_draft)
+    xp = _f32(ref_target)
+    V = xq.shape[-1]
+    assert xq.size == B * D * V and xp.shape == xq.shape
+    out = np.zeros((B, D))
+    rc = lib().vso_reference_logkappa(_ptr(xq), _ptr(xp), B, D, V, float(T), _ptr(out))
+    if rc != 0:
+        raise ValueError("oracle rejected the arguments (code %d)" % rc)
+    return out
 
 
 def topk_ce(draft_row, target_row, T=1.0, k=10):

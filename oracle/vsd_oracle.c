@@ -48,6 +48,17 @@
  *       loss_b = -J_b/N_b + kl_weight L_KL.  The paper gives no weight;
  *       kl_weight = 0 is VSD without the term.  The rows' contexts are held
  *       fixed in the gradient (as in R8).
+ *   R12 T = 0 (greedy decoding, the T in {0, 1} of the paper's tables): every
+ *       decision takes the T -> 0 limit of Eq. 1's distributions, q and p
+ *       one-hot at their argmax (lowest index on ties): z~ = argmax q,
+ *       alpha = [argmax p = z~], the residual and the later samples are
+ *       argmax p.  The M-step's log-likelihood (Eq. advance), zeta and the
+ *       top-K term use the draft's distribution at temperature 1, since log q
+ *       at T = 0 is not finite.
+ *   R13 A greedy reference path supplied as rows (Algorithm 2's z-bar drawn
+ *       from the greedy target policy, with the draft and target rows along
+ *       it): log k(z-bar_{<=l}) = sum_{d<=l} log min(1, p_d(v_d)/q_d(v_d)),
+ *       v_d = argmax p_d (vso_reference_logkappa).
  *   Tree (App. E verification): node n's token was drafted from the row of
  *   parent(n); alpha_n uses that row; A_n = a_n AND A_parent(n); a rejected node
  *   whose parent is accepted gets a residual token drawn at the parent's row.
@@ -94,6 +105,28 @@ static int64_t sample_inverse_cdf(const double* prob, int64_t V, double u, doubl
         if (prob[v] > 0.0) { *margin = 0.0; return v; }
     *margin = 0.0;
     return 0;
+}
+
+/* The T -> 0 limit of softmax(x / T) (R12): one-hot at the first maximum. */
+static int64_t greedy_one_hot(const float* x, int64_t V, double* prob)
+{
+    int64_t m = 0;
+    for (int64_t v = 1; v < V; ++v) if (x[v] > x[m]) m = v;
+    for (int64_t v = 0; v < V; ++v) prob[v] = v == m ? 1.0 : 0.0;
+    return m;
+}
+
+/* The distributions of one row that the decisions use: exp of the
+ * log-probabilities at T > 0, the one-hot limits at T = 0 (R12). */
+static void decision_dists(const float* xq, const float* xp, int64_t V, int greedy,
+                           const double* lq, const double* lp, double* q, double* p)
+{
+    if (greedy) {
+        greedy_one_hot(xq, V, q);
+        greedy_one_hot(xp, V, p);
+    } else {
+        for (int64_t v = 0; v < V; ++v) { q[v] = exp(lq[v]); p[v] = exp(lp[v]); }
+    }
 }
 
 /* ------------------------------------------------------------------ */
@@ -354,8 +387,10 @@ int vso_linear(const vso_linear_in* in, vso_linear_out* out)
 {
     const int B = in->B, K = in->K, D = in->D;
     const int64_t V = in->V;
-    const double T = in->T;
-    if (B < 1 || K < 1 || D < 1 || V < 1 || !(T > 0.0)) return 1;
+    if (B < 1 || K < 1 || D < 1 || V < 1 || !(in->T >= 0.0) || in->T == INFINITY) return 1;
+    /* R12: T = 0 decides greedily; log q is then taken at temperature 1 */
+    const int greedy = in->T == 0.0;
+    const double T = greedy ? 1.0 : in->T;
     double* lq = (double*)malloc(sizeof(double) * (size_t)V);
     double* lp = (double*)malloc(sizeof(double) * (size_t)V);
     double* q = (double*)malloc(sizeof(double) * (size_t)V);
@@ -387,7 +422,7 @@ int vso_linear(const vso_linear_in* in, vso_linear_out* out)
                 double lse_p = log_softmax_row(xp, V, T, lp);
                 out->row_lse[2 * r + 0] = lse_q;
                 out->row_lse[2 * r + 1] = lse_p;
-                for (int64_t v = 0; v < V; ++v) { q[v] = exp(lq[v]); p[v] = exp(lp[v]); }
+                decision_dists(xq, xp, V, greedy, lq, lp, q, p);
                 double mg;
                 int64_t zt = sample_inverse_cdf(q, V, (double)in->u_draft[r], &mg);
                 double alpha = p[zt] / q[zt];
@@ -436,7 +471,7 @@ int vso_linear(const vso_linear_in* in, vso_linear_out* out)
                 double mg = INFINITY;
                 log_softmax_row(in->draft + r * V, V, T, lq);
                 log_softmax_row(in->target + r * V, V, T, lp);
-                for (int64_t v = 0; v < V; ++v) { q[v] = exp(lq[v]); p[v] = exp(lp[v]); }
+                decision_dists(in->draft + r * V, in->target + r * V, V, greedy, lq, lp, q, p);
                 if (d < A) {
                     zc = out->tokens[r];
                 } else if (d == A) {
@@ -645,6 +680,41 @@ int vso_tree(const vso_tree_in* in, vso_tree_out* out)
     }
     free(lq); free(lp); free(q); free(p); free(res); free(depth);
     return rc;
+}
+
+/* ------------------------------------------------------------------ */
+/* R13: log kappa of a supplied greedy reference path (Algorithm 2).  Rows
+ * [B][D][V] of the draft and target along z-bar; out [B][D] receives
+ * sum_{d<=l} log min(1, p_d(v_d) / q_d(v_d)), v_d = argmax p_d (lowest index
+ * on ties), at temperature T (T = 0: the one-hot limits, R12). */
+int vso_reference_logkappa(const float* draft, const float* target, int32_t B, int32_t D,
+                           int64_t V, double T, double* out)
+{
+    if (B < 1 || D < 1 || V < 1 || !(T >= 0.0) || T == INFINITY) return 1;
+    const int greedy = T == 0.0;
+    double* lq = (double*)malloc(sizeof(double) * (size_t)V);
+    double* lp = (double*)malloc(sizeof(double) * (size_t)V);
+    double* q = (double*)malloc(sizeof(double) * (size_t)V);
+    double* p = (double*)malloc(sizeof(double) * (size_t)V);
+    for (int b = 0; b < B; ++b) {
+        double acc = 0.0;
+        for (int d = 0; d < D; ++d) {
+            const size_t r = (size_t)b * D + d;
+            const float* xq = draft + r * V;
+            const float* xp = target + r * V;
+            log_softmax_row(xq, V, greedy ? 1.0 : T, lq);
+            log_softmax_row(xp, V, greedy ? 1.0 : T, lp);
+            decision_dists(xq, xp, V, greedy, lq, lp, q, p);
+            int64_t vb = 0;
+            for (int64_t v = 1; v < V; ++v) if (xp[v] > xp[vb]) vb = v;
+            double ab = p[vb] / q[vb];
+            if (ab > 1.0) ab = 1.0;
+            acc += log(ab);
+            out[r] = acc;
+        }
+    }
+    free(lq); free(lp); free(q); free(p);
+    return 0;
 }
 
 /* ------------------------------------------------------------------ */

@@ -43,8 +43,12 @@ MUTATIONS = [
      "op[s] = oracle_utility(logkappa_corr[s * D + d], lkr, l, w_base);", "op[s] = 0.0;"),
     ("o' of a kept proposal is binary", "                op[s] = o_tilde; /* z = z~, o' = o(z~) */",
      "                op[s] = 1.0;"),
-    ("greedy reference ties to the highest index", "if (xp[v] > xp[vb]) vb = v;",
-     "if (xp[v] >= xp[vb]) vb = v;"),
+    ("greedy reference ties to the highest index",
+     "                for (int64_t v = 1; v < V; ++v) if (xp[v] > xp[vb]) vb = v;",
+     "                for (int64_t v = 1; v < V; ++v) if (xp[v] >= xp[vb]) vb = v;"),
+    ("supplied reference ties to the highest index",
+     "            for (int64_t v = 1; v < V; ++v) if (xp[v] > xp[vb]) vb = v;",
+     "            for (int64_t v = 1; v < V; ++v) if (xp[v] >= xp[vb]) vb = v;"),
     ("expected length skips S_1", "for (int d = 0; d < D; ++d) EA += exp(lk[s * D + d]);",
      "for (int d = 1; d < D; ++d) EA += exp(lk[s * D + d]);"),
     ("after the first rejection draws from q",
@@ -73,6 +77,14 @@ MUTATIONS = [
      "lb += in->kl_weight * kl;"),
     ("top-K gradient scale", "in->kl_weight / ((double)B * K) * dl[k];",
      "in->kl_weight / (double)B * dl[k];"),
+    ("greedy ties to the last maximum", "for (int64_t v = 1; v < V; ++v) if (x[v] > x[m]) m = v;",
+     "for (int64_t v = 1; v < V; ++v) if (x[v] >= x[m]) m = v;"),
+    ("greedy M-step at another temperature", "const double T = greedy ? 1.0 : in->T;",
+     "const double T = greedy ? 0.5 : in->T;"),
+    ("greedy decisions from the softmax", "    if (greedy) {\n        greedy_one_hot(xq, V, q);",
+     "    if (0) {\n        greedy_one_hot(xq, V, q);"),
+    ("supplied reference ratio inverted", "            double ab = p[vb] / q[vb];\n            if (ab > 1.0) ab = 1.0;\n            acc += log(ab);",
+     "            double ab = q[vb] / p[vb];\n            if (ab > 1.0) ab = 1.0;\n            acc += log(ab);"),
     ("margin: unequal sums given no margin", "if (a != b) return fabs(a - b);",
      "if (a != b) return 0.0;"),
     ("margin: a clipped tie given no margin", "        if (ra[i] < m) m = ra[i];\n", ""),

@@ -698,3 +698,121 @@ def test_kl_term_enters_loss_and_gradient(oracle):
     assert np.allclose(o1["loss"][:B], o0["loss"][:B] + add, rtol=1e-12, atol=1e-12)
     assert abs(o1["loss"][B] - o1["loss"][:B].mean()) < 1e-12
     assert np.allclose(o1["grad"], o0["grad"] + dg, rtol=1e-10, atol=1e-15)
+
+
+# --------------------------------------------------------------------------
+# Greedy decoding, T = 0 (reading R12), and a supplied greedy reference path
+# (reading R13).
+
+
+def _separated_problem(B, K, D, V, seed):
+    """Rows whose logits are distinct integers (a permutation of 0..V-1 per
+    row), so that at T = 0.01 every non-maximal token has probability below
+    e^-100 and the T -> 0 limit is reached in double precision."""
+    rng = np.random.default_rng(seed)
+    R = B * K * D
+    draft = np.stack([rng.permutation(V) for _ in range(R)]).astype(np.float32)
+    target = np.stack([rng.permutation(V) for _ in range(R)]).astype(np.float32)
+    # make about half the rows agree on the argmax
+    agree = rng.random(R) < 0.5
+    for r in np.nonzero(agree)[0]:
+        i, j = int(np.argmax(draft[r])), int(np.argmax(target[r]))
+        target[r, [i, j]] = target[r, [j, i]]
+    u = [rng.uniform(0.01, 0.99, R).astype(np.float32) for _ in range(3)]
+    return draft, target, u
+
+
+def test_greedy_is_the_small_temperature_limit(oracle):
+    B, K, D, V = 3, 4, 4, 40
+    draft, target, (ud, ua, uc) = _separated_problem(B, K, D, V, 31)
+    g = oracle.linear(draft, target, 0.0, ud, ua, uc, K, D)
+    s = oracle.linear(draft, target, 0.01, ud, ua, uc, K, D)
+    for n in ("tokens", "accept", "accept_len", "corr_tokens", "ref_tokens"):
+        assert np.array_equal(g[n], s[n]), n
+    assert np.array_equal(g["weights"][..., :2], s["weights"][..., :2])
+
+
+def test_greedy_decisions_closed_form(oracle):
+    B, K, D, V = 2, 3, 5, 30
+    draft, target, (ud, ua, uc) = _separated_problem(B, K, D, V, 32)
+    o = oracle.linear(draft, target, 0.0, ud, ua, uc, K, D)
+    am_q = np.argmax(draft, axis=1)   # numpy keeps the first maximum
+    am_p = np.argmax(target, axis=1)
+    assert np.array_equal(o["tokens"], am_q)
+    assert np.array_equal(o["accept"], (am_q == am_p).astype(np.uint8))
+    acc = (am_q == am_p).reshape(B * K, D)
+    A = np.where(acc.all(1), D, np.argmin(acc, axis=1))
+    assert np.array_equal(o["accept_len"], A)
+    d = np.arange(D)[None, :]
+    corr = np.where(d < A[:, None], am_q.reshape(B * K, D), am_p.reshape(B * K, D))
+    assert np.array_equal(o["corr_tokens"].reshape(B * K, D), corr)
+    assert np.all(o["logkappa_corr"] == 0.0) and np.all(o["logkappa_ref"] == 0.0)
+    w = o["weights"]  # [B][D][K][4]
+    Al = A.reshape(B, K)
+    for l in range(1, D + 1):
+        assert np.array_equal(w[:, l - 1, :, 0], (l <= Al).astype(float))
+        assert np.allclose(w[:, l - 1, :, 1], 1.05 ** l)
+
+
+def test_greedy_ties_take_the_lowest_index(oracle):
+    # two equal draft maxima (tokens 1 and 2) and two equal target maxima
+    # (tokens 2 and 3): z~ = 1, argmax p = 2, so the token is rejected and the
+    # corrected token is 2
+    xq = np.array([[0.0, 3.0, 3.0, -1.0]], np.float32)
+    xp = np.array([[0.0, 1.0, 2.0, 2.0]], np.float32)
+    o = oracle.linear(xq, xp, 0.0, [0.5], [0.5], [0.5], K=1, D=1)
+    assert o["tokens"][0] == 1 and o["accept"][0] == 0 and o["corr_tokens"][0] == 2
+    assert o["ref_tokens"][0] == 2
+    # supplied reference: target maxima at 0 and 1; the draft is confident on
+    # 0 (ratio below 1) and not on 1 (ratio above 1), so the tie decides
+    rq = np.array([[3.0, 0.0, 0.0, 0.0]], np.float32)
+    rp = np.array([[2.0, 2.0, 1.0, 0.0]], np.float32)
+    ref = oracle.reference_logkappa(rq, rp, 1.0, 1, 1)
+    lq, lp = oracle.log_softmax(rq[0], 1.0), oracle.log_softmax(rp[0], 1.0)
+    assert lp[0] - lq[0] < 0 and lp[1] - lq[1] > 0
+    assert abs(ref[0, 0] - (lp[0] - lq[0])) < 1e-12
+
+
+@pytest.mark.parametrize("accept", [True, False])
+def test_greedy_single_proposal_is_cross_entropy_at_temperature_one(oracle, accept):
+    import torch
+    V = 12
+    rng = np.random.default_rng(33)
+    xq = rng.permutation(V).astype(np.float32) * 0.5
+    xp = rng.permutation(V).astype(np.float32)
+    i, j = int(np.argmax(xq)), int(np.argmax(xp))
+    if accept:
+        xp[[i, j]] = xp[[j, i]]
+    o = oracle.linear(xq[None], xp[None], 0.0, [0.5], [0.5], [0.5], K=1, D=1)
+    z = i if accept else int(np.argmax(xp))
+    assert o["corr_tokens"][0] == z and o["accept"][0] == int(accept)
+    x = torch.tensor(xq.astype(np.float64), requires_grad=True)
+    ce = torch.nn.functional.cross_entropy(x[None], torch.tensor([z]))
+    ce.backward()
+    assert abs(o["loss"][0] - float(ce.detach())) < 1e-12
+    assert np.allclose(o["grad"][0], x.grad.numpy(), atol=1e-15)
+
+
+@pytest.mark.parametrize("T", [1.0, 0.7, 0.0])
+def test_reference_rows_equal_the_per_path_reference(oracle, T):
+    """With the reference rows equal to a path's own rows, log k(z-bar) of the
+    supplied rows is the per-path reference (R4) the oracle forms."""
+    from paper_2602_05774_gb300 import inputs
+    B, D, V = 3, 4, 64
+    p = inputs.linear_problem(B, 1, D, V, "f32", "gauss", seed=34)
+    f = {k: p[k].numpy() for k in ("draft", "target", "u_draft", "u_accept", "u_correct")}
+    o = oracle.linear(f["draft"], f["target"], T, f["u_draft"], f["u_accept"], f["u_correct"],
+                      1, D, want_grad=False)
+    ref = oracle.reference_logkappa(f["draft"], f["target"], T, B, D)
+    assert np.array_equal(ref.reshape(-1), o["logkappa_ref"])
+    if T == 0.0:
+        assert np.all(ref == 0.0)
+
+
+def test_reference_rows_worked_example(oracle):
+    q1, p1 = [1 / 2, 1 / 4, 1 / 8, 1 / 8], [1 / 8, 1 / 2, 1 / 4, 1 / 8]      # v = 1, ratio 2
+    q2, p2 = [1 / 8, 1 / 2, 1 / 4, 1 / 8], [1 / 4, 3 / 8, 1 / 4, 1 / 8]      # v = 1, ratio 3/4
+    draft = np.stack([logits(q1), logits(q2)])
+    target = np.stack([logits(p1), logits(p2)])
+    ref = oracle.reference_logkappa(draft, target, 1.0, 1, 2)
+    assert abs(ref[0, 0]) < 1e-7 and abs(ref[0, 1] - math.log(0.75)) < 1e-7
