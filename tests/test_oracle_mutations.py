@@ -47,8 +47,8 @@ MUTATIONS = [
      "                for (int64_t v = 1; v < V; ++v) if (xp[v] > xp[vb]) vb = v;",
      "                for (int64_t v = 1; v < V; ++v) if (xp[v] >= xp[vb]) vb = v;"),
     ("supplied reference ties to the highest index",
-     "            for (int64_t v = 1; v < V; ++v) if (xp[v] > xp[vb]) vb = v;",
-     "            for (int64_t v = 1; v < V; ++v) if (xp[v] >= xp[vb]) vb = v;"),
+     "            int64_t vb = 0;\n            for (int64_t v = 1; v < V; ++v) if (xp[v] > xp[vb])",
+     "            int64_t vb = 0;\n            for (int64_t v = 1; v < V; ++v) if (xp[v] >= xp[vb])"),
     ("expected length skips S_1", "for (int d = 0; d < D; ++d) EA += exp(lk[s * D + d]);",
      "for (int d = 1; d < D; ++d) EA += exp(lk[s * D + d]);"),
     ("after the first rejection draws from q",
