@@ -37,6 +37,14 @@
  *     identical results.
  *   - Limits: 1 <= V <= 1048576, 1 <= D <= 64, 1 <= K <= 256, 1 <= N <= 1024,
  *     B*K*D (or B*N) <= 16777216, T finite and > 0.
+ *   - T = 0 (greedy decoding, the T in {0, 1} of the paper's evaluation) is
+ *     served by vsd_estep_mstep, vsd_estep_mstep_noalloc,
+ *     vsd_lmhead_estep_mstep and vsd_reference_logkappa: every decision takes
+ *     the argmax limit of Eq. 1's distributions (z~ = argmax q, accepted iff
+ *     it is argmax p, the correction is argmax p; lowest index on ties), and
+ *     the M-step's log q, its gradient, zeta and the top-K term use the
+ *     draft's distribution at temperature 1.  The other calls return
+ *     VSD_ERR_UNSUPPORTED for T = 0.
  */
 #ifndef VSD_H_
 #define VSD_H_
@@ -51,7 +59,7 @@ extern "C" {
 typedef enum {
     VSD_OK = 0,
     VSD_ERR_INVALID_ARG = 1, /* a size, pointer, dtype or parameter is invalid */
-    VSD_ERR_UNSUPPORTED = 2, /* a valid request this build does not serve (T = 0) */
+    VSD_ERR_UNSUPPORTED = 2, /* a valid request this call does not serve          */
     VSD_ERR_CUDA = 3,        /* a CUDA runtime call failed                        */
     VSD_ERR_TIMEOUT = 4,     /* a device-side wait gave up (vsd_device_status)    */
     VSD_ERR_WORKSPACE = 5,   /* workspace missing or smaller than required        */
@@ -268,6 +276,22 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
                                   const vsd_params* params, void* draft_logits,
                                   vsd_linear_outputs* out, void* ws, size_t ws_bytes,
                                   void* stream);
+
+/* The greedy reference of Algorithm 2 from its own rows: the oracle's z-bar
+ * is drawn from the greedy target policy, so its validity log kappa(z-bar)
+ * needs the draft and target distributions along z-bar, which the caller
+ * computes (teacher-forced on z-bar) and passes here.  Writes
+ * ref_logkappa[b][l-1] = sum_{d < l} log min(1, p_d(v_d) / q_d(v_d)) with v_d
+ * the target row's argmax (lowest index on ties; Eq. 2 on the greedy path),
+ * ready to pass as `ref_logkappa` to vsd_estep_mstep / vsd_verify_paths.
+ *   ref_draft, ref_target  device, [B][D][V] of `dtype`, the rows along z-bar;
+ *   ref_logkappa           device, [B][D] float, written;
+ *   T >= 0 (T = 0: the one-hot limits, so every entry is 0);
+ *   ws of vsd_workspace_bytes({B, 1, D, V}) bytes.
+ * Errors as for vsd_verify_paths. */
+vsd_status vsd_reference_logkappa(const void* ref_draft, const void* ref_target, vsd_dtype dtype,
+                                  int32_t B, int32_t D, int32_t V, float T, float* ref_logkappa,
+                                  void* ws, size_t ws_bytes, void* stream);
 
 /* Waits for `stream`, then reads and clears the device status word of `ws`
  * into *status_bits (host).  Returns VSD_ERR_TIMEOUT if the timeout bit is set,

@@ -124,8 +124,11 @@ bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 int num_sms() { return device_sm_count(); }
 
-vsd_status check_temperature(float T) {
-    if (T == 0.f) return VSD_ERR_UNSUPPORTED;  // greedy decoding is not served here
+// T = 0 (greedy decoding) is served by the fused E-step + M-step, the LM
+// head with it and the reference log kappa (greedy = true); the separate
+// sampling, verification and M-step calls take T > 0.
+vsd_status check_temperature(float T, bool greedy_ok = false) {
+    if (T == 0.f) return greedy_ok ? VSD_OK : VSD_ERR_UNSUPPORTED;
     if (!(T > 0.f) || !isfinite(T)) return VSD_ERR_INVALID_ARG;
     return VSD_OK;
 }
@@ -188,10 +191,14 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     P.V = L.V;
     P.R = (int)rows_of(L);
     P.nch = (int)((L.V + chunk_elems<T>() - 1) / chunk_elems<T>());
-    P.ts.c = (float)(kLog2e / (double)T_);
-    P.ts.T = T_;
-    P.ts.Td = (double)T_;
-    P.ts.invTd = 1.0 / (double)T_;
+    // T = 0: decisions by argmax, log q (and everything that uses it) at
+    // temperature 1
+    P.greedy = T_ == 0.f ? 1 : 0;
+    const float Tq = T_ == 0.f ? 1.f : T_;
+    P.ts.c = (float)(kLog2e / (double)Tq);
+    P.ts.T = Tq;
+    P.ts.Td = (double)Tq;
+    P.ts.invTd = 1.0 / (double)Tq;
     P.parent = L.parent;
     P.w_base = 1.05;
     P.tau_car = 0.2;
@@ -513,7 +520,7 @@ vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtyp
         !out->grad)
         return VSD_ERR_INVALID_ARG;
     if (dtype != VSD_F32 && dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
-    vsd_status st = check_temperature(T);
+    vsd_status st = check_temperature(T, true);
     if (st) return st;
     const vsd_params p = params ? *params : default_params(dtype);
     if ((st = check_params(p))) return st;
@@ -552,7 +559,7 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
     const int64_t R = rows_of(layout);
     if (R > (1 << 30) || !lmhead_shape_ok(hidden, weight, draft_logits, (int)R, layout.V, H))
         return VSD_ERR_INVALID_ARG;
-    vsd_status st = check_temperature(T);
+    vsd_status st = check_temperature(T, true);
     if (st) return st;
     const vsd_params p = params ? *params : default_params(VSD_BF16);
     if ((st = check_params(p))) return st;
@@ -562,7 +569,7 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
     // the GEMM's epilogue writes the draft half of every row's chunk table
     // (a1 for the draft), so the E-step streams only the target rows
     const WsLayout w = ws_layout(layout);
-    const float c = (float)(kLog2e / (double)T);
+    const float c = (float)(kLog2e / (double)(T == 0.f ? 1.f : T));  // as make_problem's
     cudaError_t e = clear_counters(ws, layout, s);
     if (e == cudaSuccess)
         e = lmhead_gemm(hidden, weight, (int)R, layout.V, H, draft_logits, static_cast<int*>(ws),
@@ -571,6 +578,31 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
     if (e != cudaSuccess) return from_cuda(e);
     return fused_impl<__nv_bfloat16>(draft_logits, target, layout, T, u_draft, u_accept,
                                      u_correct, ref_logkappa, p, out, ws, s, false, true);
+}
+
+vsd_status vsd_reference_logkappa(const void* ref_draft, const void* ref_target, vsd_dtype dtype,
+                                  int32_t B, int32_t D, int32_t V, float T, float* ref_logkappa,
+                                  void* ws, size_t ws_bytes, void* stream) {
+    const vsd_layout L{B, 1, D, V, 0, nullptr};
+    if (!layout_ok(L)) return VSD_ERR_INVALID_ARG;
+    if (!ref_draft || !ref_target || !ref_logkappa) return VSD_ERR_INVALID_ARG;
+    if (dtype != VSD_F32 && dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
+    vsd_status st = check_temperature(T, true);
+    if (st) return st;
+    if ((st = check_ws(L, ws, ws_bytes))) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = clear_counters(ws, L, s);
+    if (e != cudaSuccess) return from_cuda(e);
+    if (dtype == VSD_F32) {
+        Problem<float> P = make_problem<float>(ref_draft, ref_target, L, T, ws);
+        e = Launch<float>::reference(P, vec_ok(ref_draft, ref_target, nullptr, V, 4, 0),
+                                     ref_logkappa, s);
+    } else {
+        Problem<__nv_bfloat16> P = make_problem<__nv_bfloat16>(ref_draft, ref_target, L, T, ws);
+        e = Launch<__nv_bfloat16>::reference(P, vec_ok(ref_draft, ref_target, nullptr, V, 2, 0),
+                                             ref_logkappa, s);
+    }
+    return from_cuda(e);
 }
 
 vsd_status vsd_device_status(void* ws, void* stream, int32_t* status_bits) {

@@ -50,6 +50,37 @@ __global__ void __launch_bounds__(kThreads) k_rows_verify(Problem<T> P) {
     row_pass<T, VEC, true, kGivenToken, true>(P, blockIdx.x, rg, tab, sh);
 }
 
+// Rows along supplied greedy reference paths (Algorithm 2's z-bar): per row
+// the target's argmax and log min(1, p/q) there (row_pass with the argmax).
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kThreads) k_ref_rows(Problem<T> P) {
+    extern __shared__ __align__(128) unsigned char dsm[];
+    __shared__ RowShared sh;
+    Ring* rg;
+    float4* tab;
+    smem_views<VEC>(dsm, rg, tab, P.timeout_ns);
+    row_pass<T, VEC, true, kNoToken, true>(P, blockIdx.x, rg, tab, sh);
+}
+
+// log kappa(z-bar_{<=l}) of reference path b: the prefix sums over its rows
+// of log min(1, p/q) at the argmax (one warp per path, Eq. 2).
+template <typename T>
+__global__ void k_ref_scan(Problem<T> P, float* out) {
+    const int b = blockIdx.x, lane = threadIdx.x & 31;
+    double carry = 0.0;
+    for (int d0 = 0; d0 < P.D; d0 += 32) {
+        const int d = d0 + lane;
+        double la = 0.0;
+        if (d < P.D) {
+            const RowRec rec = P.rows[(int64_t)b * P.D + d];
+            la = (rec.flags || rec.ref < 0) ? -INFINITY : (double)rec.la_ref;
+        }
+        const double inc = carry + warp_incl_scan(la, lane);
+        if (d < P.D) out[(int64_t)b * P.D + d] = (float)inc;
+        carry = __shfl_sync(0xffffffffu, inc, 31);
+    }
+}
+
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads) k_paths(Problem<T> P) {
     extern __shared__ __align__(128) unsigned char dsm[];
@@ -307,7 +338,9 @@ __device__ void post_job(const Problem<T>& P, const EStepView& E, const Job& j, 
         if (!warp_count_last(P.path_cnt + path, D, lane)) return;
         const int A = path_accept_len<T>(P, path, lane);
         const int flags = A < D ? ld_cg(P.rows + path * D + A).flags : 0;
-        if (A < D && !flags) {
+        // T = 0: the residual is the target's argmax, the row's p-draw: no
+        // residual row to read
+        if (A < D && !flags && !P.greedy) {
             if (lane == 0) {  // queue the residual row's segments
                 P.path_A[path] = A;
                 publish_residuals(P.resq_tail, P.resq_avail, P.resq_flag, P.resq, path * nseg,
@@ -649,6 +682,20 @@ cudaError_t Launch<VSD_T>::rows_verify(const Problem<VSD_T>& P, bool vec, cudaSt
     cudaError_t e = prep(kern, smem);
     if (e) return e;
     kern<<<P.R, kThreads, smem, s>>>(P);
+    return cudaGetLastError();
+}
+
+template <>
+cudaError_t Launch<VSD_T>::reference(const Problem<VSD_T>& P, bool vec, float* out,
+                                     cudaStream_t s) {
+    const size_t smem = stream_smem_bytes(P.nch, vec);
+    auto kern = vec ? k_ref_rows<VSD_T, true> : k_ref_rows<VSD_T, false>;
+    cudaError_t e = prep(kern, smem);
+    if (e) return e;
+    kern<<<P.R, kThreads, smem, s>>>(P);
+    e = cudaGetLastError();
+    if (e) return e;
+    k_ref_scan<VSD_T><<<P.B, 32, 0, s>>>(P, out);
     return cudaGetLastError();
 }
 

@@ -13,6 +13,8 @@ template <typename T> struct Launch {
     static cudaError_t sample(const Problem<T>& P, bool vec, cudaStream_t s);
     // row statistics of draft+target with given tokens (linear paths)
     static cudaError_t rows_verify(const Problem<T>& P, bool vec, cudaStream_t s);
+    // log kappa of supplied greedy reference paths: [B][D] rows -> out [B][D]
+    static cudaError_t reference(const Problem<T>& P, bool vec, float* out, cudaStream_t s);
     // accepted lengths, residual draws, corrected paths, log-kappa (linear)
     static cudaError_t paths(const Problem<T>& P, bool vec, cudaStream_t s);
     // tree verification in one persistent launch: node rows, acceptance scan,

@@ -154,6 +154,9 @@ struct Problem {
     int* row_seg_cnt;             // [R] segments of a row completed
     int* res_seg_cnt;             // [B*K] residual segments of a path completed
     int stream_tails;             // fused kernel: the streaming warps run the row tails
+    int greedy;                   // T = 0: every decision takes the argmax limit of
+                                  // Eq. 1's distributions; ts holds temperature 1,
+                                  // the M-step's
     int xtab_given;               // fused kernel: gtab[r][ch].xy (the draft's chunk
                                   // statistics) were written by the LM head's epilogue
     int* path_A;                  // [B*K] accepted length of a path
@@ -667,10 +670,11 @@ __device__ __forceinline__ int warp_sample(const T* x, const T* y, int64_t V, co
 }
 
 // First chunk whose target maximum equals the row max M (warp; -1 if none).
-__device__ __forceinline__ int table_first_max(const float4* tab, int nch, float M) {
+__device__ __forceinline__ int table_first_max(const float4* tab, int nch, float M, int comp = 1) {
     for (int g = 0; g < nch; g += 32) {
         const int cc = g + (threadIdx.x & 31);
-        const unsigned hit = __ballot_sync(0xffffffffu, cc < nch && tab[cc].z == M);
+        const unsigned hit =
+            __ballot_sync(0xffffffffu, cc < nch && tab_ms(tab[cc], comp).x == M);
         if (hit) return g + __ffs(hit) - 1;
     }
     return -1;
@@ -704,8 +708,8 @@ __device__ __forceinline__ int first_max_regs(const uint4 (&by)[kLoads], int ch,
 // Lowest index whose target logit equals the row max M (warp).
 template <typename T, bool VEC>
 __device__ __forceinline__ int warp_first_max(const T* y, int64_t V, const float4* tab, int nch,
-                                              float M, int lane, uint64_t pol) {
-    const int ch = table_first_max(tab, nch, M);
+                                              float M, int lane, uint64_t pol, int comp = 1) {
+    const int ch = table_first_max(tab, nch, M, comp);
     if (ch < 0) return -1;
     uint4 by[kLoads];
     load_chunk<T, VEC>(y, V, ch, lane, pol, by);
@@ -765,16 +769,20 @@ __device__ __forceinline__ RowTask row_task(const Problem<T>& P, int r, const fl
     if (which == 0) {
         if (XMODE == kSampleToken) {
             if (row_ok(t.M, t.S.Z))
-                t.tok = warp_sample<T, VEC>(x, y, V, tab, P.nch, 0, t.M, t.S,
-                                            __ldg(P.u_draft + r), c, lane, pol);
+                t.tok = P.greedy ? warp_first_max<T, VEC>(x, V, tab, P.nch, t.M, lane, pol, 0)
+                                 : warp_sample<T, VEC>(x, y, V, tab, P.nch, 0, t.M, t.S,
+                                                       __ldg(P.u_draft + r), c, lane, pol);
             if (t.tok >= V) t.tok = -1;
         } else if (XMODE == kGivenToken) {
             t.tok = __ldg(P.given_tokens + r);
         }
     } else {
-        if (row_ok(t.M, t.S.Z))
-            t.tok = warp_sample<T, VEC>(x, y, V, tab, P.nch, 1, t.M, t.S, __ldg(P.u_correct + r),
-                                        c, lane, pol);
+        // (no uniforms for the p-draw: the reference rows of
+        // vsd_reference_logkappa need only the argmax)
+        if (row_ok(t.M, t.S.Z) && (P.greedy || P.u_correct))
+            t.tok = P.greedy ? warp_first_max<T, VEC>(y, V, tab, P.nch, t.M, lane, pol)
+                             : warp_sample<T, VEC>(x, y, V, tab, P.nch, 1, t.M, t.S,
+                                                   __ldg(P.u_correct + r), c, lane, pol);
         if (t.tok >= V) t.tok = -1;
     }
     return t;
@@ -817,6 +825,11 @@ __device__ __forceinline__ void row_finish(const Problem<T>& P, int r, const Row
             else
                 lq = (float)(((double)xv - (double)tmp.mx) * invT - tmp.lzx);
         }
+    }
+    if (P.greedy && lane < 3 && la > -INFINITY) {
+        // T = 0: alpha is 1 where the token is the target's argmax (the
+        // p-draw and the reference are), else 0 (one-hot limits)
+        la = (lane == 0 && tok != ref) ? -INFINITY : 0.f;
     }
     const float lq1 = __shfl_sync(0xffffffffu, lq, 1), la1 = __shfl_sync(0xffffffffu, la, 1);
     const float la2 = __shfl_sync(0xffffffffu, la, 2);
@@ -1136,9 +1149,14 @@ __device__ void row_tail_warp(const Problem<T>& P, int r, float4* tab, RescanBuf
     RowTask ty{table_max(tab, nch, 1, lane), TableSum{0, 0, 0.0}, -1};
     ty.S = table_sum(tab, nch, 1, frame_of(ty.M), c, lane);
     Located lx{-1, 0.f}, ly{-1, 0.f};
-    if (row_ok(tx.M, tx.S.Z)) lx = table_locate(tab, nch, 0, frame_of(tx.M), c, tx.S, ud, lane);
-    if (row_ok(ty.M, ty.S.Z)) ly = table_locate(tab, nch, 1, frame_of(ty.M), c, ty.S, uc, lane);
     const int ca = ty.M > -INFINITY ? table_first_max(tab, nch, ty.M) : -1;
+    if (P.greedy) {  // T = 0: the argmax of each row (first chunk holding its maximum)
+        if (row_ok(tx.M, tx.S.Z)) lx.ch = table_first_max(tab, nch, tx.M, 0);
+        if (row_ok(ty.M, ty.S.Z)) ly.ch = ca;
+    } else {
+        if (row_ok(tx.M, tx.S.Z)) lx = table_locate(tab, nch, 0, frame_of(tx.M), c, tx.S, ud, lane);
+        if (row_ok(ty.M, ty.S.Z)) ly = table_locate(tab, nch, 1, frame_of(ty.M), c, ty.S, uc, lane);
+    }
     const int chs[3] = {lx.ch, ly.ch, ca};
     if (VEC) {
 #pragma unroll
@@ -1156,14 +1174,16 @@ __device__ void row_tail_warp(const Problem<T>& P, int r, float4* tab, RescanBuf
         if (VEC) chunk_from_smem<T>(rb.c[0], V, lx.ch, lane, b);
         else load_chunk<T, VEC>(x, V, lx.ch, lane, pol, b);
         const float mm = frame_of(tab_ms(tab[lx.ch], 0).x);
-        tx.tok = rescan_regs<T, true, false>(b, b, lx.ch, lx.tc, MassX{mm, c}, lane);
+        tx.tok = P.greedy ? first_max_regs<T>(b, lx.ch, tx.M)
+                          : rescan_regs<T, true, false>(b, b, lx.ch, lx.tc, MassX{mm, c}, lane);
         if (tx.tok >= V) tx.tok = -1;
     }
     if (ly.ch >= 0) {
         if (VEC) chunk_from_smem<T>(rb.c[3], V, ly.ch, lane, b);
         else load_chunk<T, VEC>(y, V, ly.ch, lane, pol, b);
         const float mm = frame_of(tab_ms(tab[ly.ch], 1).x);
-        ty.tok = rescan_regs<T, false, true>(b, b, ly.ch, ly.tc, MassY{mm, c}, lane);
+        ty.tok = P.greedy ? first_max_regs<T>(b, ly.ch, ty.M)
+                          : rescan_regs<T, false, true>(b, b, ly.ch, ly.tc, MassY{mm, c}, lane);
         if (ty.tok >= V) ty.tok = -1;
     }
     int ref = -1;

@@ -23,7 +23,8 @@ _STATUS_NAMES = {0: "VSD_OK", 1: "VSD_ERR_INVALID_ARG", 2: "VSD_ERR_UNSUPPORTED"
 SYMBOLS = ("vsd_workspace_bytes", "vsd_sample_paths", "vsd_verify_paths",
            "vsd_weighted_loss_fwd_bwd", "vsd_estep_mstep", "vsd_device_status",
            "vsd_status_string", "vsd_version", "vsd_estep_mstep_noalloc",
-           "vsd_noalloc_device_status", "vsd_lmhead_logits", "vsd_lmhead_estep_mstep")
+           "vsd_noalloc_device_status", "vsd_lmhead_logits", "vsd_lmhead_estep_mstep",
+           "vsd_reference_logkappa")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -100,12 +101,14 @@ def _lib():
                                                C.POINTER(LinearOutputs), vp, C.c_size_t, vp]
         lib.vsd_device_status.argtypes = [vp, vp, C.POINTER(C.c_int32)]
         lib.vsd_noalloc_device_status.argtypes = [vp, C.POINTER(C.c_int32)]
+        lib.vsd_reference_logkappa.argtypes = [vp, vp, C.c_int, C.c_int32, C.c_int32, C.c_int32,
+                                               C.c_float, vp, vp, C.c_size_t, vp]
         lib.vsd_status_string.argtypes = [C.c_int]
         lib.vsd_status_string.restype = C.c_char_p
         lib.vsd_version.restype = C.c_char_p
         for name in ("vsd_sample_paths", "vsd_verify_paths", "vsd_weighted_loss_fwd_bwd",
                      "vsd_estep_mstep", "vsd_device_status", "vsd_estep_mstep_noalloc",
-                     "vsd_noalloc_device_status",
+                     "vsd_noalloc_device_status", "vsd_reference_logkappa",
                      "vsd_lmhead_logits", "vsd_lmhead_estep_mstep"):
             getattr(lib, name).restype = C.c_int
         _LIB = lib
@@ -339,6 +342,24 @@ def estep_mstep(draft, target, u_draft, u_accept, u_correct, K, D, T, ref_logkap
                                   _ptr(u_draft), _ptr(u_accept), _ptr(u_correct),
                                   _ptr(ref_logkappa), C.byref(prm), C.byref(st), _ptr(ws),
                                   ws.numel(), _stream(dev)), "vsd_estep_mstep")
+    return out
+
+
+def reference_logkappa(ref_draft, ref_target, B, D, T, workspace=None):
+    """log kappa of supplied greedy reference paths (Algorithm 2's z-bar with
+    its own rows [B*D, V]): [B, D] float32, to pass as ref_logkappa."""
+    _need_cuda(ref_draft, ref_target)
+    V = ref_draft.shape[-1]
+    if _rows(ref_draft, V) != B * D or ref_target.shape != ref_draft.shape:
+        raise ValueError("reference rows must be [B*D, V] for both tensors")
+    lay = layout(B, 1, D, V)
+    dev = ref_draft.device
+    ws = _ws(workspace, lay, dev)
+    out = torch.empty(B, D, dtype=torch.float32, device=dev)
+    _check(_lib().vsd_reference_logkappa(_ptr(ref_draft), _ptr(ref_target),
+                                         _dtype_code(ref_draft), int(B), int(D), int(V), float(T),
+                                         _ptr(out), _ptr(ws), ws.numel(), _stream(dev)),
+           "vsd_reference_logkappa")
     return out
 
 

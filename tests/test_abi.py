@@ -124,5 +124,33 @@ def test_lmhead_argument_checks_before_any_launch(vsd):
     tlay = vsd.Layout(2, 1, 1, 1024, 60, 0x1000)
     assert lib.vsd_lmhead_estep_mstep(fake, fake, 128, fake, tlay, 1.0, fake, fake, fake, None,
                                       None, fake, C.byref(o), ws, 1 << 30, None) == 1
-    assert lib.vsd_lmhead_estep_mstep(fake, fake, 128, fake, lay, 0.0, fake, fake, fake, None,
-                                      None, fake, C.byref(o), ws, 1 << 30, None) == 2
+    assert lib.vsd_lmhead_estep_mstep(fake, fake, 128, fake, lay, -1.0, fake, fake, fake, None,
+                                      None, fake, C.byref(o), ws, 1 << 30, None) == 1
+
+
+def test_kl_greedy_and_reference_argument_checks(vsd):
+    lib = vsd.load()
+    fake = C.c_void_p(0x1000)  # never dereferenced: every call below fails its checks
+    big = 1 << 30
+    lay = vsd.layout(2, 4, 4, 1024)
+    o = vsd.LinearOutputs(*([0x1000] * len(vsd.LINEAR_FIELDS)))
+    # the top-K term: a weight >= 0 and 1 <= K <= 16
+    for prm in (vsd.params(kl_weight=-1.0), vsd.params(kl_weight=1.0, kl_topk=0),
+                vsd.params(kl_weight=1.0, kl_topk=17), vsd.params(kl_weight=float("inf"))):
+        assert lib.vsd_estep_mstep(fake, fake, 1, lay, 1.0, fake, fake, fake, None, C.byref(prm),
+                                   C.byref(o), fake, big, None) == 1
+    # the separate M-step does not serve it, nor T = 0
+    prm = vsd.params(kl_weight=0.5)
+    assert lib.vsd_weighted_loss_fwd_bwd(fake, 1, lay, 1.0, C.byref(o), C.byref(prm), fake,
+                                         fake, None, fake, big, None) == 2
+    assert lib.vsd_weighted_loss_fwd_bwd(fake, 1, lay, 0.0, C.byref(o), None, fake, fake, None,
+                                         fake, big, None) == 2
+    # the reference from supplied rows: pointers, temperature, workspace
+    ref = lib.vsd_reference_logkappa
+    assert ref(None, fake, 1, 2, 4, 1024, 1.0, fake, fake, big, None) == 1
+    assert ref(fake, fake, 1, 2, 4, 1024, 1.0, None, fake, big, None) == 1
+    assert ref(fake, fake, 1, 2, 4, 1024, -0.5, fake, fake, big, None) == 1
+    assert ref(fake, fake, 1, 0, 4, 1024, 1.0, fake, fake, big, None) == 1
+    assert ref(fake, fake, 1, 2, 65, 1024, 1.0, fake, fake, big, None) == 1
+    assert ref(fake, fake, 1, 2, 4, 1024, 1.0, fake, None, big, None) == 5
+    assert ref(fake, fake, 1, 2, 4, 1024, 1.0, fake, fake, 16, None) == 5
