@@ -39,8 +39,24 @@ class _TreeIn(C.Structure):
         ("draft", C.c_void_p), ("target", C.c_void_p),
         ("B", C.c_int32), ("N", C.c_int32), ("V", C.c_int64), ("T", C.c_double),
         ("parent", C.c_void_p), ("tokens", C.c_void_p),
-        ("u_accept", C.c_void_p), ("u_correct", C.c_void_p),
+        ("u_accept", C.c_void_p), ("u_correct", C.c_void_p), ("rule", C.c_int32),
     ]
+
+
+class _TreeEmIn(C.Structure):
+    _fields_ = [
+        ("draft", C.c_void_p), ("target", C.c_void_p),
+        ("B", C.c_int32), ("N", C.c_int32), ("V", C.c_int64), ("T", C.c_double),
+        ("parent", C.c_void_p), ("tokens", C.c_void_p),
+        ("u_accept", C.c_void_p), ("u_correct", C.c_void_p),
+        ("w_base", C.c_double), ("tau_car", C.c_double), ("zeta_mode", C.c_int32),
+    ]
+
+
+class _TreeEmOut(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in (
+        "corr_tokens", "logq_tok", "logq_corr", "logkappa", "logkappa_corr", "logkappa_ref",
+        "weights", "loss", "grad", "margins")]
 
 
 class _TreeOut(C.Structure):
@@ -77,6 +93,8 @@ def _bind(path):
     lib_.vso_reference_logkappa.argtypes = [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32,
                                             C.c_int64, C.c_double, C.c_void_p]
     lib_.vso_reference_logkappa.restype = C.c_int
+    lib_.vso_tree_em.argtypes = [C.POINTER(_TreeEmIn), C.POINTER(_TreeEmOut)]
+    lib_.vso_tree_em.restype = C.c_int
     return lib_
 
 
@@ -174,9 +192,10 @@ def linear(draft, target, T, u_draft, u_accept, u_correct, K, D, ref_logkappa=No
     return o
 
 
-def tree(draft, target, T, parent, tokens, u_accept, u_correct):
+def tree(draft, target, T, parent, tokens, u_accept, u_correct, rule=0):
     """Verification of a draft tree with parent pointers (App. E tree, Eq. 1 per
-    node, Sec. 3 residual).  draft/target [B*N, V]; parent, tokens, uniforms [B, N]."""
+    node, Sec. 3 residual).  draft/target [B*N, V]; parent, tokens, uniforms [B, N].
+    rule 0: every branch verified alone; 1: sequential siblings (reading R14)."""
     draft = _f32(draft)
     target = _f32(target)
     parent = _i32(parent)
@@ -191,9 +210,36 @@ def tree(draft, target, T, parent, tokens, u_accept, u_correct):
              accept_len=np.zeros(B, np.int32), bonus=np.zeros(B, np.int32),
              margins=np.zeros((B, N, 2)))
     ti = _TreeIn(_ptr(draft), _ptr(target), B, N, V, float(T), _ptr(parent), _ptr(tokens),
-                 _ptr(ua), _ptr(uc))
+                 _ptr(ua), _ptr(uc), int(rule))
     to = _TreeOut(*[_ptr(o[n]) for n, _ in _TreeOut._fields_])
     rc = lib().vso_tree(C.byref(ti), C.byref(to))
+    if rc != 0:
+        raise ValueError("oracle rejected the tree (code %d)" % rc)
+    return o
+
+
+def tree_em(draft, target, T, parent, tokens, u_accept, u_correct, w_base=1.05, tau_car=0.2,
+            zeta_mode=0, want_grad=True):
+    """E-step + M-step over draft trees, every node a latent proposal (reading
+    R15; Algorithm 1 and 2, Eqs. 1, 2, beta, zeta, advance on the tree's root
+    paths).  draft/target [B*N, V]; parent, tokens, uniforms [B, N]."""
+    draft = _f32(draft)
+    target = _f32(target)
+    parent = _i32(parent)
+    B, N = parent.shape
+    V = draft.shape[-1]
+    assert draft.size == B * N * V and target.shape == draft.shape
+    tokens = _i32(tokens).reshape(B, N)
+    ua, uc = _f32(u_accept).reshape(B, N), _f32(u_correct).reshape(B, N)
+    o = dict(corr_tokens=np.zeros((B, N), np.int32), logq_tok=np.zeros((B, N)),
+             logq_corr=np.zeros((B, N)), logkappa=np.zeros((B, N)),
+             logkappa_corr=np.zeros((B, N)), logkappa_ref=np.zeros((B, N)),
+             weights=np.zeros((B, N, 4)), loss=np.zeros(B + 1),
+             grad=np.zeros((B * N, V)) if want_grad else None, margins=np.zeros((B, N, 3)))
+    ti = _TreeEmIn(_ptr(draft), _ptr(target), B, N, V, float(T), _ptr(parent), _ptr(tokens),
+                   _ptr(ua), _ptr(uc), float(w_base), float(tau_car), int(zeta_mode))
+    to = _TreeEmOut(*[_ptr(o[n]) for n, _ in _TreeEmOut._fields_])
+    rc = lib().vso_tree_em(C.byref(ti), C.byref(to))
     if rc != 0:
         raise ValueError("oracle rejected the tree (code %d)" % rc)
     return o

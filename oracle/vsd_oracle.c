@@ -55,6 +55,26 @@
  *       argmax p.  The M-step's log-likelihood (Eq. advance), zeta and the
  *       top-K term use the draft's distribution at temperature 1, since log q
  *       at T = 0 is not finite.
+ *   R14 Tree verification with the sequential sibling rule (lossless
+ *       multi-draft; App. E trees): at a node on the accepted path its
+ *       children are tried in node order; child i is accepted with
+ *       probability min(1, p_i(t_i)/q_i(t_i)), where p_1 = p, q_1 = q,
+ *       p_{i+1} = norm(max(0, p_i - q_i)) (p_i kept if that has no mass) and
+ *       q_{i+1} = q_i with t_i removed and renormalised (siblings are distinct
+ *       draws, as without replacement); the first accepted child continues
+ *       the path and later siblings are not tried; if every child is
+ *       rejected, the correction token is drawn from p_{m+1} with the last
+ *       child's uniform.  Output is distributed as p whenever t_i ~ q_i.
+ *   R15 Tree EM (App. E trees as latent proposals): every node n >= 1 is the
+ *       proposal z~(n) = the tokens on its root path, of length l = depth(n).
+ *       Each position x on a path is verified alone as in R3 (independent
+ *       rule, the path validity of Eq. 2): z'_x = t_x on an accepted path, the
+ *       residual at the first rejected node, p-draws below it (with each
+ *       node's own u_correct); the reference per row is R4's argmax.  o~, o'
+ *       as R5 with w(depth); beta and zeta are taken over the nodes of one
+ *       depth (the proposals of one length); loss and gradient as Eq.
+ *       advance, each node's row collecting the terms of every proposal
+ *       whose path goes through one of its children.
  *   R13 A greedy reference path supplied as rows (Algorithm 2's z-bar drawn
  *       from the greedy target policy, with the draft and target rows along
  *       it): log k(z-bar_{<=l}) = sum_{d<=l} log min(1, p_d(v_d)/q_d(v_d)),
@@ -580,6 +600,7 @@ typedef struct {
     const int32_t* tokens;     /* [B][N] token of node n (n >= 1)      */
     const float* u_accept;     /* [B][N] */
     const float* u_correct;    /* [B][N] */
+    int32_t rule;              /* 0: independent per branch; 1: sequential siblings (R14) */
 } vso_tree_in;
 
 typedef struct {
@@ -595,6 +616,116 @@ typedef struct {
     double*  margins;      /* optional [B][N][2]: accept, correction sample */
 } vso_tree_out;
 
+/* R14: the sequential sibling rule.  Scratch buffers of V (lq, lp, q, p,
+ * res) and N (depth) are the caller's. */
+static int tree_sequential(const vso_tree_in* in, vso_tree_out* out, double* lq, double* lp,
+                           double* q, double* p, double* res, int* depth)
+{
+    const int B = in->B, N = in->N;
+    const int64_t V = in->V;
+    const double T = in->T;
+    for (int b = 0; b < B; ++b) {
+        const int32_t* par = in->parent + (size_t)b * N;
+        const size_t n0 = (size_t)b * N;
+        if (par[0] != -1) return 2;
+        depth[0] = 0;
+        for (int n = 1; n < N; ++n) {
+            if (par[n] < 0 || par[n] >= n) return 2;
+            depth[n] = depth[par[n]] + 1;
+        }
+        for (int n = 0; n < N; ++n) {
+            out->alpha[n0 + n] = n ? 0.0 : 1.0;
+            out->accept[n0 + n] = n ? 0 : 1;
+            out->path_accept[n0 + n] = n ? 0 : 1;
+            out->corr_tokens[n0 + n] = -1;
+            if (out->margins) {
+                out->margins[2 * (n0 + n)] = INFINITY;
+                out->margins[2 * (n0 + n) + 1] = INFINITY;
+            }
+        }
+        /* log kappa: the path validity of Eq. 2, independent ratios along the path */
+        out->logkappa[n0] = 0.0;
+        for (int n = 1; n < N; ++n) {
+            const size_t rp = n0 + (size_t)par[n];
+            log_softmax_row(in->draft + rp * V, V, T, lq);
+            log_softmax_row(in->target + rp * V, V, T, lp);
+            const int32_t t = in->tokens[n0 + n];
+            double a = exp(lp[t]) / exp(lq[t]);
+            if (a > 1.0) a = 1.0;
+            out->logkappa[n0 + n] = out->logkappa[rp] + log(a);
+        }
+        /* the accepted path, node by node (parents come first) */
+        for (int u = 0; u < N; ++u) {
+            if (!out->path_accept[n0 + u]) continue;
+            int last = -1;
+            for (int n = u + 1; n < N; ++n) if (par[n] == u) last = n;
+            if (last < 0) continue;
+            const size_t ru = n0 + (size_t)u;
+            log_softmax_row(in->draft + ru * V, V, T, lq);
+            log_softmax_row(in->target + ru * V, V, T, lp);
+            for (int64_t v = 0; v < V; ++v) { q[v] = exp(lq[v]); p[v] = exp(lp[v]); }
+            for (int n = u + 1; n < N; ++n) {
+                if (par[n] != u) continue;
+                const int32_t t = in->tokens[n0 + n];
+                double alpha;
+                if (q[t] > 0.0) {
+                    alpha = p[t] / q[t];
+                    if (alpha > 1.0) alpha = 1.0;
+                } else {
+                    alpha = p[t] > 0.0 ? 1.0 : 0.0;
+                }
+                const double uu = (double)in->u_accept[n0 + n];
+                const uint8_t a = (uu <= alpha) ? 1 : 0;
+                out->alpha[n0 + n] = alpha;
+                out->accept[n0 + n] = a;
+                if (out->margins) out->margins[2 * (n0 + n)] = fabs(uu - alpha);
+                if (a) {
+                    out->path_accept[n0 + n] = 1;
+                    break;
+                }
+                /* rejected: p <- norm(max(0, p - q)), q <- q without t */
+                double Rm = 0.0;
+                for (int64_t v = 0; v < V; ++v) {
+                    const double dv = p[v] - q[v];
+                    res[v] = dv > 0.0 ? dv : 0.0;
+                    Rm += res[v];
+                }
+                if (Rm > 0.0)
+                    for (int64_t v = 0; v < V; ++v) p[v] = res[v] / Rm;
+                q[t] = 0.0;
+                double Qs = 0.0;
+                for (int64_t v = 0; v < V; ++v) Qs += q[v];
+                for (int64_t v = 0; v < V; ++v) q[v] = Qs > 0.0 ? q[v] / Qs : 0.0;
+                if (n == last) {  /* every child rejected: the correction token */
+                    double mg;
+                    out->corr_tokens[n0 + n] =
+                        (int32_t)sample_inverse_cdf(p, V, (double)in->u_correct[n0 + n], &mg);
+                    if (out->margins) out->margins[2 * (n0 + n) + 1] = mg;
+                }
+            }
+        }
+        /* the deepest accepted node; the bonus token after it */
+        int best = 0;
+        for (int n = 1; n < N; ++n)
+            if (out->path_accept[n0 + n] && depth[n] > depth[best]) best = n;
+        out->deepest[b] = best;
+        out->accept_len[b] = depth[best];
+        int last = -1;
+        for (int n = best + 1; n < N; ++n) if (par[n] == best) last = n;
+        int32_t bonus;
+        if (last >= 0) {
+            bonus = out->corr_tokens[n0 + last];
+        } else {
+            log_softmax_row(in->target + (n0 + best) * V, V, T, lp);
+            for (int64_t v = 0; v < V; ++v) p[v] = exp(lp[v]);
+            double mg;
+            bonus = (int32_t)sample_inverse_cdf(p, V, (double)in->u_correct[n0 + best], &mg);
+        }
+        out->bonus[b] = bonus;
+    }
+    return 0;
+}
+
 int vso_tree(const vso_tree_in* in, vso_tree_out* out)
 {
     const int B = in->B, N = in->N;
@@ -608,6 +739,11 @@ int vso_tree(const vso_tree_in* in, vso_tree_out* out)
     double* res = (double*)malloc(sizeof(double) * (size_t)V);
     int* depth = (int*)malloc(sizeof(int) * (size_t)N);
     int rc = 0;
+    if (in->rule == 1) {
+        rc = tree_sequential(in, out, lq, lp, q, p, res, depth);
+        free(lq); free(lp); free(q); free(p); free(res); free(depth);
+        return rc;
+    }
     for (int b = 0; b < B && !rc; ++b) {
         const int32_t* par = in->parent + (size_t)b * N;
         const size_t n0 = (size_t)b * N;
@@ -679,6 +815,203 @@ int vso_tree(const vso_tree_in* in, vso_tree_out* out)
         out->bonus[b] = bonus;
     }
     free(lq); free(lp); free(q); free(p); free(res); free(depth);
+    return rc;
+}
+
+/* ------------------------------------------------------------------ */
+/* R15: the E-step + M-step over draft trees, every node a latent proposal.  */
+typedef struct {
+    const float* draft;
+    const float* target;
+    int32_t B, N;
+    int64_t V;
+    double T;
+    const int32_t* parent;     /* [B][N] */
+    const int32_t* tokens;     /* [B][N] */
+    const float* u_accept;     /* [B][N] */
+    const float* u_correct;    /* [B][N] */
+    double w_base, tau_car;
+    int32_t zeta_mode;
+} vso_tree_em_in;
+
+typedef struct {
+    int32_t* corr_tokens;   /* [B][N] z'_x (root -1)                          */
+    double* logq_tok;       /* [B][N] log q_{par(x)}(t_x) (root 0)            */
+    double* logq_corr;      /* [B][N] log q_{par(x)}(z'_x)                     */
+    double* logkappa;       /* [B][N] sum of log alpha on the root path        */
+    double* logkappa_corr;  /* [B][N] of log alpha' (z')                       */
+    double* logkappa_ref;   /* [B][N] of log alpha-bar (the rows' argmaxes)    */
+    double* weights;        /* [B][N][4] o~, o', beta, zeta (root 0)           */
+    double* loss;           /* [B+1]                                          */
+    double* grad;           /* optional [B*N][V]                              */
+    double* margins;        /* optional [B][N][3]: accept, z' draw, o~        */
+} vso_tree_em_out;
+
+int vso_tree_em(const vso_tree_em_in* in, vso_tree_em_out* out)
+{
+    const int B = in->B, N = in->N;
+    const int64_t V = in->V;
+    const double T = in->T;
+    if (B < 1 || N < 1 || V < 1 || !(T > 0.0)) return 1;
+    double* lq = (double*)malloc(sizeof(double) * (size_t)V);
+    double* lp = (double*)malloc(sizeof(double) * (size_t)V);
+    double* q = (double*)malloc(sizeof(double) * (size_t)V);
+    double* p = (double*)malloc(sizeof(double) * (size_t)V);
+    double* res = (double*)malloc(sizeof(double) * (size_t)V);
+    double* lqall = (double*)malloc(sizeof(double) * (size_t)V * (size_t)N); /* log q per row */
+    int* depth = (int*)malloc(sizeof(int) * (size_t)N);
+    uint8_t* pacc = (uint8_t*)malloc((size_t)N);
+    double* lqpath = (double*)malloc(sizeof(double) * (size_t)N);
+    double* lcpath = (double*)malloc(sizeof(double) * (size_t)N);
+    int* grp = (int*)malloc(sizeof(int) * (size_t)N);
+    double* ot = (double*)malloc(sizeof(double) * (size_t)N);
+    double* op = (double*)malloc(sizeof(double) * (size_t)N);
+    double* lqz = (double*)malloc(sizeof(double) * (size_t)N);
+    double* zeta = (double*)malloc(sizeof(double) * (size_t)N);
+    double loss_sum = 0.0;
+    int rc = 0;
+    for (int b = 0; b < B && !rc; ++b) {
+        const int32_t* par = in->parent + (size_t)b * N;
+        const size_t n0 = (size_t)b * N;
+        if (par[0] != -1) { rc = 2; break; }
+        depth[0] = 0;
+        for (int n = 1; n < N; ++n) {
+            if (par[n] < 0 || par[n] >= n) { rc = 2; break; }
+            depth[n] = depth[par[n]] + 1;
+        }
+        if (rc) break;
+        for (int n = 0; n < N; ++n)
+            log_softmax_row(in->draft + (n0 + n) * V, V, T, lqall + (size_t)n * V);
+        double* W = out->weights + n0 * 4;
+        for (int i = 0; i < 4 * N; ++i) W[i] = 0.0;
+        /* E-step per position x (R15 with R3, R4): the token's test at its
+         * parent's row, the corrected token, the reference of that row */
+        pacc[0] = 1;
+        out->corr_tokens[n0] = -1;
+        out->logq_tok[n0] = out->logq_corr[n0] = 0.0;
+        out->logkappa[n0] = out->logkappa_corr[n0] = out->logkappa_ref[n0] = 0.0;
+        lqpath[0] = lcpath[0] = 0.0;
+        if (out->margins)
+            for (int k = 0; k < 3; ++k) out->margins[3 * n0 + k] = INFINITY;
+        for (int x = 1; x < N; ++x) {
+            const int a = par[x];
+            const size_t ra = n0 + (size_t)a;
+            const double* lqa = lqall + (size_t)a * V;
+            log_softmax_row(in->target + ra * V, V, T, lp);
+            for (int64_t v = 0; v < V; ++v) { q[v] = exp(lqa[v]); p[v] = exp(lp[v]); }
+            const int32_t t = in->tokens[n0 + x];
+            double alpha = p[t] / q[t];
+            if (alpha > 1.0) alpha = 1.0;
+            const double u = (double)in->u_accept[n0 + x];
+            const int acc = u <= alpha;
+            pacc[x] = (uint8_t)(acc && pacc[a]);
+            double mg = INFINITY;
+            int64_t zc;
+            if (pacc[x]) {
+                zc = t;
+            } else if (pacc[a]) { /* the first rejection on the path: residual */
+                double Rm = 0.0;
+                for (int64_t v = 0; v < V; ++v) {
+                    const double dv = p[v] - q[v];
+                    res[v] = dv > 0.0 ? dv : 0.0;
+                    Rm += res[v];
+                }
+                if (Rm > 0.0) {
+                    for (int64_t v = 0; v < V; ++v) res[v] /= Rm;
+                    zc = sample_inverse_cdf(res, V, (double)in->u_correct[n0 + x], &mg);
+                } else {
+                    zc = sample_inverse_cdf(p, V, (double)in->u_correct[n0 + x], &mg);
+                }
+            } else { /* below a rejection: a draw from p */
+                zc = sample_inverse_cdf(p, V, (double)in->u_correct[n0 + x], &mg);
+            }
+            double ac = p[zc] / q[zc];
+            if (ac > 1.0) ac = 1.0;
+            int64_t vb = 0;
+            const float* xp = in->target + ra * V;
+            for (int64_t v = 1; v < V; ++v) if (xp[v] > xp[vb]) vb = v;
+            double ab = p[vb] / q[vb];
+            if (ab > 1.0) ab = 1.0;
+            out->corr_tokens[n0 + x] = (int32_t)zc;
+            out->logq_tok[n0 + x] = lqa[t];
+            out->logq_corr[n0 + x] = lqa[zc];
+            out->logkappa[n0 + x] = out->logkappa[ra] + log(alpha);
+            out->logkappa_corr[n0 + x] = out->logkappa_corr[ra] + log(ac);
+            out->logkappa_ref[n0 + x] = out->logkappa_ref[ra] + log(ab);
+            lqpath[x] = lqpath[a] + lqa[t];
+            lcpath[x] = lcpath[a] + lqa[zc];
+            if (out->margins) {
+                out->margins[3 * (n0 + x)] = fabs(u - alpha);
+                out->margins[3 * (n0 + x) + 1] = mg;
+            }
+        }
+        /* M-step: o~, o' per proposal (Algorithm 2 with w(depth)) */
+        double Nb = 0.0;
+        for (int n = 1; n < N; ++n) {
+            const double lk = out->logkappa[n0 + n], lkr = out->logkappa_ref[n0 + n];
+            const double o_tilde = oracle_utility(lk, lkr, depth[n], in->w_base);
+            W[4 * n + 0] = o_tilde > 0.0 ? 1.0 : 0.0;
+            W[4 * n + 1] = o_tilde > 0.0 ? o_tilde
+                                          : oracle_utility(out->logkappa_corr[n0 + n], lkr,
+                                                           depth[n], in->w_base);
+            Nb += W[4 * n + 1];
+            if (out->margins) {
+                const double d = lk - lkr;
+                out->margins[3 * (n0 + n) + 2] = d == 0.0 ? 0.0 : fabs(d);
+            }
+        }
+        /* beta, zeta over the proposals of one length (the nodes of one depth) */
+        int maxd = 0;
+        for (int n = 1; n < N; ++n) if (depth[n] > maxd) maxd = depth[n];
+        for (int l = 1; l <= maxd; ++l) {
+            int m = 0;
+            for (int n = 1; n < N; ++n)
+                if (depth[n] == l) {
+                    grp[m] = n;
+                    ot[m] = W[4 * n + 0];
+                    op[m] = W[4 * n + 1];
+                    lqz[m] = lqpath[n];
+                    ++m;
+                }
+            if (m == 0) continue;
+            car_zeta(lqz, m, in->tau_car, in->zeta_mode, zeta);
+            for (int i = 0; i < m; ++i) {
+                W[4 * grp[i] + 2] = arw_beta(ot, op, m, i);
+                W[4 * grp[i] + 3] = zeta[i];
+            }
+        }
+        /* the objective (Eq. advance) and its gradient */
+        double J = 0.0;
+        double* G = out->grad ? out->grad + n0 * V : NULL;
+        if (G) memset(G, 0, sizeof(double) * (size_t)N * (size_t)V);
+        for (int n = 1; n < N; ++n) {
+            const double o_t = W[4 * n], o_p = W[4 * n + 1], beta = W[4 * n + 2], z = W[4 * n + 3];
+            if (o_p == 0.0) continue;
+            const double lqn = o_t > 0.0 ? lqpath[n] : lcpath[n];
+            J += o_p * (lqn - beta * z * lqpath[n]);
+            if (!G || Nb <= 0.0) continue;
+            const double c_pos = -o_p / ((double)B * Nb);
+            const double c_neg = o_p * beta * z / ((double)B * Nb);
+            for (int x = n; x > 0; x = par[x]) { /* the positions of the path */
+                const int a = par[x];
+                const double* lqa = lqall + (size_t)a * V;
+                double* g = G + (size_t)a * V;
+                const int32_t tz = o_t > 0.0 ? in->tokens[n0 + x] : out->corr_tokens[n0 + x];
+                const int32_t tt = in->tokens[n0 + x];
+                for (int64_t v = 0; v < V; ++v) {
+                    const double qv = exp(lqa[v]);
+                    g[v] += c_pos * ((v == tz ? 1.0 : 0.0) - qv) / T +
+                            c_neg * ((v == tt ? 1.0 : 0.0) - qv) / T;
+                }
+            }
+        }
+        const double lb = Nb > 0.0 ? -J / Nb : 0.0;
+        out->loss[b] = lb;
+        loss_sum += lb;
+    }
+    if (!rc) out->loss[B] = loss_sum / (double)B;
+    free(lq); free(lp); free(q); free(p); free(res); free(lqall); free(depth); free(pacc);
+    free(lqpath); free(lcpath); free(grp); free(ot); free(op); free(lqz); free(zeta);
     return rc;
 }
 

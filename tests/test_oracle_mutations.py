@@ -85,6 +85,18 @@ MUTATIONS = [
      "    if (0) {\n        greedy_one_hot(xq, V, q);"),
     ("supplied reference ratio inverted", "            double ab = p[vb] / q[vb];\n            if (ab > 1.0) ab = 1.0;\n            acc += log(ab);",
      "            double ab = q[vb] / p[vb];\n            if (ab > 1.0) ab = 1.0;\n            acc += log(ab);"),
+    ("sequential rule keeps the residual target", "                if (Rm > 0.0)\n                    for (int64_t v = 0; v < V; ++v) p[v] = res[v] / Rm;\n                q[t] = 0.0;",
+     "                q[t] = 0.0;"),
+    ("sequential rule keeps rejected siblings in q", "                q[t] = 0.0;\n                double Qs = 0.0;",
+     "                double Qs = 0.0;"),
+    ("sequential rule tries children of rejected nodes", "            if (!out->path_accept[n0 + u]) continue;\n            int last = -1;",
+     "            int last = -1;"),
+    ("tree EM beta over all proposals", "                if (depth[n] == l) {\n                    grp[m] = n;",
+     "                if (depth[n] >= 1) {\n                    grp[m] = n;"),
+    ("tree EM z' below a rejection is the residual", "            } else { /* below a rejection: a draw from p */\n                zc = sample_inverse_cdf(p, V,",
+     "            } else { /* below a rejection: a draw from p */\n                zc = sample_inverse_cdf(q, V,"),
+    ("tree EM weight of the parent's depth", "            const double o_tilde = oracle_utility(lk, lkr, depth[n], in->w_base);",
+     "            const double o_tilde = oracle_utility(lk, lkr, depth[n] - 1, in->w_base);"),
     ("margin: unequal sums given no margin", "if (a != b) return fabs(a - b);",
      "if (a != b) return 0.0;"),
     ("margin: a clipped tie given no margin", "        if (ra[i] < m) m = ra[i];\n", ""),

@@ -816,3 +816,130 @@ def test_reference_rows_worked_example(oracle):
     target = np.stack([logits(p1), logits(p2)])
     ref = oracle.reference_logkappa(draft, target, 1.0, 1, 2)
     assert abs(ref[0, 0]) < 1e-7 and abs(ref[0, 1] - math.log(0.75)) < 1e-7
+
+
+# --------------------------------------------------------------------------
+# Trees: the sequential sibling rule (reading R14) and the tree EM (R15).
+
+
+def _chain_tree(B, N, V, seed, same=False):
+    rng = np.random.default_rng(seed)
+    draft = rng.normal(0, 2, (B * N, V)).astype(np.float32)
+    target = draft.copy() if same else (draft + rng.normal(0, 1, (B * N, V))).astype(np.float32)
+    parent = np.tile(np.arange(-1, N - 1, dtype=np.int32), (B, 1))
+    tokens = rng.integers(0, V, (B, N)).astype(np.int32)
+    ua = rng.random((B, N)).astype(np.float32)
+    uc = rng.random((B, N)).astype(np.float32)
+    return draft, target, parent, tokens, ua, uc
+
+
+def test_sequential_rule_on_chains_is_the_independent_rule(oracle):
+    """With one child per node there is nothing to try in turn: the accepted
+    path, the correction and the bonus are the independent rule's."""
+    args = _chain_tree(6, 7, 40, 51)
+    a = oracle.tree(*args[:2], 1.0, *args[2:], rule=0)
+    s = oracle.tree(*args[:2], 1.0, *args[2:], rule=1)
+    for n in ("path_accept", "deepest", "accept_len", "bonus", "corr_tokens", "logkappa"):
+        assert np.array_equal(a[n], s[n]), n
+    tried = np.zeros_like(a["accept"], bool)
+    tried[:, 1:] = a["path_accept"][:, :-1] == 1  # a child is tried when its parent is accepted
+    assert np.array_equal(a["accept"][tried], s["accept"][tried])
+    assert np.array_equal(a["alpha"][tried], s["alpha"][tried])
+    untried = ~tried[:, 1:]  # (the root is node 0)
+    assert np.all(s["accept"][:, 1:][untried] == 0) and np.all(s["alpha"][:, 1:][untried] == 0)
+
+
+def test_sequential_rule_is_lossless(oracle):
+    """A root with three children drawn without replacement from q: the token
+    the step emits (the accepted child's, or the correction when all are
+    rejected) is distributed as p.  Monte Carlo over 2^18 seeded trees: every
+    frequency within 5 standard errors of p, while the independent rule's
+    first-accepted-or-residual output is visibly off."""
+    V, m, n = 5, 3, 1 << 18
+    rng = np.random.default_rng(52)
+    xq = np.array([1.2, 0.3, -0.5, 0.9, -1.0], np.float32)
+    xp = np.array([-0.4, 1.1, 0.6, -0.2, 0.2], np.float32)
+    q = np.exp(oracle.log_softmax(xq))
+    p = np.exp(oracle.log_softmax(xp))
+    # children tokens: sequential draws from q without replacement
+    g = -np.log(-np.log(rng.random((n, V))))
+    toks = np.argsort(-(np.log(q)[None, :] + g), axis=1)[:, :m].astype(np.int32)
+    N = m + 1
+    draft = np.tile(xq, (n * N, 1))
+    target = np.tile(xp, (n * N, 1))
+    parent = np.tile(np.array([-1] + [0] * m, np.int32), (n, 1))
+    tokens = np.concatenate([np.zeros((n, 1), np.int32), toks], axis=1)
+    ua = rng.random((n, N)).astype(np.float32)
+    uc = rng.random((n, N)).astype(np.float32)
+    o = oracle.tree(draft, target, 1.0, parent, tokens, ua, uc, rule=1)
+    out = np.where(o["deepest"] > 0, tokens[np.arange(n), o["deepest"]], o["bonus"])
+    freq = np.bincount(out, minlength=V) / n
+    se = np.sqrt(p * (1 - p) / n)
+    assert np.all(np.abs(freq - p) < 5 * se), (freq, p)
+    # (the Gumbel-top-k draws above are exactly sequential draws without replacement)
+    assert abs(np.mean(toks[:, 0] == 0) - q[0]) < 5 * np.sqrt(q[0] * (1 - q[0]) / n)
+
+
+def test_sequential_first_child_accepted_when_draft_is_target(oracle):
+    B, N, V = 4, 6, 30
+    rng = np.random.default_rng(53)
+    x = rng.normal(0, 2, (B * N, V)).astype(np.float32)
+    parent = np.tile(np.array([-1, 0, 0, 0, 1, 1], np.int32), (B, 1))
+    tokens = rng.integers(0, V, (B, N)).astype(np.int32)
+    o = oracle.tree(x, x, 1.0, parent, tokens, rng.random((B, N)).astype(np.float32),
+                    rng.random((B, N)).astype(np.float32), rule=1)
+    assert np.all(o["path_accept"][:, [1, 4]] == 1) and np.all(o["path_accept"][:, [2, 3, 5]] == 0)
+    assert np.all(o["deepest"] == 4) and np.all(o["accept_len"] == 2)
+
+
+def test_tree_em_of_shared_root_chains_is_the_linear_em(oracle):
+    """K chains of depth D below one root, the root's row shared: the tree's
+    proposals at depth l are the K linear paths' length-l proposals, so the
+    tree EM equals the linear EM of K paths whose first rows coincide (the
+    root row's gradient is the sum of the K first rows')."""
+    from paper_2602_05774_gb300 import inputs
+    K, D, V, T = 4, 3, 50, 0.8
+    pr = inputs.linear_problem(1, K, D, V, "f32", "gauss", seed=56)
+    f = {k: pr[k].numpy().copy() for k in ("draft", "target", "u_draft", "u_accept", "u_correct")}
+    for s in range(1, K):  # the first rows of every path coincide
+        f["draft"][s * D] = f["draft"][0]
+        f["target"][s * D] = f["target"][0]
+    lin = oracle.linear(f["draft"], f["target"], T, f["u_draft"], f["u_accept"], f["u_correct"],
+                        K, D, w_base=1.1, tau_car=0.3)
+    # the case exercises both o~ values and positions below a rejection
+    assert set(np.unique(lin["weights"][..., 0])) == {0.0, 1.0}
+    assert np.any(lin["accept_len"] < D - 1)
+    N = 1 + K * D
+    node = lambda s, j: 1 + (j - 1) * K + s  # node of path s at depth j >= 1
+    parent = np.full(N, -1, np.int32)
+    tokens = np.zeros(N, np.int32)
+    ua = np.zeros(N, np.float32)
+    uc = np.zeros(N, np.float32)
+    draft = np.zeros((N, V), np.float32)
+    target = np.zeros((N, V), np.float32)
+    draft[0], target[0] = f["draft"][0], f["target"][0]
+    for s in range(K):
+        for j in range(1, D + 1):
+            x = node(s, j)
+            parent[x] = 0 if j == 1 else node(s, j - 1)
+            r = s * D + j - 1
+            tokens[x], ua[x], uc[x] = lin["tokens"][r], f["u_accept"][r], f["u_correct"][r]
+            rr = s * D + min(j, D - 1)  # the row of node x: linear row (s, j); leaves any row
+            draft[x], target[x] = f["draft"][rr], f["target"][rr]
+    t = oracle.tree_em(draft, target, T, parent[None], tokens[None], ua[None], uc[None],
+                       w_base=1.1, tau_car=0.3)
+    for s in range(K):
+        for j in range(1, D + 1):
+            x, r = node(s, j), s * D + j - 1
+            assert t["corr_tokens"][0, x] == lin["corr_tokens"][r]
+            for n in ("logkappa", "logkappa_corr", "logkappa_ref", "logq_corr"):
+                assert abs(t[n][0, x] - lin[n][r]) < 1e-12, n
+            assert np.allclose(t["weights"][0, x], lin["weights"][0, j - 1, s], rtol=1e-12,
+                               atol=1e-15)
+    assert abs(t["loss"][0] - lin["loss"][0]) < 1e-12
+    g = t["grad"]
+    assert np.allclose(g[0], sum(lin["grad"][s * D] for s in range(K)), atol=1e-14)
+    for s in range(K):
+        for j in range(1, D):
+            assert np.allclose(g[node(s, j)], lin["grad"][s * D + j], atol=1e-14)
+        assert np.all(g[node(s, D)] == 0.0)  # a leaf's row carries no term
