@@ -78,10 +78,23 @@ typedef enum { VSD_F32 = 0, VSD_BF16 = 1 } vsd_dtype;
 
 /* Problem shape.  parent == NULL: linear paths, R = B*K*D rows, N unused.
  * parent != NULL: draft trees, device array [B][N] of parent indices
- * (parent[b][0] = -1, 0 <= parent[b][n] < n), R = B*N rows, K and D unused. */
+ * (parent[b][0] = -1, 0 <= parent[b][n] < n), R = B*N rows, K and D unused.
+ * tree_rule (trees, vsd_verify_paths): VSD_TREE_INDEPENDENT verifies every
+ * branch alone (a node is accepted when it and its ancestors pass their own
+ * test); VSD_TREE_SEQUENTIAL is the lossless multi-draft rule: along the
+ * accepted path a node's children are tried in node order, child i accepted
+ * with probability min(1, p_i(t_i)/q_i(t_i)), where after each rejection
+ * p_{i+1} = norm(max(0, p_i - q_i)) and q_{i+1} = q_i with t_i removed and
+ * renormalised; the first accepted child continues the path, and when every
+ * child is rejected the correction token is drawn from p_{m+1} with the last
+ * child's u_correct.  The emitted token is then distributed as p whenever the
+ * siblings are drawn from q without replacement. */
+#define VSD_TREE_INDEPENDENT 0
+#define VSD_TREE_SEQUENTIAL 1
 typedef struct {
     int32_t B, K, D, V, N;
     const int32_t* parent;
+    int32_t tree_rule;
 } vsd_layout;
 
 /* M-step parameters (App. F: w(l) = 1.05^l, tau = 0.2). */
@@ -147,6 +160,30 @@ typedef struct {
                                row's invalid values then set no status bit        */
 } vsd_tree_outputs;
 
+/* Outputs of the E-step + M-step over draft trees (vsd_tree_estep_mstep;
+ * device, caller-owned, [B][N] unless noted; node 0, the root, is no
+ * proposal and holds zeros).  Every node n >= 1 is a latent proposal: the
+ * tokens on its root path, of length depth(n). */
+typedef struct {
+    int32_t* corr_tokens;   /* z'_n: n's token on an accepted path, the residual
+                               norm(max(0, p - q)) at the path's first rejected
+                               node, a draw from p below it (each with n's own
+                               u_correct, at n's parent's row); root -1          */
+    float* logq_tok;        /* log q of n's token at its parent's row            */
+    float* logq_corr;       /* log q of z'_n there                               */
+    float* logkappa;        /* log kappa of the root path of n (Eq. 2)           */
+    float* logkappa_corr;   /* of the corrected path                             */
+    float* logkappa_ref;    /* of the greedy reference along the same rows
+                               (each row's target argmax, Algorithm 2)           */
+    float* weights;         /* [B][N][4] o~, o', beta, zeta; beta and zeta over
+                               the nodes of one depth                            */
+    float* loss;            /* [B+1] loss_b = -J_b/N_b (Eq. advance), then the mean */
+    void* grad;             /* [B*N][V] d loss / d draft logits, params.grad_dtype:
+                               row n collects the terms of every proposal whose
+                               path goes through one of n's children; a leaf's
+                               row is 0                                          */
+} vsd_tree_em_outputs;
+
 /* Bytes of device workspace the calls below need for `layout` (0 if invalid). */
 size_t vsd_workspace_bytes(vsd_layout layout);
 
@@ -206,6 +243,22 @@ vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtyp
                            const float* u_accept, const float* u_correct,
                            const float* ref_logkappa, const vsd_params* params,
                            vsd_linear_outputs* out, void* ws, size_t ws_bytes, void* stream);
+
+/* The E-step + M-step over draft trees (App. E trees as the latent
+ * proposals; Algorithm 1 and 2, Eqs. 1, 2, beta, zeta, advance on the trees'
+ * root paths).  Each position x of a path is verified alone (Eq. 1 at x's
+ * parent's row; the path validity of Eq. 2), the corrected path follows
+ * Sec. 3 along the branch, o~ and o' use w(depth), beta and zeta run over the
+ * proposals of one length (the nodes of one depth), and the loss and its
+ * gradient are Eq. advance's.  Arguments as for vsd_verify_paths with a tree
+ * layout (tokens [B][N], node 0 ignored; u_accept, u_correct [B][N]) plus
+ * params (NULL: the defaults; kl_weight must be 0).  Required outputs: loss,
+ * grad; the rest optional.  T > 0.  Errors as for vsd_estep_mstep. */
+vsd_status vsd_tree_estep_mstep(const void* draft, const void* target, vsd_dtype dtype,
+                                vsd_layout layout, float T, const int32_t* tokens,
+                                const float* u_accept, const float* u_correct,
+                                const vsd_params* params, vsd_tree_em_outputs* out, void* ws,
+                                size_t ws_bytes, void* stream);
 
 /* Allocation-free variant of vsd_estep_mstep; the paper has no counterpart.
  * For callers that cannot allocate device memory where they call the library

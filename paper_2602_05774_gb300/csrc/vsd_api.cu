@@ -29,7 +29,7 @@ struct WsLayout {
     size_t status, ticket, prefix_done, grad_head, resq_head, resq_tail, resq_avail;
     size_t path_cnt, prefix_cnt, ready, grad_cnt, row_seg_cnt, res_seg_cnt, resq_flag, zero_end;
     size_t rows, rstats, es_tok, es_corr, es_lq_tok, es_lq_corr, es_lk, es_lkc, es_lkr;
-    size_t coef, wscr, path_A, resq, klr, gtab, total;
+    size_t coef, wscr, path_A, resq, klr, gtab, tnode, tcoef, tg, tbad, total;
     int nch_ws, nseg_ws;
 };
 
@@ -59,6 +59,8 @@ bool layout_ok(const vsd_layout& L) {
     if (L.B < 1 || L.V < 1 || L.V > kMaxV) return false;
     if (L.parent) {
         if (L.N < 1 || L.N > kMaxN) return false;
+        if (L.tree_rule != VSD_TREE_INDEPENDENT && L.tree_rule != VSD_TREE_SEQUENTIAL)
+            return false;
         return (int64_t)L.B * L.N <= kMaxRows;
     }
     if (L.K < 1 || L.K > kMaxK || L.D < 1 || L.D > kMaxD) return false;
@@ -112,6 +114,12 @@ WsLayout ws_layout(const vsd_layout& L) {
     w.resq = o; o = align256(o + 4 * nq);
     w.klr = o; o = align256(o + sizeof(KlRec) * R);
     w.gtab = o; o = align256(o + sizeof(float4) * R * (size_t)w.nch_ws);
+    // trees: the node records, gradient terms and flags of the tree EM
+    const size_t Rt = L.parent ? R : 0;
+    w.tnode = o; o = align256(o + sizeof(TreeNodeRec) * Rt);
+    w.tcoef = o; o = align256(o + sizeof(TreeCoef) * Rt);
+    w.tg = o; o = align256(o + 4 * Rt);
+    w.tbad = o; o = align256(o + (L.parent ? 4 * (size_t)L.B : 0));
     w.total = o;
     return w;
 }
@@ -238,6 +246,10 @@ Problem<T> make_problem(const void* draft, const void* target, const vsd_layout&
     // hold its residual lists and its nodes' log alpha
     P.stream_tails = 0;
     P.resq_sem = 1;
+    P.tnode = L.parent ? at<TreeNodeRec>(ws, w.tnode) : nullptr;
+    P.tcoef = L.parent ? at<TreeCoef>(ws, w.tcoef) : nullptr;
+    P.tg = L.parent ? at<float>(ws, w.tg) : nullptr;
+    P.tbad = L.parent ? at<int>(ws, w.tbad) : nullptr;
     P.tlist = at<int>(ws, w.es_tok);
     P.tcount = at<int>(ws, w.path_A);
     P.tla = at<float>(ws, w.es_lq_tok);
@@ -366,7 +378,9 @@ vsd_status verify_impl(const void* draft, const void* target, vsd_layout L, floa
     cudaError_t e = clear_counters(ws, L, s);
     if (L.parent) {
         P.tout = *tout;
-        if (e == cudaSuccess) e = Launch<T>::tree(P, vec, s);
+        if (e == cudaSuccess)
+            e = L.tree_rule == VSD_TREE_SEQUENTIAL ? Launch<T>::tree_seq(P, vec, s)
+                                                   : Launch<T>::tree(P, vec, s);
     } else {
         P.out = *out;
         if (e == cudaSuccess) e = Launch<T>::rows_verify(P, vec, s);
@@ -533,6 +547,46 @@ vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtyp
                                      ref_logkappa, p, out, ws, s);
 }
 
+vsd_status vsd_tree_estep_mstep(const void* draft, const void* target, vsd_dtype dtype,
+                                vsd_layout layout, float T, const int32_t* tokens,
+                                const float* u_accept, const float* u_correct,
+                                const vsd_params* params, vsd_tree_em_outputs* out, void* ws,
+                                size_t ws_bytes, void* stream) {
+    if (!layout_ok(layout) || !layout.parent) return VSD_ERR_INVALID_ARG;
+    if (!draft || !target || !tokens || !u_accept || !u_correct || !out || !out->loss ||
+        !out->grad)
+        return VSD_ERR_INVALID_ARG;
+    if (dtype != VSD_F32 && dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
+    vsd_status st = check_temperature(T);
+    if (st) return st;
+    const vsd_params p = params ? *params : default_params(dtype);
+    if ((st = check_params(p))) return st;
+    if (p.kl_weight != 0.0) return VSD_ERR_UNSUPPORTED;
+    if ((st = check_ws(layout, ws, ws_bytes))) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = clear_counters(ws, layout, s);
+    if (e != cudaSuccess) return from_cuda(e);
+    const size_t gelem = p.grad_dtype == VSD_BF16 ? 2 : 4;
+    if (dtype == VSD_F32) {
+        Problem<float> P = make_problem<float>(draft, target, layout, T, ws);
+        set_params(P, p);
+        P.given_tokens = tokens;
+        P.u_accept = u_accept;
+        P.u_correct = u_correct;
+        e = Launch<float>::tree_em(P, vec_ok(draft, target, out->grad, layout.V, 4, gelem), *out,
+                                   out->grad, P.grad_bf16, s);
+    } else {
+        Problem<__nv_bfloat16> P = make_problem<__nv_bfloat16>(draft, target, layout, T, ws);
+        set_params(P, p);
+        P.given_tokens = tokens;
+        P.u_accept = u_accept;
+        P.u_correct = u_correct;
+        e = Launch<__nv_bfloat16>::tree_em(P, vec_ok(draft, target, out->grad, layout.V, 2, gelem),
+                                           *out, out->grad, P.grad_bf16, s);
+    }
+    return from_cuda(e);
+}
+
 vsd_status vsd_lmhead_logits(const void* hidden, const void* weight, int32_t M, int32_t N,
                              int32_t K, void* logits, void* ws, size_t ws_bytes, void* stream) {
     if (!lmhead_shape_ok(hidden, weight, logits, M, N, K)) return VSD_ERR_INVALID_ARG;
@@ -583,7 +637,7 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
 vsd_status vsd_reference_logkappa(const void* ref_draft, const void* ref_target, vsd_dtype dtype,
                                   int32_t B, int32_t D, int32_t V, float T, float* ref_logkappa,
                                   void* ws, size_t ws_bytes, void* stream) {
-    const vsd_layout L{B, 1, D, V, 0, nullptr};
+    const vsd_layout L{B, 1, D, V, 0, nullptr, 0};
     if (!layout_ok(L)) return VSD_ERR_INVALID_ARG;
     if (!ref_draft || !ref_target || !ref_logkappa) return VSD_ERR_INVALID_ARG;
     if (dtype != VSD_F32 && dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;

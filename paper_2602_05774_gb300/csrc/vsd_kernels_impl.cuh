@@ -734,6 +734,44 @@ cudaError_t Launch<VSD_T>::tree(const Problem<VSD_T>& P, bool vec, cudaStream_t 
 }
 
 template <>
+cudaError_t Launch<VSD_T>::tree_seq(const Problem<VSD_T>& P, bool vec, cudaStream_t s) {
+    const size_t smem = stream_smem_bytes(P.nch, vec);
+    auto rows = vec ? k_tree_rows<VSD_T, true, false> : k_tree_rows<VSD_T, false, false>;
+    cudaError_t e = prep(rows, smem);
+    if (e) return e;
+    rows<<<P.R, kThreads, smem, s>>>(P);
+    if ((e = cudaGetLastError())) return e;
+    const size_t sm2 = sizeof(TreeSeqShared) + table_smem_bytes(P.nch);
+    auto seq = vec ? k_tree_seq<VSD_T, true> : k_tree_seq<VSD_T, false>;
+    if ((e = prep(seq, sm2))) return e;
+    seq<<<P.B, kThreads, sm2, s>>>(P);
+    return cudaGetLastError();
+}
+
+template <>
+cudaError_t Launch<VSD_T>::tree_em(const Problem<VSD_T>& P, bool vec,
+                                   const vsd_tree_em_outputs& o, void* grad, bool grad_bf16,
+                                   cudaStream_t s) {
+    const size_t smem = stream_smem_bytes(P.nch, vec);
+    auto rows = vec ? k_tree_rows<VSD_T, true, true> : k_tree_rows<VSD_T, false, true>;
+    cudaError_t e = prep(rows, smem);
+    if (e) return e;
+    rows<<<P.R, kThreads, smem, s>>>(P);
+    if ((e = cudaGetLastError())) return e;
+    if ((e = prep(k_tree_em<VSD_T>, sizeof(TreeEmShared)))) return e;
+    k_tree_em<VSD_T><<<P.B, kThreads, sizeof(TreeEmShared), s>>>(P, o);
+    if ((e = cudaGetLastError())) return e;
+#define VSD_TGRAD(V_, G_) \
+    k_tree_grad<VSD_T, V_, G_><<<P.R, kThreads, 0, s>>>(P, reinterpret_cast<G_*>(grad))
+    if (vec && grad_bf16) VSD_TGRAD(true, __nv_bfloat16);
+    else if (vec) VSD_TGRAD(true, float);
+    else if (grad_bf16) VSD_TGRAD(false, __nv_bfloat16);
+    else VSD_TGRAD(false, float);
+#undef VSD_TGRAD
+    return cudaGetLastError();
+}
+
+template <>
 cudaError_t Launch<VSD_T>::weights(const Problem<VSD_T>& P, const EStepView& E, float* weights,
                                    float* loss, cudaStream_t s) {
     k_weights<VSD_T><<<P.B, kThreads, 0, s>>>(P, E, weights, loss);

@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 
 #include "vsd_passes.cuh"
+#include "vsd_tree.cuh"
 
 namespace vsd {
 
@@ -20,6 +21,11 @@ template <typename T> struct Launch {
     // tree verification in one persistent launch: node rows, acceptance scan,
     // residual draws, deepest node, bonus
     static cudaError_t tree(const Problem<T>& P, bool vec, cudaStream_t s);
+    // tree verification with the sequential sibling rule
+    static cudaError_t tree_seq(const Problem<T>& P, bool vec, cudaStream_t s);
+    // the E-step + M-step over draft trees (node rows, per-tree M-step, gradient rows)
+    static cudaError_t tree_em(const Problem<T>& P, bool vec, const vsd_tree_em_outputs& o,
+                               void* grad, bool grad_bf16, cudaStream_t s);
     // M-step weights and loss from an E-step view
     static cudaError_t weights(const Problem<T>& P, const EStepView& E, float* weights,
                               float* loss, cudaStream_t s);

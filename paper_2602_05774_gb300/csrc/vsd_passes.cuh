@@ -160,6 +160,10 @@ struct Problem {
     int xtab_given;               // fused kernel: gtab[r][ch].xy (the draft's chunk
                                   // statistics) were written by the LM head's epilogue
     int* path_A;                  // [B*K] accepted length of a path
+    struct TreeNodeRec* tnode;    // trees beyond independent verification: [R] node records
+    struct TreeCoef* tcoef;       // [R] each node's gradient terms at its parent's row
+    float* tg;                    // [R] each row's dense gradient factor
+    int* tbad;                    // [B] the tree failed its checks
     int* tlist;                   // tree layout: [R] residual rows of each tree (its rows' slots)
     int* tcount;                  // tree layout: [B] length of each tree's list
     float* tla;                   // tree layout: [R] log alpha of each node's token

@@ -24,7 +24,7 @@ SYMBOLS = ("vsd_workspace_bytes", "vsd_sample_paths", "vsd_verify_paths",
            "vsd_weighted_loss_fwd_bwd", "vsd_estep_mstep", "vsd_device_status",
            "vsd_status_string", "vsd_version", "vsd_estep_mstep_noalloc",
            "vsd_noalloc_device_status", "vsd_lmhead_logits", "vsd_lmhead_estep_mstep",
-           "vsd_reference_logkappa")
+           "vsd_reference_logkappa", "vsd_tree_estep_mstep")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -37,7 +37,10 @@ class VsdError(RuntimeError):
 
 class Layout(C.Structure):
     _fields_ = [("B", C.c_int32), ("K", C.c_int32), ("D", C.c_int32), ("V", C.c_int32),
-                ("N", C.c_int32), ("parent", C.c_void_p)]
+                ("N", C.c_int32), ("parent", C.c_void_p), ("tree_rule", C.c_int32)]
+
+
+TREE_INDEPENDENT, TREE_SEQUENTIAL = 0, 1
 
 
 class Params(C.Structure):
@@ -53,6 +56,8 @@ LINEAR_FIELDS = ("tokens", "logq_tok", "alpha", "accept", "accept_len", "corr_to
                  "kl_loss")
 TREE_FIELDS = ("alpha", "accept", "path_accept", "logkappa", "corr_tokens", "deepest",
                "accept_len", "bonus", "row_stats")
+TREE_EM_FIELDS = ("corr_tokens", "logq_tok", "logq_corr", "logkappa", "logkappa_corr",
+                  "logkappa_ref", "weights", "loss", "grad")
 
 
 class LinearOutputs(C.Structure):
@@ -61,6 +66,10 @@ class LinearOutputs(C.Structure):
 
 class TreeOutputs(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in TREE_FIELDS]
+
+
+class TreeEmOutputs(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in TREE_EM_FIELDS]
 
 
 _LIB = None
@@ -103,12 +112,16 @@ def _lib():
         lib.vsd_noalloc_device_status.argtypes = [vp, C.POINTER(C.c_int32)]
         lib.vsd_reference_logkappa.argtypes = [vp, vp, C.c_int, C.c_int32, C.c_int32, C.c_int32,
                                                C.c_float, vp, vp, C.c_size_t, vp]
+        lib.vsd_tree_estep_mstep.argtypes = [vp, vp, C.c_int, Layout, C.c_float, vp, vp, vp,
+                                             C.POINTER(Params), C.POINTER(TreeEmOutputs), vp,
+                                             C.c_size_t, vp]
         lib.vsd_status_string.argtypes = [C.c_int]
         lib.vsd_status_string.restype = C.c_char_p
         lib.vsd_version.restype = C.c_char_p
         for name in ("vsd_sample_paths", "vsd_verify_paths", "vsd_weighted_loss_fwd_bwd",
                      "vsd_estep_mstep", "vsd_device_status", "vsd_estep_mstep_noalloc",
                      "vsd_noalloc_device_status", "vsd_reference_logkappa",
+                     "vsd_tree_estep_mstep",
                      "vsd_lmhead_logits", "vsd_lmhead_estep_mstep"):
             getattr(lib, name).restype = C.c_int
         _LIB = lib
@@ -150,9 +163,9 @@ def _need_cuda(*ts):
                 raise ValueError("tensors must be contiguous")
 
 
-def layout(B, K=1, D=1, V=1, N=0, parent=None):
+def layout(B, K=1, D=1, V=1, N=0, parent=None, tree_rule=TREE_INDEPENDENT):
     return Layout(int(B), int(K), int(D), int(V), int(N),
-                  None if parent is None else parent.data_ptr())
+                  None if parent is None else parent.data_ptr(), int(tree_rule))
 
 
 def workspace_bytes(lay):
@@ -282,12 +295,14 @@ def tree_outputs(B, N, device, row_stats=True):
     return o
 
 
-def verify_tree(draft, target, parent, tokens, u_accept, u_correct, T, workspace=None, out=None):
-    """Tree verification (App. E tree, Eq. 1 per node, Sec. 3 residual)."""
+def verify_tree(draft, target, parent, tokens, u_accept, u_correct, T, workspace=None, out=None,
+                rule=TREE_INDEPENDENT):
+    """Tree verification (App. E tree, Eq. 1 per node, Sec. 3 residual); rule
+    TREE_SEQUENTIAL tries siblings in turn (lossless multi-draft)."""
     _need_cuda(draft, target, parent, tokens, u_accept, u_correct)
     V = draft.shape[-1]
     B, N = parent.shape
-    lay = layout(B, V=V, N=N, parent=parent)
+    lay = layout(B, V=V, N=N, parent=parent, tree_rule=rule)
     dev = draft.device
     ws = _ws(workspace, lay, dev)
     o = out if out is not None else tree_outputs(B, N, dev)
@@ -296,6 +311,38 @@ def verify_tree(draft, target, parent, tokens, u_accept, u_correct, T, workspace
                                    _ptr(tokens), _ptr(u_accept), _ptr(u_correct), None, None,
                                    C.byref(st), _ptr(ws), ws.numel(), _stream(dev)),
            "vsd_verify_paths(tree)")
+    return o
+
+
+def tree_estep_mstep(draft, target, parent, tokens, u_accept, u_correct, T, prm=None,
+                     workspace=None, full=True):
+    """The E-step + M-step over draft trees, every node a latent proposal
+    (vsd_tree_estep_mstep).  Returns the outputs by name."""
+    _need_cuda(draft, target, parent, tokens, u_accept, u_correct)
+    V = draft.shape[-1]
+    B, N = parent.shape
+    lay = layout(B, V=V, N=N, parent=parent)
+    dev = draft.device
+    ws = _ws(workspace, lay, dev)
+    prm = prm or params(like=draft)
+    gdt = torch.bfloat16 if prm.grad_dtype == VSD_BF16 else torch.float32
+    f = dict(device=dev)
+    o = dict(loss=torch.empty(B + 1, dtype=torch.float32, **f),
+             grad=torch.empty(B * N, V, dtype=gdt, **f))
+    if full:
+        o.update(corr_tokens=torch.empty(B, N, dtype=torch.int32, **f),
+                 logq_tok=torch.empty(B, N, dtype=torch.float32, **f),
+                 logq_corr=torch.empty(B, N, dtype=torch.float32, **f),
+                 logkappa=torch.empty(B, N, dtype=torch.float32, **f),
+                 logkappa_corr=torch.empty(B, N, dtype=torch.float32, **f),
+                 logkappa_ref=torch.empty(B, N, dtype=torch.float32, **f),
+                 weights=torch.empty(B, N, 4, dtype=torch.float32, **f))
+    st = TreeEmOutputs(*[o[n].data_ptr() if o.get(n) is not None else None
+                         for n in TREE_EM_FIELDS])
+    _check(_lib().vsd_tree_estep_mstep(_ptr(draft), _ptr(target), _dtype_code(draft), lay,
+                                       float(T), _ptr(tokens), _ptr(u_accept), _ptr(u_correct),
+                                       C.byref(prm), C.byref(st), _ptr(ws), ws.numel(),
+                                       _stream(dev)), "vsd_tree_estep_mstep")
     return o
 
 
@@ -359,7 +406,7 @@ def reference_logkappa(ref_draft, ref_target, B, D, T, workspace=None):
     _check(_lib().vsd_reference_logkappa(_ptr(ref_draft), _ptr(ref_target),
                                          _dtype_code(ref_draft), int(B), int(D), int(V), float(T),
                                          _ptr(out), _ptr(ws), ws.numel(), _stream(dev)),
-           "vsd_reference_logkappa")
+           "vsd_reference_logkappa", "vsd_tree_estep_mstep")
     return out
 
 

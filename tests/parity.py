@@ -408,3 +408,95 @@ def compare_tree(gpu, orc, report=None):
     neg = ok[:, None] & np.isneginf(ol)
     assert np.all(np.isneginf(gl[neg])), "log kappa finite where the oracle has -inf"
     return int(div.sum())
+
+
+def compare_tree_sequential(gpu, orc, report=None):
+    """Tree parity under the sequential sibling rule.  The walk visits nodes in
+    increasing index order, so the first (lowest-index) node where an accept
+    bit or a correction token differs is the decision that flipped: it must be
+    within its margin, and the tree is then excluded (budget)."""
+    m = orc["margins"]
+    B = m.shape[0]
+    ga, oa = to_np(gpu["accept"]), orc["accept"]
+    gc, oc = to_np(gpu["corr_tokens"]), orc["corr_tokens"]
+    div = np.zeros(B, bool)
+    for b in range(B):
+        bad = np.nonzero((ga[b] != oa[b]) | (gc[b] != oc[b]))[0]
+        if bad.size == 0:
+            continue
+        n = bad[0]
+        marg = m[b, n, 0] if ga[b, n] != oa[b, n] else m[b, n, 1]
+        assert marg < PROB_MARGIN, "tree %d: decision at node %d differs outside the margin (%g)" % (
+            b, n, marg)
+        div[b] = True
+    ok = ~div
+    SESSION["trees"] += B
+    SESSION["excluded_trees"] += int(div.sum())
+    if report is not None:
+        report["excluded_trees"] = int(div.sum())
+    assert div.sum() <= exclusion_budget(B) and div.sum() < B, \
+        "too many diverged trees: %d of %d" % (int(div.sum()), B)
+    for name in ("accept", "path_accept", "corr_tokens"):
+        assert np.array_equal(to_np(gpu[name])[ok], orc[name][ok]), name
+    for name in ("deepest", "accept_len", "bonus"):
+        assert np.array_equal(to_np(gpu[name])[ok], orc[name][ok]), name
+    _close_mask("alpha", to_np(gpu["alpha"])[ok], orc["alpha"][ok], ALPHA_ATOL, 1e-6,
+                np.ones(orc["alpha"][ok].shape, bool))
+    _close_mask("logkappa", to_np(gpu["logkappa"])[ok], orc["logkappa"][ok], LOGK_MARGIN, 1e-6,
+                np.ones(orc["logkappa"][ok].shape, bool))
+    return int(div.sum())
+
+
+def compare_tree_em(gpu, orc, B, N, V, grad_dtype="bf16", report=None):
+    """Parity of the tree EM: a tree where an accept decision, a corrected
+    draw or an o~ comparison went the other way within its margin is
+    excluded (budget); every other tree is compared in full."""
+    m = orc["margins"]  # [B][N][3]: accept, z' draw, o~
+    gz = to_np(gpu["corr_tokens"])
+    gw = to_np(gpu["weights"]).reshape(B, N, 4)
+    ow = orc["weights"]
+    div = np.zeros(B, bool)
+    for b in range(B):
+        bad = np.nonzero(gz[b] != orc["corr_tokens"][b])[0]
+        if bad.size:
+            # z' differs: the draw itself, or an accept decision above it
+            assert (np.minimum(m[b, :, 0], m[b, :, 1]) < PROB_MARGIN).any(), \
+                "tree %d: corrected token differs at %s with no near-boundary decision" % (b, bad[:4])
+            div[b] = True
+            continue
+        bad = np.nonzero(gw[b, :, 0] != ow[b, :, 0])[0]
+        if bad.size:
+            assert (m[b, bad, 2] < LOGK_MARGIN).all(), "tree %d: o~ differs outside the margin" % b
+            div[b] = True
+    ok = ~div
+    SESSION["trees"] += B
+    SESSION["excluded_trees"] += int(div.sum())
+    if report is not None:
+        report["excluded_trees"] = int(div.sum())
+    assert div.sum() <= exclusion_budget(B) and div.sum() < B, \
+        "too many diverged trees: %d of %d" % (int(div.sum()), B)
+    full = np.ones((int(ok.sum()), N), bool)
+    assert np.array_equal(gz[ok], orc["corr_tokens"][ok]), "z'"
+    for name, atol in (("logq_tok", 2e-5), ("logq_corr", 2e-5), ("logkappa", LOGK_MARGIN),
+                       ("logkappa_corr", LOGK_MARGIN), ("logkappa_ref", LOGK_MARGIN)):
+        _close_mask(name, to_np(gpu[name])[ok], orc[name][ok], atol, 1e-6, full)
+    assert np.array_equal(gw[ok][..., 0], ow[ok][..., 0]), "o~"
+    assert np.allclose(gw[ok][..., 1], ow[ok][..., 1], rtol=1e-6, atol=0), "o'"
+    assert np.allclose(gw[ok][..., 2], ow[ok][..., 2], rtol=1e-5, atol=1e-6), "beta"
+    assert np.allclose(gw[ok][..., 3], ow[ok][..., 3], rtol=1e-5, atol=1e-6), "zeta"
+    lg = to_np(gpu["loss"]).astype(np.float64)
+    for b in np.nonzero(ok)[0]:
+        assert abs(lg[b] - orc["loss"][b]) <= LOSS_RTOL * max(1.0, abs(orc["loss"][b])), \
+            "loss[%d] gpu %r oracle %r" % (b, lg[b], orc["loss"][b])
+    if not div.any():
+        assert abs(lg[B] - orc["loss"][B]) <= LOSS_RTOL * max(1.0, abs(orc["loss"][B]))
+    g_all = gpu["grad"]
+    o_all = orc["grad"].reshape(B * N, V)
+    scale = float(np.abs(o_all).max()) if o_all.size else 0.0
+    emax = 0.0
+    for b in np.nonzero(ok)[0]:
+        emax = max(emax, _grad_rows("tree grad", to_np(g_all[b * N:(b + 1) * N]).reshape(N, V),
+                                    o_all[b * N:(b + 1) * N], grad_dtype, scale))
+    if report is not None:
+        report["grad_max_abs_err"] = emax
+    return int(div.sum())
