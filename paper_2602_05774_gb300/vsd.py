@@ -406,7 +406,7 @@ def reference_logkappa(ref_draft, ref_target, B, D, T, workspace=None):
     _check(_lib().vsd_reference_logkappa(_ptr(ref_draft), _ptr(ref_target),
                                          _dtype_code(ref_draft), int(B), int(D), int(V), float(T),
                                          _ptr(out), _ptr(ws), ws.numel(), _stream(dev)),
-           "vsd_reference_logkappa", "vsd_tree_estep_mstep")
+           "vsd_reference_logkappa")
     return out
 
 
