@@ -326,6 +326,19 @@ def lmhead_logits(hidden, weight):
     return h @ w.T
 
 
+def lmhead_backward(grad, hidden, weight):
+    """The LM head's backward (Algorithm 1's M-step carried into the draft
+    head): with logits = hidden . weight^T and G = d loss / d logits,
+    d loss / d hidden = G . weight and d loss / d weight = G^T . hidden, in
+    float64 library matmuls of the exact inputs (no blocking of our own).
+    grad [R, V], hidden [R, H], weight [V, H]; returns (d_hidden, d_weight),
+    with None for the one whose other factor (weight, hidden) is None."""
+    G = np.asarray(grad, dtype=np.float64)
+    d_hidden = None if weight is None else G @ np.asarray(weight, dtype=np.float64)
+    d_weight = None if hidden is None else G.T @ np.asarray(hidden, dtype=np.float64)
+    return d_hidden, d_weight
+
+
 def round_bf16(x):
     """Round float64 values to the nearest bfloat16 (8 significant bits), ties
     to even, returned as float32 holding the bfloat16 value exactly.  Finite

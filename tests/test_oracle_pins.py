@@ -943,3 +943,31 @@ def test_tree_em_of_shared_root_chains_is_the_linear_em(oracle):
         for j in range(1, D):
             assert np.allclose(g[node(s, j)], lin["grad"][s * D + j], atol=1e-14)
         assert np.all(g[node(s, D)] == 0.0)  # a leaf's row carries no term
+
+
+# --------------------------------------------------------------------------
+# The LM head's backward: d hidden = G W, d weight = G^T H.
+
+
+def test_lmhead_backward_one_hot_and_chain_rule(oracle):
+    import torch
+    rng = np.random.default_rng(61)
+    R, V, H = 5, 7, 3
+    h = rng.normal(size=(R, H))
+    w = rng.normal(size=(V, H))
+    # one-hot gradients pick rows and columns: G = e_(r,v) gives d hidden row r
+    # = weight row v and d weight row v = hidden row r
+    for r, v in ((0, 0), (3, 6), (4, 2)):
+        G = np.zeros((R, V))
+        G[r, v] = 1.0
+        dh, dw = oracle.lmhead_backward(G, h, w)
+        assert np.array_equal(dh[r], w[v]) and np.count_nonzero(dh.sum(1)) <= 1
+        assert np.array_equal(dw[v], h[r]) and np.count_nonzero(dw.sum(1)) <= 1
+    # the chain rule through torch's autograd of the forward
+    G = rng.normal(size=(R, V))
+    ht = torch.tensor(h, requires_grad=True)
+    wt = torch.tensor(w, requires_grad=True)
+    (ht @ wt.T).backward(torch.tensor(G))
+    dh, dw = oracle.lmhead_backward(G, h, w)
+    assert np.allclose(dh, ht.grad.numpy(), rtol=1e-13, atol=1e-13)
+    assert np.allclose(dw, wt.grad.numpy(), rtol=1e-13, atol=1e-13)
