@@ -330,6 +330,30 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
                                   vsd_linear_outputs* out, void* ws, size_t ws_bytes,
                                   void* stream);
 
+/* The draft LM head's backward: the M-step's gradient (Algorithm 1, the
+ * gradient of Eq. advance, plus VSD (KL)'s top-K term when params->kl_weight
+ * is nonzero) carried from the draft logits into the head's input and weight:
+ *   d_hidden[R][H] = G . weight        d_weight[V][H] = G^T . hidden
+ * with G[r][v] the gradient with respect to draft_logits[r][v], the bf16 value
+ * the preceding call writes to out->grad with grad_dtype VSD_BF16.  G is not
+ * read from memory: it is made on chip from draft_logits and the row records
+ * and M-step coefficients that call left in `ws`, so this call must follow a
+ * vsd_lmhead_estep_mstep, or a vsd_estep_mstep with dtype VSD_BF16, on the
+ * same draft_logits, layout (linear), T, params->kl_weight and workspace, with
+ * nothing else run on that workspace in between.
+ *   hidden, weight   device, bf16 [R][H] and [V][H], as for the LM head;
+ *   draft_logits     device, bf16 [R][V];
+ *   d_hidden         device, float [R][H], written; NULL to skip;
+ *   d_weight         device, float [V][H], written; NULL to skip.
+ * Products of bf16 values are exact and summed in fp32 on the tensor cores.
+ * H and V must be multiples of 8 and the pointers 16-byte aligned
+ * (VSD_ERR_INVALID_ARG); T >= 0 as given to the preceding call.  A device wait
+ * that runs out sets the timeout bit of the status word of `ws`. */
+vsd_status vsd_lmhead_backward(const void* hidden, const void* weight, int32_t H,
+                               const void* draft_logits, vsd_layout layout, float T,
+                               const vsd_params* params, float* d_hidden, float* d_weight,
+                               void* ws, size_t ws_bytes, void* stream);
+
 /* The greedy reference of Algorithm 2 from its own rows: the oracle's z-bar
  * is drawn from the greedy target policy, so its validity log kappa(z-bar)
  * needs the draft and target distributions along z-bar, which the caller

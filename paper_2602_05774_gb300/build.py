@@ -16,7 +16,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libvsd.so")
 SOURCES = ["vsd_api.cu", "vsd_kernels_f32.cu", "vsd_kernels_bf16.cu", "vsd_noalloc.cu",
-           "vsd_lmhead.cu"]
+           "vsd_lmhead.cu", "vsd_lmhead_bwd.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
 

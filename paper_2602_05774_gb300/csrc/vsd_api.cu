@@ -29,7 +29,7 @@ struct WsLayout {
     size_t status, ticket, prefix_done, grad_head, resq_head, resq_tail, resq_avail;
     size_t path_cnt, prefix_cnt, ready, grad_cnt, row_seg_cnt, res_seg_cnt, resq_flag, zero_end;
     size_t rows, rstats, es_tok, es_corr, es_lq_tok, es_lq_corr, es_lk, es_lkc, es_lkr;
-    size_t coef, wscr, path_A, resq, klr, gtab, tnode, tcoef, tg, tbad, total;
+    size_t coef, wscr, path_A, resq, klr, gtab, tnode, tcoef, tg, tbad, bfac, total;
     int nch_ws, nseg_ws;
 };
 
@@ -120,6 +120,8 @@ WsLayout ws_layout(const vsd_layout& L) {
     w.tcoef = o; o = align256(o + sizeof(TreeCoef) * Rt);
     w.tg = o; o = align256(o + 4 * Rt);
     w.tbad = o; o = align256(o + (L.parent ? 4 * (size_t)L.B : 0));
+    // linear layouts: the rows' packed factors of the LM head's backward
+    w.bfac = o; o = align256(o + (L.parent ? 0 : lmhead_backward_fac_bytes((int)R)));
     w.total = o;
     return w;
 }
@@ -632,6 +634,30 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
     if (e != cudaSuccess) return from_cuda(e);
     return fused_impl<__nv_bfloat16>(draft_logits, target, layout, T, u_draft, u_accept,
                                      u_correct, ref_logkappa, p, out, ws, s, false, true);
+}
+
+vsd_status vsd_lmhead_backward(const void* hidden, const void* weight, int32_t H,
+                               const void* draft_logits, vsd_layout layout, float T,
+                               const vsd_params* params, float* d_hidden, float* d_weight,
+                               void* ws, size_t ws_bytes, void* stream) {
+    if (!layout_ok(layout) || layout.parent) return VSD_ERR_INVALID_ARG;
+    const int64_t R = rows_of(layout);
+    if (R > (1 << 30) || !lmhead_shape_ok(hidden, weight, draft_logits, (int)R, layout.V, H))
+        return VSD_ERR_INVALID_ARG;
+    if (((uintptr_t)d_hidden | (uintptr_t)d_weight) & 15) return VSD_ERR_INVALID_ARG;
+    vsd_status st = check_temperature(T, true);
+    if (st) return st;
+    const vsd_params p = params ? *params : default_params(VSD_BF16);
+    if ((st = check_params(p))) return st;
+    if ((st = check_ws(layout, ws, ws_bytes))) return st;
+    if (!d_hidden && !d_weight) return VSD_OK;
+    const WsLayout w = ws_layout(layout);
+    cudaError_t e = lmhead_backward(
+        hidden, weight, draft_logits, (int)R, layout.V, H, T, at<RowRec>(ws, w.rows),
+        at<Coef>(ws, w.coef), p.kl_weight != 0.0 ? at<KlRec>(ws, w.klr) : nullptr,
+        at<void>(ws, w.bfac), d_hidden, d_weight, at<int>(ws, w.status), p.wait_timeout_ns ? p.wait_timeout_ns : kDefaultTimeoutNs,
+        static_cast<cudaStream_t>(stream));
+    return from_cuda(e);
 }
 
 vsd_status vsd_reference_logkappa(const void* ref_draft, const void* ref_target, vsd_dtype dtype,

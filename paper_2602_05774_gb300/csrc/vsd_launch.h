@@ -67,5 +67,16 @@ bool lmhead_shape_ok(const void* hidden, const void* weight, const void* logits,
 cudaError_t lmhead_gemm(const void* hidden, const void* weight, int M, int N, int K, void* logits,
                         int* status, uint64_t timeout_ns, cudaStream_t s,
                         float4* chunk_tab = nullptr, int chunk_stride = 0, float chunk_c = 0.f);
+// The LM head's backward (vsd_lmhead_bwd.cu): d_hidden = G . weight and
+// d_weight = G^T . hidden (fp32, either may be null), with G the gradient of
+// the bf16 draft logits made on chip from the E-step's row records, M-step
+// coefficients and (klr non-null) top-K terms.
+// fac_scratch: lmhead_backward_fac_bytes(R) bytes of device memory, 16-byte
+// aligned, for the rows' packed factors.
+size_t lmhead_backward_fac_bytes(int R);
+cudaError_t lmhead_backward(const void* hidden, const void* weight, const void* logits, int R,
+                            int V, int H, float T, const RowRec* rows, const Coef* coef,
+                            const KlRec* klr, void* fac_scratch, float* d_hidden,
+                            float* d_weight, int* status, uint64_t timeout_ns, cudaStream_t s);
 
 }  // namespace vsd

@@ -24,7 +24,7 @@ SYMBOLS = ("vsd_workspace_bytes", "vsd_sample_paths", "vsd_verify_paths",
            "vsd_weighted_loss_fwd_bwd", "vsd_estep_mstep", "vsd_device_status",
            "vsd_status_string", "vsd_version", "vsd_estep_mstep_noalloc",
            "vsd_noalloc_device_status", "vsd_lmhead_logits", "vsd_lmhead_estep_mstep",
-           "vsd_reference_logkappa", "vsd_tree_estep_mstep")
+           "vsd_reference_logkappa", "vsd_tree_estep_mstep", "vsd_lmhead_backward")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -108,6 +108,8 @@ def _lib():
         lib.vsd_lmhead_estep_mstep.argtypes = [vp, vp, C.c_int32, vp, Layout, C.c_float, vp, vp,
                                                vp, vp, C.POINTER(Params), vp,
                                                C.POINTER(LinearOutputs), vp, C.c_size_t, vp]
+        lib.vsd_lmhead_backward.argtypes = [vp, vp, C.c_int32, vp, Layout, C.c_float,
+                                            C.POINTER(Params), vp, vp, vp, C.c_size_t, vp]
         lib.vsd_device_status.argtypes = [vp, vp, C.POINTER(C.c_int32)]
         lib.vsd_noalloc_device_status.argtypes = [vp, C.POINTER(C.c_int32)]
         lib.vsd_reference_logkappa.argtypes = [vp, vp, C.c_int, C.c_int32, C.c_int32, C.c_int32,
@@ -122,7 +124,7 @@ def _lib():
                      "vsd_estep_mstep", "vsd_device_status", "vsd_estep_mstep_noalloc",
                      "vsd_noalloc_device_status", "vsd_reference_logkappa",
                      "vsd_tree_estep_mstep",
-                     "vsd_lmhead_logits", "vsd_lmhead_estep_mstep"):
+                     "vsd_lmhead_logits", "vsd_lmhead_estep_mstep", "vsd_lmhead_backward"):
             getattr(lib, name).restype = C.c_int
         _LIB = lib
     return _LIB
@@ -456,6 +458,32 @@ def lmhead_estep_mstep(hidden, weight, target, u_draft, u_accept, u_correct, K, 
                                          _stream(dev)), "vsd_lmhead_estep_mstep")
     out["draft_logits"] = draft_logits
     return out
+
+
+def lmhead_backward(hidden, weight, draft_logits, K, D, T, workspace, prm=None,
+                    d_hidden=True, d_weight=True):
+    """The draft LM head's backward after lmhead_estep_mstep() (or estep_mstep()
+    on bf16 draft logits) on the same workspace: returns {"d_hidden": [R][H],
+    "d_weight": [V][H]} (float32), the M-step gradient of the draft logits
+    carried through logits = hidden . weight^T.  Pass False to skip one, or a
+    float32 tensor to write into."""
+    _need_cuda(hidden, weight, draft_logits)
+    V, H = weight.shape
+    R = hidden.numel() // H
+    lay = layout(R // (K * D), K, D, V)
+    dev = hidden.device
+    prm = prm or params(like=draft_logits)
+    res = {}
+    for name, shape, want in (("d_hidden", (R, H), d_hidden), ("d_weight", (V, H), d_weight)):
+        if want is True:
+            res[name] = torch.empty(*shape, dtype=torch.float32, device=dev)
+        elif want is not False and want is not None:
+            res[name] = want
+    _check(_lib().vsd_lmhead_backward(_ptr(hidden), _ptr(weight), H, _ptr(draft_logits), lay,
+                                      float(T), C.byref(prm), _ptr(res.get("d_hidden")),
+                                      _ptr(res.get("d_weight")), _ptr(workspace),
+                                      workspace.numel(), _stream(dev)), "vsd_lmhead_backward")
+    return res
 
 
 def estep_mstep_noalloc(draft, target, u_draft, u_accept, u_correct, K, D, T,

@@ -128,6 +128,31 @@ def test_lmhead_argument_checks_before_any_launch(vsd):
                                       None, fake, C.byref(o), ws, 1 << 30, None) == 1
 
 
+def test_lmhead_backward_argument_checks_before_any_launch(vsd):
+    lib = vsd.load()
+    fake = C.c_void_p(0x1000)  # never dereferenced: every call below returns before a launch
+    lay = vsd.layout(2, 4, 4, 1024)
+    big = 1 << 30
+    # H a multiple of 8, linear layouts only, outputs 16-byte aligned, T >= 0
+    assert lib.vsd_lmhead_backward(fake, fake, 100, fake, lay, 1.0, None, fake, fake, fake, big,
+                                   None) == 1
+    tlay = vsd.Layout(2, 1, 1, 1024, 60, 0x1000)
+    assert lib.vsd_lmhead_backward(fake, fake, 128, fake, tlay, 1.0, None, fake, fake, fake, big,
+                                   None) == 1
+    assert lib.vsd_lmhead_backward(fake, fake, 128, fake, lay, 1.0, None, C.c_void_p(0x1004),
+                                   fake, fake, big, None) == 1
+    assert lib.vsd_lmhead_backward(fake, fake, 128, fake, lay, -1.0, None, fake, fake, fake, big,
+                                   None) == 1
+    assert lib.vsd_lmhead_backward(None, fake, 128, fake, lay, 1.0, None, fake, fake, fake, big,
+                                   None) == 1
+    # the workspace of the preceding call's layout
+    assert lib.vsd_lmhead_backward(fake, fake, 128, fake, lay, 1.0, None, fake, fake, fake, 256,
+                                   None) == 5
+    # nothing asked for: nothing launched
+    assert lib.vsd_lmhead_backward(fake, fake, 128, fake, lay, 1.0, None, None, None, fake, big,
+                                   None) == 0
+
+
 def test_kl_greedy_and_reference_argument_checks(vsd):
     lib = vsd.load()
     fake = C.c_void_p(0x1000)  # never dereferenced: every call below fails its checks
