@@ -55,7 +55,7 @@ constexpr int kXWarps = VSD_BWD_XWARPS;
 static_assert(kXWarps == 4 || kXWarps == 8 || kXWarps == 16, "a whole share of chunks per thread");
 constexpr int kThreads = 32 * (kXWarps + 6);
 #ifndef VSD_BWD_XGROUPS
-#define VSD_BWD_XGROUPS 2
+#define VSD_BWD_XGROUPS 1
 #endif
 // The transform warps form up to kXGroups groups, so that several stages are
 // made at once.  Stage s belongs to group s % groups: a group makes every
@@ -243,7 +243,8 @@ __device__ __forceinline__ void make_chunk(uint4* cp, const Fac& f, float c, con
             o[e] = *reinterpret_cast<const uint32_t*>(&h);
         }
     } else {
-#pragma unroll 1
+        // (unrolled: constant indices keep w and o in registers)
+#pragma unroll
         for (int e = 0; e < 4; ++e) {
             const int v = v0 + 2 * e;
             const float lo = v < V ? grad_elem(__uint_as_float(w[e] << 16), v, f, c, kl) : 0.f;
@@ -519,7 +520,7 @@ namespace {
 #define VSD_BWD_KB_DH 32
 #endif
 #ifndef VSD_BWD_KB_DW
-#define VSD_BWD_KB_DW 64
+#define VSD_BWD_KB_DW 32
 #endif
 
 template <int MODE, int NT, int KB>
