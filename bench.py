@@ -31,7 +31,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = ("draft-logit rows/s and achieved HBM GB/s (fraction of GB300 roofline) for fused "
           "E/M step")
-WORKLOADS = ("vocab128k", "vocab32k", "tiny", "lmhead", "tree60")
+WORKLOADS = ("vocab128k", "vocab32k", "tiny", "lmhead", "tree60", "lmhead_train")
 
 
 def parse():
@@ -192,7 +192,7 @@ def _cpu_unit(task):
     name, i, T = task
     from paper_2602_05774_gb300 import inputs
     from oracle import oracle
-    c = inputs.CONFIGS[name]
+    c = inputs.CONFIGS["lmhead" if name == "lmhead_train" else name]
     seed = inputs.BASE_SEED + 5000 + i
     if name == "tree60":
         p = inputs.config("tree60", device="cpu", seed=seed, B=1)
@@ -202,15 +202,17 @@ def _cpu_unit(task):
         oracle.tree(f["draft"], f["target"], T, f["parent"], f["tokens"], f["u_accept"],
                     f["u_correct"])
         return time.perf_counter() - t0
-    if name == "lmhead":
+    if name in ("lmhead", "lmhead_train"):
         p = inputs.lmhead_problem(1, c["K"], c["D"], c["V"], c["H"], device="cpu", seed=seed)
         h = p["hidden"].float().numpy()
         w = p["weight"].float().numpy()
         f = {k: p[k].float().numpy() for k in ("target", "u_draft", "u_accept", "u_correct")}
         t0 = time.perf_counter()
         draft = oracle.round_bf16(oracle.lmhead_logits(h, w))
-        oracle.linear(draft, f["target"], T, f["u_draft"], f["u_accept"], f["u_correct"],
-                      c["K"], c["D"])
+        o = oracle.linear(draft, f["target"], T, f["u_draft"], f["u_accept"], f["u_correct"],
+                          c["K"], c["D"])
+        if name == "lmhead_train":  # the head's backward of this prefix's gradient
+            oracle.lmhead_backward(o["grad"], h, w)
         return time.perf_counter() - t0
     p = inputs.linear_problem(1, c["K"], c["D"], c["V"], c["dtype"], _KIND[name], device="cpu",
                               seed=seed)
@@ -228,12 +230,13 @@ def host_cores():
         return os.cpu_count() or 1
 
 
-def cpu_baseline(name, T, rows_per_unit, unit):
+def cpu_baseline(name, T, rows_per_unit, unit, max_workers=None):
     """The oracle single-core (one unit per repetition) and on every host core
-    (one unit per core at once), each the median of three repetitions, in
-    rows/s.  A spawned pool: the GPU context of this process is not forked."""
+    (one unit per core at once; at most max_workers), each the median of three
+    repetitions, in rows/s.  A spawned pool: the GPU context of this process
+    is not forked."""
     import multiprocessing as mp
-    cores = host_cores()
+    cores = host_cores() if max_workers is None else min(host_cores(), max_workers)
     _cpu_unit((name, 0, T))  # builds the oracle and warms the import
     single = [rows_per_unit / _cpu_unit((name, k, T)) for k in range(3)]
     ctx = mp.get_context("spawn")
@@ -450,9 +453,10 @@ def run_ours(args):
 
 
 
-def oracle_lmhead_sample(prob, rows, T):
+def oracle_lmhead_sample(prob, rows, T, train=False):
     """The oracle's LM head (fp64 matmul, one bf16 rounding) and E/M step on the
-    first `rows` rows: seconds."""
+    first `rows` rows (train: and the head's backward of their gradient):
+    seconds."""
     from oracle import oracle
     K, D = prob["K"], prob["D"]
     h = prob["hidden"][:rows].float().cpu().numpy()
@@ -461,14 +465,17 @@ def oracle_lmhead_sample(prob, rows, T):
            ("target", "u_draft", "u_accept", "u_correct")}
     t0 = time.perf_counter()
     draft = oracle.round_bf16(oracle.lmhead_logits(h, w))
-    oracle.linear(draft, sub["target"], T, sub["u_draft"], sub["u_accept"], sub["u_correct"],
-                  min(K, rows // D), D)
+    o = oracle.linear(draft, sub["target"], T, sub["u_draft"], sub["u_accept"], sub["u_correct"],
+                      min(K, rows // D), D)
+    if train:
+        oracle.lmhead_backward(o["grad"], h, w)
     return time.perf_counter() - t0
 
 
-def run_reference_lmhead(args):
+def run_reference_lmhead(args, train=False):
     """The oracle on the host cores for the LM-head workload: each step the LM
-    head and E/M step of one path (D rows) of one prefix."""
+    head and E/M step of one path (D rows) of one prefix (train: and the
+    head's backward)."""
     rank, world, _ = dist_env()
     if rank != 0:
         return
@@ -480,8 +487,8 @@ def run_reference_lmhead(args):
     small = inputs.lmhead_problem(1, K, D, V, H, device="cpu", seed=inputs.BASE_SEED + 99)
     rows = D
     for i in range(args.warmup):
-        oracle_lmhead_sample(small, rows, 1.0)
-    t = sum(oracle_lmhead_sample(small, rows, 1.0) for _ in range(args.steps))
+        oracle_lmhead_sample(small, rows, 1.0, train)
+    t = sum(oracle_lmhead_sample(small, rows, 1.0, train) for _ in range(args.steps))
     ms = t / args.steps * 1e3
     val = rows / (ms / 1e3)
     print(json.dumps({
@@ -489,7 +496,8 @@ def run_reference_lmhead(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded; same recipe)",
-        "config": {"workload": "lmhead", "B": c["B"], "K": K, "D": D, "V": V, "H": H,
+        "config": {"workload": "lmhead_train" if train else "lmhead", "B": c["B"], "K": K,
+                   "D": D, "V": V, "H": H,
                    "sample_per_step": "1 path x %d rows of one prefix" % D},
         "cpu_baseline": {"value": val, "unit": "rows/s", "cores": 1, "kind": "oracle",
                          "sample": "%d rows per step (one path of one prefix)" % rows},
@@ -498,10 +506,13 @@ def run_reference_lmhead(args):
     }), flush=True)
 
 
-def run_lmhead(args):
+def run_lmhead(args, train=False):
     """Config 5: the LM head on the tensor cores fused with the E/M step.  The
     step is vsd_lmhead_estep_mstep; the roofline is the GEMM's (tensor), timed
-    on its own with CUDA events per launch."""
+    on its own with CUDA events per launch.  train: the draft head's training
+    step, vsd_lmhead_estep_mstep with no dense gradient, then
+    vsd_lmhead_backward (d_hidden and d_weight from the factored gradient);
+    the roofline is the backward's (tensor), timed per call."""
     import torch
     rank, world, local = dist_env()
     from paper_2602_05774_gb300 import multirank
@@ -518,13 +529,23 @@ def run_lmhead(args):
     T = 1.0
     prm = vsd.params(like=prob["target"])
     ws = vsd.new_workspace(vsd.layout(B, K, D, V), dev)
-    out = vsd.linear_outputs(B, K, D, V, dev, grad_dtype=torch.bfloat16, full=True)
+    out = vsd.linear_outputs(B, K, D, V, dev, grad_dtype=torch.bfloat16, full=True,
+                             grad=not train)
     dl = torch.empty(R, V, dtype=torch.bfloat16, device=dev)
+    if train:
+        d_hidden = torch.empty(R, H, dtype=torch.float32, device=dev)
+        d_weight = torch.empty(V, H, dtype=torch.float32, device=dev)
+
+    def backward(i):
+        vsd.lmhead_backward(prob["hidden"], prob["weight"], dl, K, D, T, ws, prm=prm,
+                            d_hidden=d_hidden, d_weight=d_weight)
 
     def step(i):
         vsd.lmhead_estep_mstep(prob["hidden"], prob["weight"], prob["target"], prob["u_draft"],
                                prob["u_accept"], prob["u_correct"], K, D, T, prm=prm,
                                workspace=ws, out=out, draft_logits=dl)
+        if train:
+            backward(i)
 
     def barrier():
         multirank.barrier(world, dev)
@@ -552,12 +573,14 @@ def run_lmhead(args):
         raise RuntimeError("device status after warm-up: %s" % (vsd.device_status(ws),))
     with ClockSampler(local) as clk:
         total_ms, _ = timed(step, args.steps)
-        # the GEMM alone, per launch (the roofline's kernel)
         gws = torch.zeros(256, dtype=torch.uint8, device=dev)
-        for _ in range(3):
-            vsd.lmhead_logits(prob["hidden"], prob["weight"], out=dl, workspace=gws)
-        _, gemm_ms = timed(lambda i: vsd.lmhead_logits(prob["hidden"], prob["weight"], out=dl,
-                                                       workspace=gws), args.steps)
+        if train:  # the backward alone, per call (the roofline's kernels)
+            _, gemm_ms = timed(backward, args.steps)
+        else:  # the GEMM alone, per launch (the roofline's kernel)
+            for _ in range(3):
+                vsd.lmhead_logits(prob["hidden"], prob["weight"], out=dl, workspace=gws)
+            _, gemm_ms = timed(lambda i: vsd.lmhead_logits(prob["hidden"], prob["weight"],
+                                                           out=dl, workspace=gws), args.steps)
     total_ms = multirank.max_over_ranks(total_ms, world, dev)
     ms = total_ms / args.steps
     if vsd.device_status(ws)[0] != 0 or vsd.device_status(gws)[0] != 0:
@@ -568,7 +591,7 @@ def run_lmhead(args):
         h_hidden = prob["hidden"].cpu().pin_memory()
         h_target = prob["target"].cpu().pin_memory()
         h_u = torch.stack([prob["u_draft"], prob["u_accept"], prob["u_correct"]]).cpu().pin_memory()
-        hs = vsd.HostLMHeadStep(prob["weight"], B, K, D, V, prm=prm)
+        hs = vsd.HostLMHeadStep(prob["weight"], B, K, D, V, prm=prm, train=train)
         losses = []
 
         def e2e_step(i):
@@ -588,26 +611,36 @@ def run_lmhead(args):
     if rank != 0:
         return
     peak, peak_kind = tensor_peak()
-    flops = 2.0 * R * V * H
+    flops = (4.0 if train else 2.0) * R * V * H
     achieved = flops / (gemm_ms / 1e3) / 1e12
     line = {
         "metric": METRIC, "value": multirank.job_rate(R, world, ms), "unit": "rows/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; hidden ~N(0,1), LM-head weight ~N(0,0.02^2), spiked target)",
-        "config": {"workload": "lmhead", "B": B, "K": K, "D": D, "V": V, "H": H,
-                   "logits": "bf16", "grad": "bf16", "temperatures": [T],
+        "config": {"workload": "lmhead_train" if train else "lmhead", "B": B, "K": K, "D": D,
+                   "V": V, "H": H, "logits": "bf16",
+                   "grad": "factored: made on chip by the backward, never in HBM" if train
+                   else "bf16", "temperatures": [T],
                    "l2": "inputs larger than L2 (no flush)", "rows_per_gpu": R},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
-                     "kernel": "k_lmhead", "flops_per_launch": flops, "launch_ms": gemm_ms},
-        "gpu_launches": 2 * args.steps,
+                     "kernel": "k_lmhead_bwd (d_hidden + d_weight)" if train else "k_lmhead",
+                     "flops_per_launch": flops, "launch_ms": gemm_ms},
+        # per step: GEMM, fused E/M (+ row factors, d_hidden, d_weight)
+        "gpu_launches": (5 if train else 2) * args.steps,
         "clocks": clk.summary(),
     }
     if e2e is not None:
         line["e2e"] = e2e
     if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline("lmhead", T, K * D, "prefix (LM head in fp64 + E/M step)")
+        if train:  # the fp64 V x H product of each unit: four workers at most
+            line["cpu_baseline"] = cpu_baseline(
+                "lmhead_train", T, K * D,
+                "prefix (LM head in fp64 + E/M step + the head's backward)", max_workers=4)
+        else:
+            line["cpu_baseline"] = cpu_baseline("lmhead", T, K * D,
+                                                "prefix (LM head in fp64 + E/M step)")
     print(json.dumps(line), flush=True)
 
 
@@ -777,8 +810,12 @@ def run_tree(args):
 
 def main():
     args = parse()
-    if args.config == "lmhead":
-        run_reference_lmhead(args) if args.impl == "reference" else run_lmhead(args)
+    if args.config in ("lmhead", "lmhead_train"):
+        train = args.config == "lmhead_train"
+        if args.impl == "reference":
+            run_reference_lmhead(args, train)
+        else:
+            run_lmhead(args, train)
     elif args.config == "tree60":
         run_reference_tree(args) if args.impl == "reference" else run_tree(args)
     elif args.impl == "reference":

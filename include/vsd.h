@@ -137,7 +137,9 @@ typedef struct {
                                log q(v) = (x_v - m_q)/T - logZ_q                     */
     float* weights;         /* [B][D][K][4] o~, o', beta, zeta (Alg. 1, Eq. beta/zeta)*/
     float* loss;            /* [B+1] loss_b = -J_b/N_b, then mean over b (Eq. advance)*/
-    void* grad;             /* [R][V] d loss / d draft logits, params.grad_dtype      */
+    void* grad;             /* [R][V] d loss / d draft logits, params.grad_dtype;
+                               NULL (fused calls): not written, the M-step's
+                               coefficients stay in ws for vsd_lmhead_backward */
     float* kl_loss;         /* [R] the row's top-K term of Eq. klv (with kl_weight)   */
 } vsd_linear_outputs;
 
@@ -233,7 +235,9 @@ vsd_status vsd_weighted_loss_fwd_bwd(const void* draft, vsd_dtype dtype, vsd_lay
  * calls: draft, target [R][V] of `dtype`; u_draft, u_accept, u_correct [R];
  * ref_logkappa optional [B][D]; params NULL for the defaults (App. F:
  * w(l) = 1.05^l, tau = 0.2).  Required members of `out`: tokens, accept_len,
- * corr_tokens, logkappa, loss, grad; the rest are optional.  Linear layout
+ * corr_tokens, logkappa, loss; the rest are optional (grad NULL: the dense
+ * gradient is not written, for a vsd_lmhead_backward that makes it on chip
+ * from what the call leaves in ws).  Linear layout
  * only.  Errors: VSD_ERR_INVALID_ARG for a bad shape, pointer, dtype or
  * parameter, VSD_ERR_UNSUPPORTED for T = 0, VSD_ERR_WORKSPACE for a missing
  * or small workspace, VSD_ERR_CUDA if a launch fails; data errors on the

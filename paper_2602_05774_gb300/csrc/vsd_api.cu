@@ -436,6 +436,9 @@ vsd_status fused_impl(const void* draft, const void* target, vsd_layout L, float
     // V=32000 0.107 vs 0.136 ms, V=128256 0.669 vs 0.642 ms.
     P.resq_sem = P.stream_tails;
     P.xtab_given = xtab_given ? 1 : 0;
+    // no dense gradient asked for: no gradient jobs (the M-step's coefficients
+    // stay in the workspace for vsd_lmhead_backward)
+    if (!out->grad) P.gnseg = 0;
     const int64_t tickets = (int64_t)P.R * (P.nseg + P.gnseg);
     int ctas = per_sm * num_sms();
     if ((int64_t)ctas > tickets) ctas = (int)tickets;
@@ -532,8 +535,7 @@ vsd_status vsd_estep_mstep(const void* draft, const void* target, vsd_dtype dtyp
     if (!layout_ok(layout) || layout.parent) return VSD_ERR_INVALID_ARG;
     if (!draft || !target || !u_draft || !u_accept || !u_correct || !out)
         return VSD_ERR_INVALID_ARG;
-    if (!out->tokens || !out->accept_len || !out->corr_tokens || !out->logkappa || !out->loss ||
-        !out->grad)
+    if (!out->tokens || !out->accept_len || !out->corr_tokens || !out->logkappa || !out->loss)
         return VSD_ERR_INVALID_ARG;
     if (dtype != VSD_F32 && dtype != VSD_BF16) return VSD_ERR_INVALID_ARG;
     vsd_status st = check_temperature(T, true);
@@ -609,8 +611,7 @@ vsd_status vsd_lmhead_estep_mstep(const void* hidden, const void* weight, int32_
                                   void* stream) {
     if (!layout_ok(layout) || layout.parent) return VSD_ERR_INVALID_ARG;
     if (!target || !u_draft || !u_accept || !u_correct || !out) return VSD_ERR_INVALID_ARG;
-    if (!out->tokens || !out->accept_len || !out->corr_tokens || !out->logkappa || !out->loss ||
-        !out->grad)
+    if (!out->tokens || !out->accept_len || !out->corr_tokens || !out->logkappa || !out->loss)
         return VSD_ERR_INVALID_ARG;
     const int64_t R = rows_of(layout);
     if (R > (1 << 30) || !lmhead_shape_ok(hidden, weight, draft_logits, (int)R, layout.V, H))

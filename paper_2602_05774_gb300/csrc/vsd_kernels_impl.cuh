@@ -448,9 +448,10 @@ __global__ void __launch_bounds__(kFusedThreads, VSD_FUSED_MIN_BLOCKS)
                         both = false;
                     }
                 }
-                if (both)
+                if (both)  // (with no gradient jobs the draft row is read once)
                     stream_tables<T, VEC, true>(rg, x, P.target + (int64_t)j.r * V, V, j.c0,
-                                                j.c1, rtab, P.ts.c, policy_evict_last(),
+                                                j.c1, rtab, P.ts.c,
+                                                P.gnseg ? policy_evict_last() : policy_evict_first(),
                                                 policy_evict_first(), P.status);
                 if (P.stream_tails) {  // short rows: the tail here, three draws at once
                     asm volatile("bar.sync %0, %1;" ::"r"(kStreamBar), "r"(kThreads) : "memory");

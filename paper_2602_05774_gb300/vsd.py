@@ -373,8 +373,9 @@ def weighted_loss_fwd_bwd(draft, estep, K, D, T, prm=None, workspace=None, grad=
 
 
 def estep_mstep(draft, target, u_draft, u_accept, u_correct, K, D, T, ref_logkappa=None,
-                prm=None, workspace=None, out=None, full=True):
-    """The fused E-step + M-step (one persistent kernel).  Returns the outputs."""
+                prm=None, workspace=None, out=None, full=True, grad=True):
+    """The fused E-step + M-step (one persistent kernel).  Returns the outputs
+    (grad=False: no dense gradient, for lmhead_backward on the same workspace)."""
     _need_cuda(draft, target, u_draft, u_accept, u_correct, ref_logkappa)
     V = draft.shape[-1]
     R = _rows(draft, V)
@@ -385,7 +386,8 @@ def estep_mstep(draft, target, u_draft, u_accept, u_correct, K, D, T, ref_logkap
     prm = prm or params(like=draft)
     if out is None:
         gdt = torch.bfloat16 if prm.grad_dtype == VSD_BF16 else torch.float32
-        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full, kl=prm.kl_weight != 0)
+        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, grad=grad, full=full,
+                             kl=prm.kl_weight != 0)
     st = _linear_struct(out)
     _check(_lib().vsd_estep_mstep(_ptr(draft), _ptr(target), _dtype_code(draft), lay, float(T),
                                   _ptr(u_draft), _ptr(u_accept), _ptr(u_correct),
@@ -433,7 +435,7 @@ def lmhead_logits(hidden, weight, out=None, workspace=None):
 
 def lmhead_estep_mstep(hidden, weight, target, u_draft, u_accept, u_correct, K, D, T,
                        ref_logkappa=None, prm=None, workspace=None, out=None, draft_logits=None,
-                       full=True):
+                       full=True, grad=True):
     """The LM head, then the fused E-step + M-step on its logits.  Returns the
     outputs of estep_mstep() plus "draft_logits"."""
     _need_cuda(hidden, weight, target, u_draft, u_accept, u_correct, ref_logkappa)
@@ -449,7 +451,8 @@ def lmhead_estep_mstep(hidden, weight, target, u_draft, u_accept, u_correct, K, 
         draft_logits = torch.empty(R, V, dtype=torch.bfloat16, device=dev)
     if out is None:
         gdt = torch.bfloat16 if prm.grad_dtype == VSD_BF16 else torch.float32
-        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, full=full, kl=prm.kl_weight != 0)
+        out = linear_outputs(B, K, D, V, dev, grad_dtype=gdt, grad=grad, full=full,
+                             kl=prm.kl_weight != 0)
     st = _linear_struct(out)
     _check(_lib().vsd_lmhead_estep_mstep(_ptr(hidden), _ptr(weight), H, _ptr(target), lay,
                                          float(T), _ptr(u_draft), _ptr(u_accept),
@@ -608,9 +611,11 @@ class HostStep:
 class HostLMHeadStep:
     """HostStep for the LM head fused with the E-step + M-step: per call the
     hidden states, target logits and uniforms come from pinned host tensors
-    (double-buffered); the LM-head weight stays on the device."""
+    (double-buffered); the LM-head weight stays on the device.  train=True:
+    the draft head's training step, no dense gradient and the LM head's
+    backward (d_hidden, d_weight left on the device)."""
 
-    def __init__(self, weight, B, K, D, V, prm=None, full=True):
+    def __init__(self, weight, B, K, D, V, prm=None, full=True, train=False):
         self.B, self.K, self.D, self.V = B, K, D, V
         R, H = B * K * D, weight.shape[1]
         self.dev = weight.device
@@ -619,9 +624,13 @@ class HostLMHeadStep:
                                  u=((3, R), torch.float32)), self.dev)
         self.prm = prm or params(grad_dtype=torch.bfloat16)
         gdt = torch.bfloat16 if self.prm.grad_dtype == VSD_BF16 else torch.float32
-        self.out = linear_outputs(B, K, D, V, self.dev, grad_dtype=gdt, full=full)
+        self.train = train
+        self.out = linear_outputs(B, K, D, V, self.dev, grad_dtype=gdt, full=full, grad=not train)
         self.ws = new_workspace(layout(B, K, D, V), self.dev)
         self.logits = torch.empty(R, V, dtype=torch.bfloat16, device=self.dev)
+        if train:
+            self.d_hidden = torch.empty(R, H, dtype=torch.float32, device=self.dev)
+            self.d_weight = torch.empty(V, H, dtype=torch.float32, device=self.dev)
         self.loss_host = [torch.empty(B + 1, dtype=torch.float32).pin_memory() for _ in range(2)]
 
     def h2d_bytes(self):
@@ -635,6 +644,9 @@ class HostLMHeadStep:
         lmhead_estep_mstep(d["hidden"], self.weight, d["target"], d["u"][0], d["u"][1],
                            d["u"][2], self.K, self.D, T, prm=self.prm, workspace=self.ws,
                            out=self.out, draft_logits=self.logits)
+        if self.train:
+            lmhead_backward(d["hidden"], self.weight, self.logits, self.K, self.D, T, self.ws,
+                            prm=self.prm, d_hidden=self.d_hidden, d_weight=self.d_weight)
         self.feed.release(s)
         self.loss_host[s].copy_(self.out["loss"], non_blocking=True)
         return self.loss_host[s]

@@ -22,7 +22,7 @@ def _run(args, timeout=240):
     return [l for l in r.stdout.splitlines() if l.startswith("{")]
 
 
-@pytest.mark.parametrize("config", ["vocab128k", "tree60", "lmhead"])
+@pytest.mark.parametrize("config", ["vocab128k", "tree60", "lmhead", "lmhead_train"])
 def test_reference_arm_json_line(config):
     lines = _run(["bench.py", "--impl", "reference", "--config", config, "--steps", "1",
                   "--warmup", "1"])

@@ -94,3 +94,33 @@ def test_host_tree_step_overlapped_calls(vsd):
     for i, g in enumerate(got):
         for k in keys:
             assert torch.equal(g[k], want[i % 2][k]), (i, k)
+
+
+def test_host_lmhead_training_step_overlapped_calls(vsd):
+    """train=True: the draft head's training step from pinned host buffers (no
+    dense gradient, then the backward) gives, call after call, the
+    d_hidden / d_weight of the same calls made directly on device tensors."""
+    from paper_2602_05774_gb300 import inputs
+    B, K, D, V, H, T = 2, 4, 4, 4096, 256, 1.0
+    probs = [inputs.lmhead_exact_problem(B, K, D, V, H, device="cpu", seed=s) for s in (8, 9)]
+    weight = probs[0]["weight"].cuda()
+    prm = vsd.params(grad_dtype=torch.bfloat16)
+    want = []
+    for p in probs:
+        c = {k: (v.cuda() if torch.is_tensor(v) else v) for k, v in p.items()}
+        ws = vsd.new_workspace(vsd.layout(B, K, D, V), "cuda")
+        o = vsd.lmhead_estep_mstep(c["hidden"], weight, c["target"], c["u_draft"], c["u_accept"],
+                                   c["u_correct"], K, D, T, prm=prm, workspace=ws, grad=False)
+        b = vsd.lmhead_backward(c["hidden"], weight, o["draft_logits"], K, D, T, ws, prm=prm)
+        want.append((o["loss"].clone(), b["d_hidden"].clone(), b["d_weight"].clone()))
+    host = [(p["hidden"].pin_memory(), p["target"].pin_memory(), _u(p).pin_memory()) for p in probs]
+    hs = vsd.HostLMHeadStep(weight, B, K, D, V, prm=prm, train=True)
+    got = []
+    for i in range(5):
+        hs(*host[i % 2], T)
+        got.append((hs.out["loss"].clone(), hs.d_hidden.clone(), hs.d_weight.clone()))
+    torch.cuda.synchronize()
+    assert vsd.device_status(hs.ws) == (0, 0)
+    for i, g in enumerate(got):
+        for a, b in zip(g, want[i % 2]):
+            assert torch.equal(a, b), i

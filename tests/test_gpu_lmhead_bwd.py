@@ -264,3 +264,31 @@ def test_full_size_sampled(vsd, oracle):
     cols = torch.tensor([0, 1, 255, 256, 17000, 31998, 31999], device="cuda")
     Gc = _np(fw["grad"][:, cols]).T  # [7][R]
     _check_bound(Gc, _np(p["hidden"]), _np(bw["d_weight"][cols]), "d_weight")
+
+
+@pytest.mark.parametrize("kl_weight", [0.0, 0.5])
+def test_factored_step_without_dense_gradient(vsd, kl_weight):
+    """The training step that never writes the dense gradient: the fused call
+    with no grad output, then the backward from what it left in the
+    workspace.  Every output equals the one of the step that writes the
+    gradient, bit for bit."""
+    B, K, D, V, H = 3, 5, 4, 4104, 264
+    p = _problem(B, K, D, V, H, "gauss", 808)
+    prm = vsd.params(like=p["target"], kl_weight=kl_weight)
+    res = []
+    for grad in (True, False):
+        ws = vsd.new_workspace(vsd.layout(B, K, D, V), "cuda")
+        fw = vsd.lmhead_estep_mstep(p["hidden"], p["weight"], p["target"], p["u_draft"],
+                                    p["u_accept"], p["u_correct"], K, D, 1.0, prm=prm,
+                                    workspace=ws, grad=grad)
+        bw = vsd.lmhead_backward(p["hidden"], p["weight"], fw["draft_logits"], K, D, 1.0, ws,
+                                 prm=prm)
+        torch.cuda.synchronize()
+        assert vsd.device_status(ws) == (0, 0)
+        assert ("grad" in fw) == grad
+        res.append((fw, bw))
+    (f1, b1), (f2, b2) = res
+    for name in f2:
+        assert torch.equal(f1[name], f2[name]), name
+    assert torch.equal(b1["d_hidden"], b2["d_hidden"])
+    assert torch.equal(b1["d_weight"], b2["d_weight"])
