@@ -146,6 +146,39 @@ __device__ __forceinline__ uint64_t sdesc_sw64(uint32_t saddr) {
     return d;
 }
 
+// The persistent loop's work, segments (tile t, K blocks kb0 .. kb1 - 1).
+// Tile mode: whole tiles blockIdx.x, blockIdx.x + gridDim.x, ...  Stream-K
+// mode: the units (tile, K block) in tile order are shared out evenly, CTA c
+// taking units [c U / G, (c + 1) U / G); a share is at least one tile long,
+// so at most two CTAs meet on a tile and add into the zeroed output.
+struct Seg {
+    int t, kb0, kb1;
+};
+template <bool SK> struct SegIter {
+    long long u, u1;  // stream-K: the next unit and the end of this CTA's share
+    int t, nk, ntiles;
+    __device__ SegIter(int ntiles_, int nk_) : nk(nk_), ntiles(ntiles_) {
+        const long long U = (long long)ntiles_ * nk_;
+        u = SK ? U * blockIdx.x / gridDim.x : 0;
+        u1 = SK ? U * (blockIdx.x + 1) / gridDim.x : 0;
+        t = blockIdx.x;
+    }
+    __device__ bool next(Seg& g) {
+        if (!SK) {
+            if (t >= ntiles) return false;
+            g = Seg{t, 0, nk};
+            t += gridDim.x;
+            return true;
+        }
+        if (u >= u1) return false;
+        g.t = (int)(u / nk);
+        g.kb0 = (int)(u - (long long)g.t * nk);
+        g.kb1 = (int)min((long long)nk, u1 - (long long)g.t * nk);
+        u = (long long)g.t * nk + g.kb1;
+        return true;
+    }
+};
+
 #ifndef VSD_BWD_NFAST
 #define VSD_BWD_NFAST 1
 #endif
@@ -264,7 +297,7 @@ __device__ __forceinline__ void make_chunk(uint4* cp, const Fac& f, float c, con
 // MODE kDWeight: out[V][H] = G^T . hidden.  The A tile is x[k0 .. k0+KB)[m0 ..
 // m0+127] read MN-major (two 64-column boxes); B is hidden[k0 .. k0+KB)[n0 ..)
 // read MN-major like W above.
-template <int MODE, int NT, int KB>
+template <int MODE, int NT, int KB, bool SK>
 __global__ void __launch_bounds__(kThreads, 1)
     k_lmhead_bwd(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmB,
                  const Fac* __restrict__ fac, const KlRec* __restrict__ klr, float c, int R,
@@ -315,11 +348,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             uint32_t it = 0;
             bool ok = true;
-            for (int t = blockIdx.x; ok && t < ntiles && !*(volatile int*)&sb->err;
-                 t += gridDim.x) {
+            SegIter<SK> si(ntiles, nk);
+            Seg sg;
+            while (ok && !*(volatile int*)&sb->err && si.next(sg)) {
                 int m0, n0;
-                tile_origin(t, mt, ntn, TN, m0, n0);
-                for (int kb = 0; kb < nk; ++kb) {
+                tile_origin(sg.t, mt, ntn, TN, m0, n0);
+                for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
                     const int s = (int)(it % S);
                     const uint32_t round = it / S;
                     if (round > 0 && !wait_phase(&sb->empty[s], (round - 1) & 1u, sb, status)) {
@@ -356,14 +390,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t it = 0;
             int lt = 0;
             bool ok = true;
-            for (int t = blockIdx.x; ok && t < ntiles && !*(volatile int*)&sb->err;
-                 t += gridDim.x, ++lt) {
+            SegIter<SK> si(ntiles, nk);
+            Seg sg;
+            for (; ok && !*(volatile int*)&sb->err && si.next(sg); ++lt) {
                 const int buf = C::kAccBufs == 2 ? (lt & 1) : 0;
                 const uint32_t use = C::kAccBufs == 2 ? ((uint32_t)lt >> 1) : (uint32_t)lt;
                 if (use > 0 && !wait_phase(&sb->acc_empty[buf], (use - 1) & 1u, sb, status)) break;
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(buf * BN);
-                for (int kb = 0; kb < nk; ++kb) {
+                for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
                     const int s = (int)(it % S);
                     if (!wait_phase(&sb->xform[s], (it / S) & 1u, sb, status)) {
                         ok = false;
@@ -386,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int i = 0; i < NT; ++i)
                             mma_bf16(d + (uint32_t)(i * BN), ad,
                                      sdesc_mn_sw128(b + (uint32_t)(i * 4 * kBox) + 2048u * k, kBox),
-                                     kIdesc, (kb | k) != 0 ? 1u : 0u);
+                                     kIdesc, (kb != sg.kb0 || k != 0) ? 1u : 0u);
                     }
                     mma_commit(&sb->empty[s]);
                     ++it;
@@ -418,9 +453,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int sw = (MODE == kDHidden && KB == 32) ? ((rl >> 1) & 3) : (rl & 7);
         uint32_t it = 0;
         bool ok = true;
-        for (int t = blockIdx.x; ok && t < ntiles && !*(volatile int*)&sb->err; t += gridDim.x) {
+        SegIter<SK> si(ntiles, nk);
+        Seg sg;
+        while (ok && !*(volatile int*)&sb->err && si.next(sg)) {
             int m0, n0;
-            tile_origin(t, mt, ntn, TN, m0, n0);
+            tile_origin(sg.t, mt, ntn, TN, m0, n0);
             Fac f = no_row();
             const KlRec* kl = nullptr;
             if (MODE == kDHidden && m0 + rl < R) {
@@ -428,7 +465,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (klr) kl = klr + (m0 + rl);
                 if (!kl) f.nkl = 0;
             }
-            for (int kb = 0; kb < nk; ++kb, ++it) {
+            for (int kb = sg.kb0; kb < sg.kb1; ++kb, ++it) {
                 const int s = (int)(it % S);
                 if (s % C::kGroups != xg) continue;  // another group's stage
                 const int k0 = kb * KB;
@@ -469,13 +506,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------ epilogue
         const int q = warp & 3;  // TMEM lanes 32q .. 32q + 31
         int lt = 0;
-        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++lt) {
+        SegIter<SK> si(ntiles, nk);
+        Seg sg;
+        for (; si.next(sg); ++lt) {
             const int buf = C::kAccBufs == 2 ? (lt & 1) : 0;
             const uint32_t use = C::kAccBufs == 2 ? ((uint32_t)lt >> 1) : (uint32_t)lt;
             if (!wait_phase(&sb->acc_full[buf], use & 1u, sb, status)) break;
             tc_fence_after();
             int m0, n0;
-            tile_origin(t, mt, ntn, TN, m0, n0);
+            tile_origin(sg.t, mt, ntn, TN, m0, n0);
+            // a tile this CTA holds in part: added into the zeroed output
+            const bool part = SK && (sg.kb0 != 0 || sg.kb1 != nk);
             const int row = m0 + 32 * q + lane;
             const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * BN);
 #pragma unroll 1
@@ -487,10 +528,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                     float* o = out + (size_t)row * H + col;
 #pragma unroll
                     for (int v4 = 0; v4 < 8; ++v4)
-                        if (col + 4 * v4 < H)
-                            *reinterpret_cast<uint4*>(o + 4 * v4) =
-                                make_uint4(rg[4 * v4], rg[4 * v4 + 1], rg[4 * v4 + 2],
-                                           rg[4 * v4 + 3]);
+                        if (col + 4 * v4 < H) {
+                            if (part)
+                                atomicAdd(reinterpret_cast<float4*>(o + 4 * v4),
+                                          make_float4(__uint_as_float(rg[4 * v4]),
+                                                      __uint_as_float(rg[4 * v4 + 1]),
+                                                      __uint_as_float(rg[4 * v4 + 2]),
+                                                      __uint_as_float(rg[4 * v4 + 3])));
+                            else
+                                *reinterpret_cast<uint4*>(o + 4 * v4) =
+                                    make_uint4(rg[4 * v4], rg[4 * v4 + 1], rg[4 * v4 + 2],
+                                               rg[4 * v4 + 3]);
+                        }
                 }
             }
             tc_fence_before();
@@ -516,6 +565,9 @@ namespace {
 #ifndef VSD_BWD_NT
 #define VSD_BWD_NT 2
 #endif
+#ifndef VSD_BWD_STREAM_K
+#define VSD_BWD_STREAM_K 1
+#endif
 #ifndef VSD_BWD_KB_DH
 #define VSD_BWD_KB_DH 32
 #endif
@@ -537,15 +589,24 @@ cudaError_t launch_bwd(const void* logits, const void* bmat, int brows, const vs
                          : make_map_box(&tx, logits, R, V, 64, KB, 128);
     // B: W [V][H] or hidden [R][H], 64-column boxes of KB rows
     if (!okx || !make_map_box(&tb, bmat, brows, H, 64, KB, 128)) return cudaErrorInvalidValue;
-    auto kern = vsd_bwd::k_lmhead_bwd<MODE, NT, KB>;
     const size_t smem = vsd_bwd::smem_bytes<MODE, NT, KB>();
-    cudaError_t e = ensure_dyn_smem((const void*)kern, smem);
-    if (e != cudaSuccess) return e;
     constexpr int BM = vsd_bwd::BM, TN = vsd_bwd::BN * NT;
     const int M = MODE == vsd_bwd::kDHidden ? R : V;
     const long long tiles = (long long)((M + BM - 1) / BM) * ((H + TN - 1) / TN);
     const int sms = device_sm_count();
     const int grid = (int)(tiles < sms ? tiles : sms);
+    // Stream-K when whole tiles would leave more than a tenth of the SM time
+    // idle (and there are more tiles than SMs, so a share is at least a
+    // tile): the output is zeroed first, which costs less than that idle time
+    // at these sizes.
+    const long long slots = (tiles + sms - 1) / sms * sms;
+    const bool sk = VSD_BWD_STREAM_K && tiles > sms && (slots - tiles) * 10 > slots;
+    auto kern = sk ? vsd_bwd::k_lmhead_bwd<MODE, NT, KB, true>
+                   : vsd_bwd::k_lmhead_bwd<MODE, NT, KB, false>;
+    cudaError_t e = ensure_dyn_smem((const void*)kern, smem);
+    if (e != cudaSuccess) return e;
+    if (sk && (e = cudaMemsetAsync(out, 0, (size_t)M * H * sizeof(float), s)) != cudaSuccess)
+        return e;
     kern<<<grid, vsd_bwd::kThreads, smem, s>>>(tx, tb, fac, klr, c, R, V, H, out, status,
                                                timeout_ns);
     return cudaGetLastError();

@@ -292,3 +292,25 @@ def test_factored_step_without_dense_gradient(vsd, kl_weight):
         assert torch.equal(f1[name], f2[name]), name
     assert torch.equal(b1["d_hidden"], b2["d_hidden"])
     assert torch.equal(b1["d_weight"], b2["d_weight"])
+
+
+def test_d_hidden_exactly_with_stream_k(vsd):
+    """160 output tiles of 128 x 512 on the GPU's SMs: d_hidden is shared out
+    by stream-K (tiles split between two CTAs and added into the zeroed
+    output).  With W the identity it is still the written gradient bit for
+    bit, and two calls give the same bits."""
+    B, K, D, V, H = 64, 8, 8, 2560, 2560
+    p = _problem(B, K, D, V, H, "dh_exact", 4321)
+    fw, bw = _run(vsd, p, K, D, 1.0)
+    G = fw["grad"].float()
+    assert torch.equal(bw["d_hidden"][:, :V], G)
+    ws = vsd.new_workspace(vsd.layout(B, K, D, V), "cuda")
+    fw2 = vsd.lmhead_estep_mstep(p["hidden"], p["weight"], p["target"], p["u_draft"],
+                                 p["u_accept"], p["u_correct"], K, D, 1.0, workspace=ws)
+    a = vsd.lmhead_backward(p["hidden"], p["weight"], fw2["draft_logits"], K, D, 1.0, ws,
+                            d_weight=False)
+    b = vsd.lmhead_backward(p["hidden"], p["weight"], fw2["draft_logits"], K, D, 1.0, ws,
+                            d_weight=False)
+    torch.cuda.synchronize()
+    assert torch.equal(a["d_hidden"], b["d_hidden"])
+    assert torch.equal(a["d_hidden"], bw["d_hidden"])
