@@ -90,10 +90,11 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(workload):
-    """DRAM bytes per launch of the fused kernel from the committed ncu summary,
-    if it was taken on the current kernel sources; else None."""
-    path = os.path.join(ROOT, "profiles", "k_fused_%s_traffic.json" % workload)
+def ncu_traffic(workload, kernel="k_fused"):
+    """DRAM bytes per launch of the roofline's kernel (k_fused; k_lmhead_bwd:
+    per backward call) from the committed ncu summary, if it was taken on the
+    current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "%s_%s_traffic.json" % (kernel, workload))
     try:
         d = json.load(open(path))
         if d.get("kernel_source_hash") == kernel_source_hash():
@@ -624,7 +625,9 @@ def run_lmhead(args, train=False):
                    else "bf16", "temperatures": [T],
                    "l2": "inputs larger than L2 (no flush)", "rows_per_gpu": R},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
+                     "frac": achieved / peak,
+                     "traffic": ncu_traffic("lmhead_train", "k_lmhead_bwd") if train else None,
+                     "peak_kind": peak_kind,
                      "kernel": "k_lmhead_bwd (d_hidden + d_weight)" if train else "k_lmhead",
                      "flops_per_launch": flops, "launch_ms": gemm_ms},
         # per step: GEMM, fused E/M (+ row factors, d_hidden, d_weight)
