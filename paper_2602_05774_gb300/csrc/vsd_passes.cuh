@@ -1581,13 +1581,19 @@ __device__ void weights_warp(const Problem<T>& P, const EStepView& E, int b, flo
         const int nd = min(dt, D - d0);
         const int ne = K * nd;
         mstep_tile<T, false>(P, E, b, d0, nd, sh, lane);
-        // running sums of log q over l, per proposal
+        // running sums of log q over l, per proposal: the fixed-point terms
+        // for every entry at once, then integer adds along l
+        each_entry(ne, lane, [&](int e) {
+            sh.elqt[e] = to_fixed(sh.lq[e], kLqE);
+            sh.elqc[e] = to_fixed(sh.lqcz[e], kLqE);
+        });
+        __syncwarp();
         for (int s = lane; s < K; s += 32) {
             long long a = sh.lqt[s], q = sh.lqc[s];
             for (int dd = 0; dd < nd; ++dd) {
                 const int e = s * nd + dd;
-                a += to_fixed(sh.lq[e], kLqE);
-                q += to_fixed(sh.lqcz[e], kLqE);
+                a += sh.elqt[e];
+                q += sh.elqc[e];
                 sh.elqt[e] = a;
                 sh.elqc[e] = q;
             }
@@ -1685,31 +1691,40 @@ __device__ void weights_warp(const Problem<T>& P, const EStepView& E, int b, flo
             __syncwarp();
             mstep_tile<T, true>(P, E, b, d0, nd, sh, lane);
         }
+        // integer adds along l from the end, then every entry's coefficients
+        // at once
         for (int s = lane; s < K; s += 32) {
             long long c0 = sh.lqt[s], c1 = sh.lqc[s];
             for (int dd = nd - 1; dd >= 0; --dd) {
                 const int e = s * nd + dd;
                 c0 += sh.et0[e];
                 c1 += sh.elqc[e];
-                Coef cf;
-                cf.t0 = sh.tok[e];
-                cf.t1 = sh.corr[e];
-                const float g = from_fixed(c0 + c1, kLqE) * scale;
-                if (cf.t1 == cf.t0) {
-                    cf.c0 = g;
-                    cf.c1 = 0.f;
-                    cf.t1 = -1;
-                } else {
-                    cf.c0 = from_fixed(c0, kLqE) * scale;
-                    cf.c1 = from_fixed(c1, kLqE) * scale;
-                }
-                cf.g = g;
-                cf.pad0 = cf.pad1 = cf.pad2 = 0.f;
-                P.coef[(b * K + s) * D + d0 + dd] = cf;
+                sh.et0[e] = c0;
+                sh.elqc[e] = c1;
             }
             sh.lqt[s] = c0;
             sh.lqc[s] = c1;
         }
+        __syncwarp();
+        each_entry(K * nd, lane, [&](int e) {
+            const int s = e / nd, dd = e - s * nd;
+            const long long c0 = sh.et0[e], c1 = sh.elqc[e];
+            Coef cf;
+            cf.t0 = sh.tok[e];
+            cf.t1 = sh.corr[e];
+            const float g = from_fixed(c0 + c1, kLqE) * scale;
+            if (cf.t1 == cf.t0) {
+                cf.c0 = g;
+                cf.c1 = 0.f;
+                cf.t1 = -1;
+            } else {
+                cf.c0 = from_fixed(c0, kLqE) * scale;
+                cf.c1 = from_fixed(c1, kLqE) * scale;
+            }
+            cf.g = g;
+            cf.pad0 = cf.pad1 = cf.pad2 = 0.f;
+            P.coef[(b * K + s) * D + d0 + dd] = cf;
+        });
     }
     float klterm = 0.f;
     if (P.kl_topk) {  // VSD (KL): + kl_weight (1/K) sum of the prefix's rows' top-K terms
