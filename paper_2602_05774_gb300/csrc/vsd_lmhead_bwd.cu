@@ -19,17 +19,23 @@
 // W and hidden are read as they lie, as MN-major B operands (no transposes),
 // and so is the logits tile of d_weight as an MN-major A operand.
 //
-// One persistent CTA per SM computes 128 x (256 NT) output tiles, K in blocks
-// of 64 through a shared-memory ring:
-//   warp 0     TMA producer: the logits tile and the B tile of each K block
-//              (128-byte swizzle);
-//   warp 1     MMA issuer: one thread issues tcgen05.mma (kind::f16, M = 128,
-//              N = 256, K = 16; NT of them per K step, sharing A) into TMEM;
-//   warps 2-5  transform: the logits tile becomes the A operand in place;
-//   warps 6-9  epilogue: tcgen05.ld of the accumulator, fp32 stores.
-// Every wait is bounded; a wait that runs out sets VSD_STATUS_TIMEOUT in the
-// status word and the CTA winds down (waiting, again bounded, for its copies
-// and MMAs in flight) and frees its tensor memory.
+// One persistent CTA per SM computes 128 x (256 NT) output tiles (NT = 2: a
+// tile fills the 512 TMEM columns), K in blocks of KB (32) through a ring of
+// shared-memory stages:
+//   warp 0          TMA producer: the logits tile and the B tile of each K
+//                   block (for d_weight also the block's row factors);
+//   warp 1          MMA issuer: one thread issues tcgen05.mma (kind::f16,
+//                   M = 128, N = 256, K = 16; NT of them per K step, sharing
+//                   A) into TMEM;
+//   warps 2 .. 17   transform: the logits tile becomes the A operand in place;
+//   the last 4      epilogue: tcgen05.ld of the accumulator, fp32 stores.
+// d_hidden's 256 tiles at the lmhead sizes would leave a third of the SMs
+// idle in a second wave, so there the (tile, K block) units are shared out
+// evenly (stream-K) and tiles split between two CTAs are added into the
+// zeroed output.  Every wait is bounded; a wait that runs out sets
+// VSD_STATUS_TIMEOUT in the status word and the CTA winds down (waiting,
+// again bounded, for its copies and MMAs in flight) and frees its tensor
+// memory.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
