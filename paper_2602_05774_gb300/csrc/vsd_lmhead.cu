@@ -72,6 +72,13 @@ __device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity, Bars*
                                            int* status) {
     return wait_phase_err(bar, parity, &sb->err, sb->timeout_ns, status);
 }
+// The same wait by a whole warp, with one outcome for all its lanes (a lane
+// that gave up while another saw the phase complete would split the warp
+// between the loop's __syncwarp and the final __syncthreads).
+__device__ __forceinline__ bool wait_phase_warp(uint64_t* bar, uint32_t parity, Bars* sb,
+                                                int* status) {
+    return __all_sync(0xffffffffu, wait_phase(bar, parity, sb, status));
+}
 
 // Work is cut into units of one 128-row M tile by one 1024-column chunk (the
 // E-step's chunk of bf16 logits): kTilesPerChunk consecutive 128 x 256 tiles,
@@ -212,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int nt = nt0; nt < nt1; ++nt, ++lt) {
                 const int buf = lt & 1;
                 const uint32_t use = (uint32_t)lt >> 1;
-                if (!wait_phase(&sb->acc_full[buf], use & 1u, sb, status)) {
+                if (!wait_phase_warp(&sb->acc_full[buf], use & 1u, sb, status)) {
                     ok = false;
                     break;
                 }

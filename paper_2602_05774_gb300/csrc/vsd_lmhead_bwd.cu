@@ -123,6 +123,13 @@ template <int MODE, int NT, int KB> constexpr size_t smem_bytes() {
 __device__ __forceinline__ bool wait_phase(uint64_t* bar, uint32_t parity, Bars* sb, int* status) {
     return wait_phase_err(bar, parity, &sb->err, sb->timeout_ns, status);
 }
+// The same wait by a whole warp, with one outcome for all its lanes (a lane
+// that gave up while another saw the phase complete would split the warp
+// between the loop's __syncwarp and the final __syncthreads).
+__device__ __forceinline__ bool wait_phase_warp(uint64_t* bar, uint32_t parity, Bars* sb,
+                                                int* status) {
+    return __all_sync(0xffffffffu, wait_phase(bar, parity, sb, status));
+}
 
 // Shared-memory descriptor of an MN-major bf16 operand in the 128-byte
 // swizzle: 8-row K groups of 128-byte rows (64 MN elements) 1024 bytes apart
@@ -479,7 +486,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 uint4* rowp;
                 int vb;
                 uint32_t slow = 0;
-                if (!wait_phase(&sb->full[s], (it / S) & 1u, sb, status)) {
+                if (!wait_phase_warp(&sb->full[s], (it / S) & 1u, sb, status)) {
                     ok = false;
                     break;
                 }
@@ -517,7 +524,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (; si.next(sg); ++lt) {
             const int buf = C::kAccBufs == 2 ? (lt & 1) : 0;
             const uint32_t use = C::kAccBufs == 2 ? ((uint32_t)lt >> 1) : (uint32_t)lt;
-            if (!wait_phase(&sb->acc_full[buf], use & 1u, sb, status)) break;
+            if (!wait_phase_warp(&sb->acc_full[buf], use & 1u, sb, status)) break;
             tc_fence_after();
             int m0, n0;
             tile_origin(sg.t, mt, ntn, TN, m0, n0);
